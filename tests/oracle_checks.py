@@ -1,0 +1,338 @@
+"""Checks that pin the fp64 oracle to something other than itself.
+
+Each ``check_*`` takes the implementation under test (normally the oracle's
+own function) and raises AssertionError when it disagrees with a hand-derived
+fixture, a library special case, an exact brute force or an invariant.  The
+mutation tests hand these checks deliberately broken copies of the oracle
+and require at least one check to fail, so a plausible slip (a dropped
+term, a wrong index, a wrong sign) cannot pass unnoticed.
+"""
+import itertools
+import math
+import os
+
+import numpy as np
+import torch
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _nums(s):
+    return [float(x) for x in s.split()]
+
+
+def _rows(s):
+    return np.array([_nums(r) for r in s.split("|")], dtype=np.float64)
+
+
+def read_kv(name):
+    out = {}
+    for line in open(os.path.join(GOLDEN, name)):
+        line = line.strip()
+        if not line or line.startswith("#"):
+            continue
+        k, v = line.split(":", 1)
+        out[k.strip()] = v.strip()
+    return out
+
+
+# ----------------------------------------------------------------------------
+# attention
+# ----------------------------------------------------------------------------
+def _sdpa(q, k, v, mask, scale):
+    """torch's scaled_dot_product_attention in float64 on the CPU:
+    q [Hq, M, D], k/v [Hq, S, D], mask [M, S] bool (True = attend)."""
+    with torch.no_grad():
+        o = torch.nn.functional.scaled_dot_product_attention(
+            torch.from_numpy(q)[None], torch.from_numpy(k)[None],
+            torch.from_numpy(v)[None], attn_mask=torch.from_numpy(mask),
+            scale=scale)
+    return o[0].numpy()
+
+
+def _expand_gqa(x, G):
+    """[Hkv, S, D] -> [Hkv*G, S, D], query head h uses KV head h // G."""
+    return np.repeat(x, G, axis=0)
+
+
+def _random_attention_case(rng, N, P, Hq, Hkv, D, parent):
+    q = rng.standard_normal((N, Hq, D))
+    pk = rng.standard_normal((Hkv, P, D))
+    pv = rng.standard_normal((Hkv, P, D))
+    tk = rng.standard_normal((N, Hkv, D))
+    tv = rng.standard_normal((N, Hkv, D))
+    return q, pk, pv, tk, tv, np.asarray(parent)
+
+
+def check_attention_golden(attn):
+    g = read_kv("attention_worked.txt")
+    parent = np.array(_nums(g["parent"]), dtype=np.int64)
+    N = len(parent)
+    q = np.tile(np.array(_nums(g["q"]))[None, None, :], (N, 1, 1))
+    pk = np.array(_nums(g["prefix_k"]))[None, None, :]
+    pv = np.array(_nums(g["prefix_v"]))[None, None, :]
+    tk = _rows(g["tree_k"])[:, None, :]
+    tv = _rows(g["tree_v"])[:, None, :]
+    out = attn(q, pk, pv, tk, tv, parent)
+    for n in range(N):
+        np.testing.assert_allclose(out[n, 0], _nums(g[f"out{n}"]), rtol=0, atol=1e-12)
+
+
+def check_attention_chain_is_causal(attn, seed=1):
+    """A linear chain is ordinary causal attention over prefix + chain."""
+    rng = np.random.default_rng(seed)
+    N, P, Hq, Hkv, D = 7, 11, 4, 2, 8
+    parent = np.arange(-1, N - 1)
+    q, pk, pv, tk, tv, parent = _random_attention_case(rng, N, P, Hq, Hkv, D, parent)
+    K = np.concatenate([pk, tk.transpose(1, 0, 2)], axis=1)
+    V = np.concatenate([pv, tv.transpose(1, 0, 2)], axis=1)
+    G = Hq // Hkv
+    mask = np.arange(P + N)[None, :] <= (P + np.arange(N))[:, None]
+    ref = _sdpa(q.transpose(1, 0, 2), _expand_gqa(K, G), _expand_gqa(V, G), mask,
+                1.0 / math.sqrt(D))
+    np.testing.assert_allclose(attn(q, pk, pv, tk, tv, parent), ref.transpose(1, 0, 2),
+                               rtol=0, atol=1e-10)
+
+
+def _children(parent):
+    ch = {i: [] for i in range(len(parent))}
+    for j in range(1, len(parent)):
+        ch[int(parent[j])].append(j)
+    return ch
+
+
+def _paths_by_dfs(parent):
+    """Every root -> node path, found by depth-first search over child lists."""
+    ch = _children(parent)
+    paths = {}
+    stack = [[0]]
+    while stack:
+        p = stack.pop()
+        paths[p[-1]] = p
+        for c in ch[p[-1]]:
+            stack.append(p + [c])
+    return paths
+
+
+def check_attention_tree_paths(attn, seed=2):
+    """Brute force: node n of a tree equals the last query of plain attention
+    over prefix + its own root path (one SDPA call per node)."""
+    rng = np.random.default_rng(seed)
+    N, P, Hq, Hkv, D = 10, 5, 6, 2, 8
+    parent = [-1, 0, 0, 1, 1, 2, 4, 4, 3, 6]
+    q, pk, pv, tk, tv, parent = _random_attention_case(rng, N, P, Hq, Hkv, D, parent)
+    out = attn(q, pk, pv, tk, tv, parent)
+    G = Hq // Hkv
+    for n, path in _paths_by_dfs(parent).items():
+        K = np.concatenate([pk, tk[path].transpose(1, 0, 2)], axis=1)
+        V = np.concatenate([pv, tv[path].transpose(1, 0, 2)], axis=1)
+        mask = np.ones((1, K.shape[1]), dtype=bool)
+        ref = _sdpa(q[n][:, None, :], _expand_gqa(K, G), _expand_gqa(V, G), mask,
+                    1.0 / math.sqrt(D))
+        np.testing.assert_allclose(out[n], ref[:, 0, :], rtol=0, atol=1e-10)
+
+
+def check_attention_star_and_root(attn, seed=3):
+    """Star tree = independent single-query decodes; N = 1 = plain decode;
+    P = 0 = attention over the node's own path only."""
+    rng = np.random.default_rng(seed)
+    Hq, Hkv, D = 4, 1, 16
+    for N, P in ((6, 9), (1, 13), (5, 0)):
+        parent = [-1] + [0] * (N - 1)
+        q, pk, pv, tk, tv, parent = _random_attention_case(rng, N, P, Hq, Hkv, D, parent)
+        out = attn(q, pk, pv, tk, tv, parent)
+        for n in range(N):
+            rows = [0] if n == 0 else [0, n]
+            K = np.concatenate([pk, tk[rows].transpose(1, 0, 2)], axis=1)
+            V = np.concatenate([pv, tv[rows].transpose(1, 0, 2)], axis=1)
+            ref = _sdpa(q[n][:, None, :], _expand_gqa(K, Hq), _expand_gqa(V, Hq),
+                        np.ones((1, K.shape[1]), dtype=bool), 1.0 / math.sqrt(D))
+            np.testing.assert_allclose(out[n], ref[:, 0, :], rtol=0, atol=1e-10)
+
+
+def check_attention_uniform_values(attn, seed=4):
+    """If every visible value row equals c, the output is c whatever the scores."""
+    rng = np.random.default_rng(seed)
+    N, P, Hq, Hkv, D = 5, 7, 4, 2, 8
+    parent = [-1, 0, 1, 1, 0]
+    q, pk, _, tk, _, parent = _random_attention_case(rng, N, P, Hq, Hkv, D, parent)
+    c = rng.standard_normal((Hkv, D))
+    pv = np.repeat(c[:, None, :], P, axis=1)
+    tv = np.repeat(c[None, :, :], N, axis=0)
+    out = attn(q * 3.0, pk, pv, tk, tv, parent)
+    for h in range(Hq):
+        np.testing.assert_allclose(out[:, h, :], np.repeat(c[h // (Hq // Hkv)][None], N, 0),
+                                   rtol=0, atol=1e-12)
+
+
+ATTENTION_CHECKS = [check_attention_golden, check_attention_chain_is_causal,
+                    check_attention_tree_paths, check_attention_star_and_root,
+                    check_attention_uniform_values]
+
+
+# ----------------------------------------------------------------------------
+# LM head and greedy prediction
+# ----------------------------------------------------------------------------
+def check_lmhead_golden(logits_fn, greedy_fn):
+    g = read_kv("lmhead_worked.txt")
+    hidden, weight = _rows(g["hidden"]), _rows(g["weight"])
+    lg = logits_fn(hidden, weight)
+    np.testing.assert_array_equal(lg[0], _nums(g["logits0"]))
+    np.testing.assert_array_equal(lg[1], _nums(g["logits1"]))
+    am, margin, _ = greedy_fn(lg)
+    np.testing.assert_array_equal(am, [int(x) for x in _nums(g["argmax"])])
+    np.testing.assert_array_equal(margin, _nums(g["margin"]))
+
+
+def check_lmhead_exact_integers(logits_fn, greedy_fn, seed=5):
+    """Small-integer inputs: every logit is exact, so compare with Python
+    integer dot products, and argmax/margin with a scan written out here."""
+    rng = np.random.default_rng(seed)
+    N, V, H = 5, 37, 23
+    hidden = rng.integers(-3, 4, size=(N, H))
+    weight = rng.integers(-3, 4, size=(V, H))
+    lg = logits_fn(hidden.astype(np.float64), weight.astype(np.float64), chunk=8)
+    for n in range(N):
+        row = [sum(int(hidden[n, c]) * int(weight[v, c]) for c in range(H)) for v in range(V)]
+        assert list(lg[n].astype(np.int64)) == row
+        best = max(row)
+        first = row.index(best)
+        second = max(x for i, x in enumerate(row) if i != first)
+        am, margin, top = greedy_fn(lg[n:n + 1])
+        assert int(am[0]) == first and margin[0] == best - second and top[0] == best
+
+
+def check_lmhead_ties_lowest(logits_fn, greedy_fn):
+    lg = np.array([[0.5, 2.0, 2.0, -1.0], [3.0, 3.0, 3.0, 3.0], [-2.0, -1.0, -3.0, -1.0]])
+    am, margin, _ = greedy_fn(lg)
+    assert list(am) == [1, 0, 1]
+    assert list(margin) == [0.0, 0.0, 0.0]
+
+
+def check_lmhead_float_bruteforce(logits_fn, greedy_fn, seed=6):
+    """Random float64 inputs against math.fsum dot products."""
+    rng = np.random.default_rng(seed)
+    hidden = rng.standard_normal((3, 19))
+    weight = rng.standard_normal((29, 19))
+    lg = logits_fn(hidden, weight, chunk=7)
+    for n in range(3):
+        for v in range(29):
+            ref = math.fsum(float(hidden[n, c]) * float(weight[v, c]) for c in range(19))
+            assert abs(lg[n, v] - ref) <= 1e-12 * (1 + abs(ref))
+
+
+LMHEAD_CHECKS = [check_lmhead_golden, check_lmhead_exact_integers,
+                 check_lmhead_ties_lowest, check_lmhead_float_bruteforce]
+
+
+# ----------------------------------------------------------------------------
+# acceptance
+# ----------------------------------------------------------------------------
+def _ints(s):
+    return [int(x) for x in s.split()]
+
+
+def check_accept_golden(walk):
+    for line in open(os.path.join(GOLDEN, "accept_worked.txt")):
+        line = line.strip()
+        if not line or line.startswith("#"):
+            continue
+        lhs, rhs = line.split("||")
+        parent, tokens, greedy = [_ints(x) for x in lhs.split("|")]
+        a, path, out_tokens, last = [x.strip() for x in rhs.split("|")]
+        got = walk(parent, tokens, greedy)
+        assert got[0] == int(a), (line, got)
+        assert list(got[1]) == _ints(path), (line, got)
+        assert list(got[2]) == _ints(out_tokens), (line, got)
+        assert got[3] == int(last), (line, got)
+
+
+def check_accept_chain_prefix(walk, seed=7):
+    """Chain: accepted length = longest draft prefix equal to the greedy
+    predictions (Section 3.2), for every planted length."""
+    rng = np.random.default_rng(seed)
+    for ell in (0, 1, 2, 5, 12):
+        for planted in range(ell + 1):
+            greedy = rng.integers(0, 50, size=ell + 1)
+            drafts = [int(greedy[i]) if i < planted else int((greedy[i] + 1 + rng.integers(48)) % 50)
+                      for i in range(ell)]
+            tokens = [int(rng.integers(50))] + drafts
+            parent = list(range(-1, ell))
+            a, path, out_tokens, last = walk(parent, tokens, greedy)
+            assert a == planted
+            assert list(path) == list(range(planted + 1))
+            assert list(out_tokens) == drafts[:planted] + [int(greedy[planted])]
+            assert last == planted
+
+
+def check_accept_exhaustive(walk, seed=8):
+    """Trees with distinct sibling tokens: the walk's path is the unique
+    longest root path whose every edge matches the parent's prediction,
+    found by enumerating all node subsets that form root paths."""
+    rng = np.random.default_rng(seed)
+    for trial in range(60):
+        N = int(rng.integers(1, 9))
+        parent = [-1] + [int(rng.integers(0, j)) for j in range(1, N)]
+        V = 6
+        greedy = rng.integers(0, V, size=N)
+        tokens = [int(rng.integers(V))]
+        used = {}
+        for j in range(1, N):
+            choices = [t for t in range(V) if t not in used.get(parent[j], set())]
+            t = int(choices[rng.integers(len(choices))])
+            used.setdefault(parent[j], set()).add(t)
+            tokens.append(t)
+        best = [0]
+        for r in range(1, N + 1):
+            for subset in itertools.combinations(range(N), r):
+                if subset[0] != 0:
+                    continue
+                ok = all(parent[subset[i]] == subset[i - 1] and
+                         tokens[subset[i]] == greedy[subset[i - 1]] for i in range(1, r))
+                if ok and r > len(best):
+                    best = list(subset)
+        a, path, out_tokens, last = walk(parent, tokens, greedy)
+        assert list(path) == best, (parent, tokens, list(greedy), path, best)
+        assert a == len(best) - 1 and last == best[-1]
+        assert list(out_tokens) == [tokens[c] for c in best[1:]] + [int(greedy[best[-1]])]
+
+
+ACCEPT_CHECKS = [check_accept_golden, check_accept_chain_prefix, check_accept_exhaustive]
+
+
+# ----------------------------------------------------------------------------
+# commit
+# ----------------------------------------------------------------------------
+def check_commit_postcondition(commit, seed=9):
+    """Rows P..P+a hold the accepted path's tree rows; every other cache row
+    is untouched; the new length is P + a + 1."""
+    rng = np.random.default_rng(seed)
+    Hkv, S, D, N = 2, 20, 4, 6
+    for P, path in ((5, [0, 2, 3]), (0, [0]), (14, [0, 1, 4, 5])):
+        cache = rng.standard_normal((Hkv, S, D))
+        tree = rng.standard_normal((N, Hkv, D))
+        new, n1 = commit(cache, P, path, tree)
+        assert n1 == P + len(path)
+        for pos in range(S):
+            if P <= pos < P + len(path):
+                np.testing.assert_array_equal(new[:, pos, :], tree[path[pos - P]])
+            else:
+                np.testing.assert_array_equal(new[:, pos, :], cache[:, pos, :])
+
+
+COMMIT_CHECKS = [check_commit_postcondition]
+
+
+# ----------------------------------------------------------------------------
+# tree structure
+# ----------------------------------------------------------------------------
+def check_tree_structure(validate, depths, ancestors):
+    assert validate([-1]) and validate([-1, 0, 0, 1, 2])
+    for bad in ([], [0], [-1, 1], [-1, 0, 2], [-1, -1], [-1, 0, 3, 1]):
+        assert not validate(bad), bad
+    parent = [-1, 0, 0, 1, 3, 2]
+    assert list(depths(parent)) == [0, 1, 1, 2, 3, 2]
+    assert ancestors(parent, 4) == {0, 1, 3, 4}
+    assert ancestors(parent, 5) == {0, 2, 5}
+    assert ancestors(parent, 0) == {0}
+

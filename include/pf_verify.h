@@ -1,0 +1,241 @@
+/*
+ * pf_verify.h -- C ABI of the GB300 verify step for retrieval-based
+ * multi-token proposals (PastForward, "Experience-Guided Adaptive Decoding").
+ *
+ * Section 3.2 ("Single-pass token verification"): given the current token
+ * y_i and a proposal retrieved from decoding-experience memory, one forward
+ * pass predicts a token at every proposed position plus one more; the
+ * longest proposal prefix equal to those greedy predictions is accepted and
+ * the model's prediction at the first mismatch is appended, so the output
+ * advances by l_acc + 1 tokens.  Section 3.4 / Section 4 ("Runtime state
+ * management"): K/V states are carried forward in a cache and reused.
+ *
+ * This library runs the data-parallel part of that pass on one GPU:
+ *   pf_verify_attention  tree-masked GQA attention of the proposal nodes over
+ *                        the cached prefix (one call = one layer)
+ *   pf_lmhead_accept     LM-head logits, greedy argmax per node and the greedy
+ *                        descent of the proposal tree (accepted length, tokens)
+ *   pf_kv_commit         copy of the accepted path's K/V rows into the cache,
+ *                        all layers in one launch
+ * A proposal is a tree: node 0 is the current token (its K/V is not cached
+ * yet), nodes 1..N-1 are drafts, parent[j] < j.  A chain is the special case
+ * parent[j] = j - 1.  Queries and tree keys arrive rotary-embedded at
+ * position P + depth(node); hidden states arrive after the final norm.
+ *
+ * Conventions shared by every call
+ *   - All tensor pointers are caller-owned DEVICE memory unless stated; the
+ *     library keeps no pointer after a call returns and allocates no device
+ *     memory.  Tensors are dense row-major in the layouts documented below.
+ *   - Calls are asynchronous and stream-ordered on the given cudaStream_t
+ *     (passed as void*; NULL = legacy default stream).
+ *   - Argument errors are detected on the host before any launch and return a
+ *     non-zero pf_status; pf_last_error() then describes the problem.  No
+ *     call aborts the process and no kernel traps.
+ *   - error_flag (optional, may be NULL): a device int32 the kernels OR a
+ *     PF_DEVERR_* bit into when a device-side check fails (a bounded wait ran
+ *     out, or a row fell outside the cache); the caller clears and reads it.
+ */
+#ifndef PF_VERIFY_H
+#define PF_VERIFY_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define PF_API __attribute__((visibility("default")))
+#else
+#define PF_API
+#endif
+
+#define PF_MAX_NODES 128       /* nodes per proposal tree, root included   */
+#define PF_MASK_WORDS 2        /* uint64 words of ancestor mask per node   */
+#define PF_PAGE_SIZE 16        /* tokens per page of a paged KV cache      */
+#define PF_MAX_LM_ROWS 256     /* total proposal nodes of one LM-head call */
+
+typedef enum pf_status {
+  PF_OK = 0,
+  PF_ERR_NULL = 1,        /* a required pointer is NULL                    */
+  PF_ERR_SHAPE = 2,       /* a size is out of range or inconsistent        */
+  PF_ERR_DTYPE = 3,       /* unsupported dtype or dtype/shape combination  */
+  PF_ERR_TREE = 4,        /* parent[] is not a topologically ordered tree  */
+  PF_ERR_CAPACITY = 5,    /* the cache cannot hold prefix + committed rows */
+  PF_ERR_ALIGN = 6,       /* a pointer or stride breaks 16-byte alignment  */
+  PF_ERR_CUDA = 7,        /* the CUDA runtime reported an error            */
+  PF_ERR_WORKSPACE = 8    /* workspace missing or smaller than required    */
+} pf_status;
+
+typedef enum pf_dtype { PF_F32 = 0, PF_BF16 = 1 } pf_dtype;
+typedef enum pf_kv_layout { PF_KV_CONTIGUOUS = 0, PF_KV_PAGED = 1 } pf_kv_layout;
+
+/* Device error bits written into *error_flag. */
+#define PF_DEVERR_TIMEOUT 1    /* a bounded wait on a barrier ran out      */
+#define PF_DEVERR_CAPACITY 2   /* a commit row fell outside the cache      */
+#define PF_DEVERR_BOUNDS 4     /* device-side sizes (cu_nodes, prefix_len,
+                                  page_table) contradict the host bounds;
+                                  the affected work was skipped            */
+
+/* Message for the last non-OK status returned on this host thread. */
+PF_API const char* pf_last_error(void);
+/* Library ABI version (major * 100 + minor). */
+PF_API int32_t pf_version(void);
+
+/*
+ * pf_tree_prepare -- host-side validation of one proposal tree and its
+ * ancestor bitmap (the proposal-tree structure of Section 3.2 generalised
+ * from a chain to the union of retrieved chains).
+ *   parent    HOST [n_nodes]; parent[0] = -1, 0 <= parent[j] < j
+ *   n_nodes   1 .. PF_MAX_NODES
+ *   depth_out HOST [n_nodes] or NULL; edges between node and root
+ *   mask_out  HOST [n_nodes][PF_MASK_WORDS]; bit i of node j's mask is set
+ *             iff node i lies on the path root -> j (j included)
+ * Returns PF_ERR_TREE for a malformed tree, PF_ERR_SHAPE for a bad n_nodes.
+ */
+PF_API pf_status pf_tree_prepare(const int32_t* parent, int32_t n_nodes,
+                          int32_t* depth_out, uint64_t* mask_out);
+
+/* One layer's prefix KV cache. */
+typedef struct pf_kv_view {
+  int32_t layout;              /* pf_kv_layout                               */
+  void* k;                     /* contiguous: [B][Hkv][max_seq][D];          */
+  void* v;                     /* paged: [num_pages][Hkv][PF_PAGE_SIZE][D]   */
+  int32_t max_seq;             /* contiguous: rows per (sequence, KV head)   */
+  int32_t num_pages;           /* paged: pages in the pool                   */
+  const int32_t* page_table;   /* paged: device [B][pages_per_seq]           */
+  int32_t pages_per_seq;       /* paged: row length of page_table            */
+} pf_kv_view;
+
+/*
+ * pf_verify_attention -- tree-masked grouped-query attention of the
+ * proposal nodes of one layer over the reused prefix KV (Section 3.2
+ * single-pass verification, over the cache carried forward per Section
+ * 3.4).  For node n (global index t = cu_nodes[b] + n) and query head h,
+ * KV head g = h / (Hq / Hkv):
+ *   out[t,h] = sum_j softmax_j(scale * q[t,h] . k_j) v_j
+ * over j in { prefix rows 0 .. prefix_len[b]-1 of sequence b, head g }
+ *   U { tree rows i of sequence b : bit i of mask[t] is set }.
+ * Layouts: q, out [T][Hq][D]; tree_k, tree_v [T][Hkv][D]; mask [T][2]
+ * (from pf_tree_prepare, local node indices); cu_nodes [B+1] with
+ * cu_nodes[0] = 0, cu_nodes[B] = T; prefix_len [B].
+ * dtype PF_BF16 (D = 64 or 128, tensor cores, fp32 softmax, bf16 P.V) or
+ * PF_F32 (D <= 128, CUDA cores).  Every node must have
+ * 1 <= cu_nodes[b+1]-cu_nodes[b] <= max_nodes <= PF_MAX_NODES and
+ * prefix_len[b] <= max_prefix_len (and <= max_seq or the page table's
+ * reach).  Pointers must be 16-byte aligned.  Cache rows at positions
+ * >= prefix_len[b] are never used, whatever they hold.
+ */
+typedef struct pf_attn_desc {
+  int32_t dtype;               /* pf_dtype of q, tree_k/v, cache and out     */
+  int32_t batch;               /* B >= 1                                     */
+  int32_t n_q_heads;           /* Hq, a multiple of n_kv_heads               */
+  int32_t n_kv_heads;          /* Hkv                                        */
+  int32_t head_dim;            /* D                                          */
+  float scale;                 /* <= 0 selects 1/sqrt(D)                     */
+  int32_t total_nodes;         /* T = cu_nodes[B]                            */
+  int32_t max_nodes;           /* bound on the nodes of any one sequence     */
+  int32_t max_prefix_len;      /* bound on every prefix_len[b]               */
+  const int32_t* cu_nodes;     /* device [B+1]                               */
+  const int32_t* prefix_len;   /* device [B]                                 */
+  const void* q;               /* device [T][Hq][D]                          */
+  const void* tree_k;          /* device [T][Hkv][D]                         */
+  const void* tree_v;          /* device [T][Hkv][D]                         */
+  const uint64_t* mask;        /* device [T][PF_MASK_WORDS]                  */
+  pf_kv_view cache;            /* this layer's prefix cache                  */
+  void* out;                   /* device [T][Hq][D]                          */
+  int32_t* error_flag;         /* optional device int32                      */
+} pf_attn_desc;
+
+PF_API pf_status pf_verify_attention(const pf_attn_desc* d, void* stream);
+
+/*
+ * pf_lmhead_accept -- LM head, greedy prediction and acceptance
+ * (Section 3.2: predictions at every proposed position and one more; accept
+ * the longest matching proposal prefix; append the model's prediction).
+ *   logits[t, v] = sum_c hidden[t, c] * W[v, c]   (fp32 accumulation)
+ *   argmax[t]    = argmax_v logits[t, v], ties -> lowest v
+ * then, per sequence b, descend from the root: at node u the prediction is
+ * argmax[u]; move to the lowest-index child of u whose token equals it, or
+ * stop.  Outputs for sequence b (path length a+1, a = accept_len[b]):
+ *   path[b][0..a]        local node indices, path[b][0] = 0
+ *   out_tokens[b][0..a]  tokens of path[1..a], then the bonus argmax[path[a]]
+ *   last_node[b]         path[b][a] (its state is the next retrieval query)
+ * Rows of path/out_tokens have stride max_nodes.
+ * Layouts: hidden [T][H], weight [V][H] (row-major, H % 8 == 0), tokens and
+ * parent [T] (parent local to its sequence, -1 at each root).
+ * T <= PF_MAX_LM_ROWS.  dtype PF_BF16 (tensor cores) or PF_F32.
+ * Workspace: device memory of pf_lmhead_accept_workspace_size() bytes,
+ * zero-filled before its first use; every call leaves it zero-filled again,
+ * so one workspace serves calls in stream order but not concurrent calls.
+ */
+typedef struct pf_lm_desc {
+  int32_t dtype;               /* pf_dtype of hidden and weight              */
+  int32_t batch;               /* B >= 1                                     */
+  int32_t hidden;              /* H                                          */
+  int32_t vocab;               /* V                                          */
+  int32_t total_nodes;         /* T = cu_nodes[B]                            */
+  int32_t max_nodes;           /* bound on nodes per sequence; row stride    */
+  const int32_t* cu_nodes;     /* device [B+1]                               */
+  const void* hidden_states;   /* device [T][H]                              */
+  const void* weight;          /* device [V][H]                              */
+  const int32_t* tokens;       /* device [T]                                 */
+  const int32_t* parent;       /* device [T]                                 */
+  int32_t* argmax;             /* out device [T]                             */
+  float* max_logit;            /* out device [T], optional                   */
+  int32_t* accept_len;         /* out device [B]                             */
+  int32_t* path;               /* out device [B][max_nodes]                  */
+  int32_t* out_tokens;         /* out device [B][max_nodes]                  */
+  int32_t* last_node;          /* out device [B], optional                   */
+  int32_t* error_flag;         /* optional device int32                      */
+} pf_lm_desc;
+
+PF_API size_t pf_lmhead_accept_workspace_size(const pf_lm_desc* d);
+PF_API pf_status pf_lmhead_accept(const pf_lm_desc* d, void* workspace, size_t workspace_bytes,
+                           void* stream);
+
+/*
+ * pf_kv_commit -- carry the accepted rows forward (Section 1 and Section
+ * 3.4: accepted positions keep their K/V; Section 4: one contiguous cache).
+ * For every layer l, K and V, sequence b and k = 0..accept_len[b]:
+ *   cache_l[b, g, prefix_len[b] + k, :] = tree_l[cu_nodes[b] + path[b][k], g, :]
+ * and new_len[b] = prefix_len[b] + accept_len[b] + 1.  Rejected proposal rows
+ * are not copied.  accept_len and path are read from device memory (the
+ * outputs of pf_lmhead_accept), so no host synchronisation is needed.
+ * Layer l of the tree K/V starts at tree_k + l * tree_layer_stride elements
+ * ([T][Hkv][D] per layer); layer l of the cache at cache.k + l *
+ * cache_layer_stride elements (the pf_kv_view layout per layer).  The host
+ * checks max_prefix_len + max_nodes fits the cache; the kernel re-checks
+ * every row and sets PF_DEVERR_CAPACITY instead of writing outside it.
+ * new_len must not alias prefix_len.  The copy is bit-exact.
+ */
+typedef struct pf_commit_desc {
+  int32_t dtype;               /* pf_dtype (element size only)               */
+  int32_t batch;               /* B                                          */
+  int32_t n_layers;            /* L                                          */
+  int32_t n_kv_heads;          /* Hkv                                        */
+  int32_t head_dim;            /* D; D * element size must be a multiple of 16 */
+  int32_t total_nodes;         /* T                                          */
+  int32_t max_nodes;           /* bound on nodes per sequence; path row stride */
+  int32_t max_prefix_len;      /* bound on every prefix_len[b]               */
+  const int32_t* cu_nodes;     /* device [B+1]                               */
+  const int32_t* prefix_len;   /* device [B]                                 */
+  const int32_t* accept_len;   /* device [B]                                 */
+  const int32_t* path;         /* device [B][max_nodes]                      */
+  const void* tree_k;          /* device [L][T][Hkv][D] (see stride)         */
+  const void* tree_v;
+  int64_t tree_layer_stride;   /* elements between layers of tree_k/v        */
+  pf_kv_view cache;            /* layer 0's view; k and v advance per layer  */
+  int64_t cache_layer_stride;  /* elements between layers of cache.k/v       */
+  int32_t* new_len;            /* out device [B]                             */
+  int32_t* error_flag;         /* optional device int32                      */
+} pf_commit_desc;
+
+PF_API pf_status pf_kv_commit(const pf_commit_desc* d, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PF_VERIFY_H */

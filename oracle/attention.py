@@ -23,7 +23,7 @@ import numpy as np
 from .tree import ancestors_or_self
 
 
-def tree_attention(q, prefix_k, prefix_v, tree_k, tree_v, parent, scale=None):
+def tree_attention(q, prefix_k, prefix_v, tree_k, tree_v, parent, scale=None, nodes=None):
     """One sequence, one layer.
 
     q        [N, Hq, D]     queries of the N proposal nodes
@@ -33,6 +33,7 @@ def tree_attention(q, prefix_k, prefix_v, tree_k, tree_v, parent, scale=None):
     tree_v   [N, Hkv, D]    values of the proposal nodes
     parent   [N]            parent[0] = -1
     scale    softmax scale, default 1/sqrt(D)
+    nodes    optional subset of nodes to compute (others are left zero)
     returns  [N, Hq, D] float64
     """
     q = np.asarray(q, dtype=np.float64)
@@ -46,7 +47,7 @@ def tree_attention(q, prefix_k, prefix_v, tree_k, tree_v, parent, scale=None):
     if scale is None:
         scale = 1.0 / math.sqrt(D)
     out = np.zeros((N, Hq, D), dtype=np.float64)
-    for n in range(N):
+    for n in (range(N) if nodes is None else nodes):
         visible = sorted(ancestors_or_self(parent, n))
         for h in range(Hq):
             g = h // G

@@ -1,0 +1,160 @@
+"""ctypes binding of libpfverify.so (include/pf_verify.h).
+
+Argument marshalling only: every step of the verify path runs in the CUDA
+library.  The functions carry the C names; descriptors are the C structs.
+Tensors are passed as raw device pointers (``tensor.data_ptr()``); torch is
+used by callers for device memory and streams only.
+
+There is no fallback: if the library is missing or fails to load, every
+entry point raises ``PfLibraryMissing``.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import re
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libpfverify.so")
+HEADER = os.path.join(os.path.dirname(_PKG), "include", "pf_verify.h")
+
+PF_OK, PF_ERR_NULL, PF_ERR_SHAPE, PF_ERR_DTYPE, PF_ERR_TREE = 0, 1, 2, 3, 4
+PF_ERR_CAPACITY, PF_ERR_ALIGN, PF_ERR_CUDA, PF_ERR_WORKSPACE = 5, 6, 7, 8
+PF_F32, PF_BF16 = 0, 1
+PF_KV_CONTIGUOUS, PF_KV_PAGED = 0, 1
+PF_MAX_NODES, PF_MASK_WORDS, PF_PAGE_SIZE, PF_MAX_LM_ROWS = 128, 2, 16, 256
+PF_DEVERR_TIMEOUT, PF_DEVERR_CAPACITY, PF_DEVERR_BOUNDS = 1, 2, 4
+
+STATUS_NAMES = {0: "PF_OK", 1: "PF_ERR_NULL", 2: "PF_ERR_SHAPE", 3: "PF_ERR_DTYPE",
+                4: "PF_ERR_TREE", 5: "PF_ERR_CAPACITY", 6: "PF_ERR_ALIGN", 7: "PF_ERR_CUDA",
+                8: "PF_ERR_WORKSPACE"}
+
+
+class PfLibraryMissing(RuntimeError):
+    pass
+
+
+class PfError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {message}")
+        self.status = status
+
+
+class pf_kv_view(C.Structure):
+    _fields_ = [("layout", C.c_int32), ("k", C.c_void_p), ("v", C.c_void_p),
+                ("max_seq", C.c_int32), ("num_pages", C.c_int32),
+                ("page_table", C.c_void_p), ("pages_per_seq", C.c_int32)]
+
+
+class pf_attn_desc(C.Structure):
+    _fields_ = [("dtype", C.c_int32), ("batch", C.c_int32), ("n_q_heads", C.c_int32),
+                ("n_kv_heads", C.c_int32), ("head_dim", C.c_int32), ("scale", C.c_float),
+                ("total_nodes", C.c_int32), ("max_nodes", C.c_int32),
+                ("max_prefix_len", C.c_int32), ("cu_nodes", C.c_void_p),
+                ("prefix_len", C.c_void_p), ("q", C.c_void_p), ("tree_k", C.c_void_p),
+                ("tree_v", C.c_void_p), ("mask", C.c_void_p), ("cache", pf_kv_view),
+                ("out", C.c_void_p), ("error_flag", C.c_void_p)]
+
+
+class pf_lm_desc(C.Structure):
+    _fields_ = [("dtype", C.c_int32), ("batch", C.c_int32), ("hidden", C.c_int32),
+                ("vocab", C.c_int32), ("total_nodes", C.c_int32), ("max_nodes", C.c_int32),
+                ("cu_nodes", C.c_void_p), ("hidden_states", C.c_void_p),
+                ("weight", C.c_void_p), ("tokens", C.c_void_p), ("parent", C.c_void_p),
+                ("argmax", C.c_void_p), ("max_logit", C.c_void_p),
+                ("accept_len", C.c_void_p), ("path", C.c_void_p),
+                ("out_tokens", C.c_void_p), ("last_node", C.c_void_p),
+                ("error_flag", C.c_void_p)]
+
+
+class pf_commit_desc(C.Structure):
+    _fields_ = [("dtype", C.c_int32), ("batch", C.c_int32), ("n_layers", C.c_int32),
+                ("n_kv_heads", C.c_int32), ("head_dim", C.c_int32),
+                ("total_nodes", C.c_int32), ("max_nodes", C.c_int32),
+                ("max_prefix_len", C.c_int32), ("cu_nodes", C.c_void_p),
+                ("prefix_len", C.c_void_p), ("accept_len", C.c_void_p), ("path", C.c_void_p),
+                ("tree_k", C.c_void_p), ("tree_v", C.c_void_p),
+                ("tree_layer_stride", C.c_int64), ("cache", pf_kv_view),
+                ("cache_layer_stride", C.c_int64), ("new_len", C.c_void_p),
+                ("error_flag", C.c_void_p)]
+
+
+_lib = None
+
+
+def lib() -> C.CDLL:
+    """The loaded library; raises PfLibraryMissing if it is not built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise PfLibraryMissing(
+            f"{LIB_PATH} is not built; run __graft_entry__.build() (nvcc, sm_103a)")
+    try:
+        L = C.CDLL(LIB_PATH)
+    except OSError as e:
+        raise PfLibraryMissing(f"cannot load {LIB_PATH}: {e}") from e
+    L.pf_last_error.restype = C.c_char_p
+    L.pf_last_error.argtypes = []
+    L.pf_version.restype = C.c_int32
+    L.pf_tree_prepare.restype = C.c_int
+    L.pf_tree_prepare.argtypes = [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p]
+    L.pf_verify_attention.restype = C.c_int
+    L.pf_verify_attention.argtypes = [C.POINTER(pf_attn_desc), C.c_void_p]
+    L.pf_lmhead_accept_workspace_size.restype = C.c_size_t
+    L.pf_lmhead_accept_workspace_size.argtypes = [C.POINTER(pf_lm_desc)]
+    L.pf_lmhead_accept.restype = C.c_int
+    L.pf_lmhead_accept.argtypes = [C.POINTER(pf_lm_desc), C.c_void_p, C.c_size_t, C.c_void_p]
+    L.pf_kv_commit.restype = C.c_int
+    L.pf_kv_commit.argtypes = [C.POINTER(pf_commit_desc), C.c_void_p]
+    _lib = L
+    return L
+
+
+def header_functions() -> list:
+    """Names of the functions include/pf_verify.h declares."""
+    src = open(HEADER).read()
+    return re.findall(r"PF_API\s+[\w\s\*]+?\b(pf_\w+)\s*\(", src)
+
+
+def _check(status: int) -> None:
+    if status != PF_OK:
+        raise PfError(status, lib().pf_last_error().decode())
+
+
+def pf_version() -> int:
+    return int(lib().pf_version())
+
+
+def pf_last_error() -> str:
+    return lib().pf_last_error().decode()
+
+
+def pf_tree_prepare(parent) -> tuple:
+    """Host call: returns (depth int32 [N], mask uint64 [N, 2])."""
+    p = np.ascontiguousarray(parent, dtype=np.int32)
+    n = int(p.shape[0])
+    depth = np.zeros(max(n, 1), dtype=np.int32)
+    mask = np.zeros((max(n, 1), PF_MASK_WORDS), dtype=np.uint64)
+    _check(lib().pf_tree_prepare(p.ctypes.data, n, depth.ctypes.data, mask.ctypes.data))
+    return depth[:n], mask[:n]
+
+
+def pf_verify_attention(desc: pf_attn_desc, stream: int = 0) -> None:
+    _check(lib().pf_verify_attention(C.byref(desc), C.c_void_p(stream)))
+
+
+def pf_lmhead_accept_workspace_size(desc: pf_lm_desc = None) -> int:
+    return int(lib().pf_lmhead_accept_workspace_size(C.byref(desc) if desc else None))
+
+
+def pf_lmhead_accept(desc: pf_lm_desc, workspace: int, workspace_bytes: int,
+                     stream: int = 0) -> None:
+    _check(lib().pf_lmhead_accept(C.byref(desc), C.c_void_p(workspace),
+                                  C.c_size_t(workspace_bytes), C.c_void_p(stream)))
+
+
+def pf_kv_commit(desc: pf_commit_desc, stream: int = 0) -> None:
+    _check(lib().pf_kv_commit(C.byref(desc), C.c_void_p(stream)))

@@ -1,0 +1,390 @@
+// C ABI of the verify step: argument validation on the host, TMA tensor-map
+// encoding, launch-shape selection and the kernel launches.  See
+// include/pf_verify.h for the contract of every entry point.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <string>
+
+#include "pf_internal.h"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+pf_status fail(pf_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return s;
+}
+
+pf_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(PF_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* e = getenv("PF_PDL");
+    return !(e && e[0] == '0');
+  }();
+  return on;
+}
+
+int num_sms() {
+  static int cache[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (dev >= 0 && dev < 64 && cache[dev]) return cache[dev];
+  int n = 0;
+  cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+  if (dev >= 0 && dev < 64) cache[dev] = n;
+  return n;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// bf16 tensor map with the 128-byte swizzle; dims/strides innermost first,
+// strides in bytes for dims 1..rank-1.
+pf_status make_map(CUtensorMap* m, int rank, const void* base, const cuuint64_t* dims,
+                   const cuuint64_t* strides, const cuuint32_t* box, const char* what) {
+  auto fn = encode_fn();
+  if (!fn) return fail(PF_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable (no CUDA driver?)");
+  cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void*>(base),
+                  dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(PF_ERR_CUDA, "tensor map for %s: CUresult %d", what, (int)r);
+  return PF_OK;
+}
+
+int elem_size(int dtype) { return dtype == PF_BF16 ? 2 : 4; }
+
+pf_status check_cache_view(const pf_kv_view& c, int need_rows, const char* who) {
+  if (!c.k || !c.v) return fail(PF_ERR_NULL, "%s: cache.k/cache.v is NULL", who);
+  if (!aligned16(c.k) || !aligned16(c.v))
+    return fail(PF_ERR_ALIGN, "%s: cache pointers must be 16-byte aligned", who);
+  if (c.layout == PF_KV_CONTIGUOUS) {
+    if (c.max_seq < 1) return fail(PF_ERR_SHAPE, "%s: cache.max_seq must be >= 1", who);
+    if (need_rows > c.max_seq)
+      return fail(PF_ERR_CAPACITY, "%s: %d rows needed but cache.max_seq = %d", who, need_rows,
+                  c.max_seq);
+  } else if (c.layout == PF_KV_PAGED) {
+    if (!c.page_table) return fail(PF_ERR_NULL, "%s: cache.page_table is NULL", who);
+    if (c.num_pages < 1 || c.pages_per_seq < 1)
+      return fail(PF_ERR_SHAPE, "%s: num_pages and pages_per_seq must be >= 1", who);
+    const int pages = (need_rows + PF_PAGE_SIZE - 1) / PF_PAGE_SIZE;
+    if (pages > c.pages_per_seq)
+      return fail(PF_ERR_CAPACITY, "%s: %d pages needed but pages_per_seq = %d", who, pages,
+                  c.pages_per_seq);
+  } else {
+    return fail(PF_ERR_SHAPE, "%s: unknown cache layout %d", who, c.layout);
+  }
+  return PF_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* pf_last_error(void) { return g_last_error.c_str(); }
+
+int32_t pf_version(void) { return 100; }
+
+pf_status pf_tree_prepare(const int32_t* parent, int32_t n_nodes, int32_t* depth_out,
+                          uint64_t* mask_out) {
+  if (!parent || !mask_out) return fail(PF_ERR_NULL, "pf_tree_prepare: parent/mask_out is NULL");
+  if (n_nodes < 1 || n_nodes > PF_MAX_NODES)
+    return fail(PF_ERR_SHAPE, "pf_tree_prepare: n_nodes = %d outside 1..%d", n_nodes,
+                PF_MAX_NODES);
+  if (parent[0] != -1) return fail(PF_ERR_TREE, "pf_tree_prepare: parent[0] must be -1");
+  for (int j = 1; j < n_nodes; ++j)
+    if (parent[j] < 0 || parent[j] >= j)
+      return fail(PF_ERR_TREE, "pf_tree_prepare: parent[%d] = %d is not in [0, %d)", j,
+                  parent[j], j);
+  // Nodes are topologically ordered, so each node's mask is its parent's
+  // mask plus its own bit.
+  for (int j = 0; j < n_nodes; ++j) {
+    uint64_t* mj = mask_out + (size_t)j * PF_MASK_WORDS;
+    if (j == 0) {
+      for (int w = 0; w < PF_MASK_WORDS; ++w) mj[w] = 0;
+      if (depth_out) depth_out[0] = 0;
+    } else {
+      const uint64_t* mp = mask_out + (size_t)parent[j] * PF_MASK_WORDS;
+      for (int w = 0; w < PF_MASK_WORDS; ++w) mj[w] = mp[w];
+      if (depth_out) depth_out[j] = depth_out[parent[j]] + 1;
+    }
+    mj[j >> 6] |= 1ull << (j & 63);
+  }
+  return PF_OK;
+}
+
+pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
+  static const char* who = "pf_verify_attention";
+  if (!d) return fail(PF_ERR_NULL, "%s: desc is NULL", who);
+  if (!d->cu_nodes || !d->prefix_len || !d->q || !d->tree_k || !d->tree_v || !d->mask || !d->out)
+    return fail(PF_ERR_NULL, "%s: a required pointer is NULL", who);
+  if (d->dtype != PF_BF16 && d->dtype != PF_F32)
+    return fail(PF_ERR_DTYPE, "%s: dtype %d unsupported", who, d->dtype);
+  if (d->batch < 1 || d->n_kv_heads < 1 || d->n_q_heads < 1 ||
+      d->n_q_heads % d->n_kv_heads != 0)
+    return fail(PF_ERR_SHAPE, "%s: need batch >= 1 and n_q_heads a multiple of n_kv_heads", who);
+  const int D = d->head_dim;
+  const int G = d->n_q_heads / d->n_kv_heads;
+  if (d->dtype == PF_BF16 && D != 64 && D != 128)
+    return fail(PF_ERR_SHAPE, "%s: bf16 head_dim must be 64 or 128 (got %d)", who, D);
+  if (d->dtype == PF_F32 && (D < 1 || D > 128))
+    return fail(PF_ERR_SHAPE, "%s: fp32 head_dim must be in 1..128 (got %d)", who, D);
+  if (d->dtype == PF_BF16 && G > 128)
+    return fail(PF_ERR_SHAPE, "%s: query heads per KV head must be <= 128", who);
+  if (d->max_nodes < 1 || d->max_nodes > PF_MAX_NODES || d->total_nodes < 1)
+    return fail(PF_ERR_SHAPE, "%s: max_nodes must be in 1..%d and total_nodes >= 1", who,
+                PF_MAX_NODES);
+  if (d->max_prefix_len < 0) return fail(PF_ERR_SHAPE, "%s: max_prefix_len < 0", who);
+  pf_status st = check_cache_view(d->cache, d->max_prefix_len, who);
+  if (st != PF_OK) return st;
+  if (!aligned16(d->q) || !aligned16(d->tree_k) || !aligned16(d->tree_v) || !aligned16(d->out) ||
+      !aligned16(d->mask))
+    return fail(PF_ERR_ALIGN, "%s: tensor pointers must be 16-byte aligned", who);
+
+  pf::AttnArgs a = {};
+  a.B = d->batch;
+  a.Hq = d->n_q_heads;
+  a.Hkv = d->n_kv_heads;
+  a.D = D;
+  a.G = G;
+  a.T = d->total_nodes;
+  a.max_nodes = d->max_nodes;
+  a.max_prefix = d->max_prefix_len;
+  a.scale = d->scale > 0.f ? d->scale : 1.0f / sqrtf((float)D);
+  a.scale_log2 = a.scale * 1.4426950408889634f;
+  a.cu_nodes = d->cu_nodes;
+  a.prefix_len = d->prefix_len;
+  a.mask = d->mask;
+  a.out = d->out;
+  a.layout = d->cache.layout;
+  a.max_seq = d->cache.max_seq;
+  a.page_table = d->cache.page_table;
+  a.pages_per_seq = d->cache.pages_per_seq;
+  a.num_pages = d->cache.num_pages;
+  a.err = d->error_flag;
+  a.q = d->q;
+  a.tk = d->tree_k;
+  a.tv = d->tree_v;
+  a.ck = d->cache.k;
+  a.cv = d->cache.v;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int sms = num_sms();
+  if (sms <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
+
+  if (d->dtype == PF_F32) {
+    a.nb = 0;
+    a.rb_count = (d->max_nodes * G + 31) / 32;
+    a.splits = 1;
+    cudaError_t e = pf::launch_attention_f32(a, s, pdl_enabled());
+    return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
+  }
+
+  a.nb = 128 / G;
+  a.rb_count = (d->max_nodes + a.nb - 1) / a.nb;
+  const int base = a.B * a.Hkv * a.rb_count;
+  const int max_tiles = (d->max_prefix_len + 63) / 64 + (d->max_nodes + 63) / 64;
+  int splits = sms / base;
+  if (const char* e = getenv("PF_ATTN_SPLITS")) splits = atoi(e);
+  if (splits > 8) splits = 8;
+  if (splits > max_tiles) splits = max_tiles;
+  if (splits < 1) splits = 1;
+  a.splits = splits;
+
+  pf::AttnMaps m;
+  const cuuint64_t es = 2;
+  {
+    cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)a.Hq, (cuuint64_t)a.T};
+    cuuint64_t str[2] = {D * es, (cuuint64_t)a.Hq * D * es};
+    cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)a.nb};
+    if ((st = make_map(&m.q, 3, d->q, dims, str, box, "q")) != PF_OK) return st;
+  }
+  {
+    cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)a.Hkv, (cuuint64_t)a.T};
+    cuuint64_t str[2] = {D * es, (cuuint64_t)a.Hkv * D * es};
+    cuuint32_t box[3] = {64, 1, 64};
+    if ((st = make_map(&m.tk, 3, d->tree_k, dims, str, box, "tree_k")) != PF_OK) return st;
+    if ((st = make_map(&m.tv, 3, d->tree_v, dims, str, box, "tree_v")) != PF_OK) return st;
+  }
+  if (a.layout == PF_KV_CONTIGUOUS) {
+    cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)a.max_seq, (cuuint64_t)a.B * a.Hkv};
+    cuuint64_t str[2] = {D * es, (cuuint64_t)a.max_seq * D * es};
+    cuuint32_t box[3] = {64, 64, 1};
+    if ((st = make_map(&m.ck, 3, d->cache.k, dims, str, box, "cache.k")) != PF_OK) return st;
+    if ((st = make_map(&m.cv, 3, d->cache.v, dims, str, box, "cache.v")) != PF_OK) return st;
+  } else {
+    cuuint64_t dims[4] = {(cuuint64_t)D, PF_PAGE_SIZE, (cuuint64_t)a.Hkv,
+                          (cuuint64_t)a.num_pages};
+    cuuint64_t str[3] = {D * es, PF_PAGE_SIZE * D * es, (cuuint64_t)a.Hkv * PF_PAGE_SIZE * D * es};
+    cuuint32_t box[4] = {64, PF_PAGE_SIZE, 1, 1};
+    if ((st = make_map(&m.ck, 4, d->cache.k, dims, str, box, "cache.k")) != PF_OK) return st;
+    if ((st = make_map(&m.cv, 4, d->cache.v, dims, str, box, "cache.v")) != PF_OK) return st;
+  }
+  cudaError_t e = pf::launch_attention_bf16(a, m, s, sms, pdl_enabled());
+  return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
+}
+
+size_t pf_lmhead_accept_workspace_size(const pf_lm_desc*) { return pf::kLmWorkspaceBytes; }
+
+pf_status pf_lmhead_accept(const pf_lm_desc* d, void* workspace, size_t workspace_bytes,
+                           void* stream) {
+  static const char* who = "pf_lmhead_accept";
+  if (!d) return fail(PF_ERR_NULL, "%s: desc is NULL", who);
+  if (!d->cu_nodes || !d->hidden_states || !d->weight || !d->tokens || !d->parent ||
+      !d->argmax || !d->accept_len || !d->path || !d->out_tokens)
+    return fail(PF_ERR_NULL, "%s: a required pointer is NULL", who);
+  if (!workspace || workspace_bytes < pf::kLmWorkspaceBytes)
+    return fail(PF_ERR_WORKSPACE, "%s: workspace needs %zu bytes", who, pf::kLmWorkspaceBytes);
+  if (d->dtype != PF_BF16 && d->dtype != PF_F32)
+    return fail(PF_ERR_DTYPE, "%s: dtype %d unsupported", who, d->dtype);
+  if (d->batch < 1 || d->hidden < 1 || d->vocab < 1)
+    return fail(PF_ERR_SHAPE, "%s: batch, hidden and vocab must be >= 1", who);
+  if (d->total_nodes < 1 || d->total_nodes > PF_MAX_LM_ROWS)
+    return fail(PF_ERR_SHAPE, "%s: total_nodes = %d outside 1..%d", who, d->total_nodes,
+                PF_MAX_LM_ROWS);
+  if (d->max_nodes < 1 || d->max_nodes > PF_MAX_NODES)
+    return fail(PF_ERR_SHAPE, "%s: max_nodes outside 1..%d", who, PF_MAX_NODES);
+  if (d->dtype == PF_BF16 && d->hidden % 8 != 0)
+    return fail(PF_ERR_ALIGN, "%s: bf16 hidden size must be a multiple of 8", who);
+  if (!aligned16(d->hidden_states) || !aligned16(d->weight) || !aligned16(workspace))
+    return fail(PF_ERR_ALIGN, "%s: hidden, weight and workspace must be 16-byte aligned", who);
+
+  pf::LmArgs a = {};
+  a.T = d->total_nodes;
+  a.H = d->hidden;
+  a.V = d->vocab;
+  a.B = d->batch;
+  a.max_nodes = d->max_nodes;
+  a.npad = (a.T + 15) / 16 * 16;
+  a.num_tiles = (a.V + 127) / 128;
+  a.nk = (a.H + 63) / 64;
+  a.cu_nodes = d->cu_nodes;
+  a.tokens = d->tokens;
+  a.parent = d->parent;
+  a.argmax = d->argmax;
+  a.max_logit = d->max_logit;
+  a.accept_len = d->accept_len;
+  a.path = d->path;
+  a.out_tokens = d->out_tokens;
+  a.last_node = d->last_node;
+  a.best = static_cast<unsigned long long*>(workspace);
+  a.ticket = reinterpret_cast<unsigned int*>(static_cast<char*>(workspace) + 8 * PF_MAX_LM_ROWS);
+  a.err = d->error_flag;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int sms = num_sms();
+  if (sms <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
+
+  if (d->dtype == PF_F32) {
+    a.hidden_f32 = static_cast<const float*>(d->hidden_states);
+    a.weight_f32 = static_cast<const float*>(d->weight);
+    cudaError_t e = pf::launch_lmhead_f32(a, s, sms, pdl_enabled());
+    return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
+  }
+  a.stages = pf::lmhead_bf16_stages(a.npad);
+  CUtensorMap wm, hm;
+  pf_status st;
+  {
+    cuuint64_t dims[2] = {(cuuint64_t)a.H, (cuuint64_t)a.V};
+    cuuint64_t str[1] = {(cuuint64_t)a.H * 2};
+    cuuint32_t box[2] = {64, 128};
+    if ((st = make_map(&wm, 2, d->weight, dims, str, box, "weight")) != PF_OK) return st;
+  }
+  {
+    cuuint64_t dims[2] = {(cuuint64_t)a.H, (cuuint64_t)a.T};
+    cuuint64_t str[1] = {(cuuint64_t)a.H * 2};
+    cuuint32_t box[2] = {64, (cuuint32_t)a.npad};
+    if ((st = make_map(&hm, 2, d->hidden_states, dims, str, box, "hidden")) != PF_OK) return st;
+  }
+  cudaError_t e = pf::launch_lmhead_bf16(a, wm, hm, s, sms, pdl_enabled());
+  return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
+}
+
+pf_status pf_kv_commit(const pf_commit_desc* d, void* stream) {
+  static const char* who = "pf_kv_commit";
+  if (!d) return fail(PF_ERR_NULL, "%s: desc is NULL", who);
+  if (!d->cu_nodes || !d->prefix_len || !d->accept_len || !d->path || !d->tree_k || !d->tree_v ||
+      !d->new_len)
+    return fail(PF_ERR_NULL, "%s: a required pointer is NULL", who);
+  if (d->dtype != PF_BF16 && d->dtype != PF_F32)
+    return fail(PF_ERR_DTYPE, "%s: dtype %d unsupported", who, d->dtype);
+  if (d->batch < 1 || d->n_layers < 1 || d->n_kv_heads < 1 || d->head_dim < 1 ||
+      d->total_nodes < 1)
+    return fail(PF_ERR_SHAPE, "%s: batch, n_layers, n_kv_heads, head_dim, total_nodes >= 1", who);
+  if (d->max_nodes < 1 || d->max_nodes > PF_MAX_NODES)
+    return fail(PF_ERR_SHAPE, "%s: max_nodes outside 1..%d", who, PF_MAX_NODES);
+  if (d->max_prefix_len < 0) return fail(PF_ERR_SHAPE, "%s: max_prefix_len < 0", who);
+  const int es = elem_size(d->dtype);
+  const int row_bytes = d->head_dim * es;
+  if (row_bytes % 16 != 0)
+    return fail(PF_ERR_ALIGN, "%s: head_dim * element size must be a multiple of 16", who);
+  if (d->n_layers > 1 && ((d->tree_layer_stride * es) % 16 != 0 ||
+                          (d->cache_layer_stride * es) % 16 != 0))
+    return fail(PF_ERR_ALIGN, "%s: layer strides must be multiples of 16 bytes", who);
+  if (!aligned16(d->tree_k) || !aligned16(d->tree_v))
+    return fail(PF_ERR_ALIGN, "%s: tree pointers must be 16-byte aligned", who);
+  if (d->new_len == d->prefix_len)
+    return fail(PF_ERR_SHAPE, "%s: new_len must not alias prefix_len", who);
+  pf_status st = check_cache_view(d->cache, d->max_prefix_len + d->max_nodes, who);
+  if (st != PF_OK) return st;
+
+  pf::CommitArgs a = {};
+  a.B = d->batch;
+  a.L = d->n_layers;
+  a.Hkv = d->n_kv_heads;
+  a.row_bytes = row_bytes;
+  a.max_nodes = d->max_nodes;
+  a.T = d->total_nodes;
+  a.cu_nodes = d->cu_nodes;
+  a.prefix_len = d->prefix_len;
+  a.accept_len = d->accept_len;
+  a.path = d->path;
+  a.tree_k = static_cast<const char*>(d->tree_k);
+  a.tree_v = static_cast<const char*>(d->tree_v);
+  a.tree_layer_bytes = d->tree_layer_stride * es;
+  a.cache_k = static_cast<char*>(d->cache.k);
+  a.cache_v = static_cast<char*>(d->cache.v);
+  a.cache_layer_bytes = d->cache_layer_stride * es;
+  a.layout = d->cache.layout;
+  a.max_seq = d->cache.max_seq;
+  a.page_table = d->cache.page_table;
+  a.pages_per_seq = d->cache.pages_per_seq;
+  a.num_pages = d->cache.num_pages;
+  a.new_len = d->new_len;
+  a.err = d->error_flag;
+  const int sms = num_sms();
+  if (sms <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
+  cudaError_t e = pf::launch_kv_commit(a, static_cast<cudaStream_t>(stream), sms, pdl_enabled());
+  return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
+}
+
+}  // extern "C"

@@ -1,0 +1,83 @@
+// Carry-forward of the accepted rows (Section 1; Section 3.4; Section 4's
+// contiguous cache): for every layer, K and V, sequence b and path slot
+// k <= accept_len[b], the row of proposal node path[b][k] moves to cache
+// position prefix_len[b] + k.  One launch covers all layers; each thread
+// moves one 16-byte chunk, so a 256-byte row is one fully coalesced group of
+// 16 threads.  accept_len and path are read on the device, straight from the
+// LM-head kernel's outputs, so the host never waits for them.
+#include "pf_internal.h"
+#include "pf_ptx.cuh"
+
+namespace pf {
+
+namespace {
+
+__global__ void __launch_bounds__(256) kv_commit_kernel(const CommitArgs a) {
+  pdl_wait();
+  const int chunks = a.row_bytes / 16;
+  const long long per_layer_kv = (long long)a.B * a.max_nodes * a.Hkv * chunks;
+  const long long total = per_layer_kv * 2 * a.L;
+  for (long long u = (long long)blockIdx.x * blockDim.x + threadIdx.x; u < total;
+       u += (long long)gridDim.x * blockDim.x) {
+    long long r = u;
+    const int c = (int)(r % chunks);
+    r /= chunks;
+    const int g = (int)(r % a.Hkv);
+    r /= a.Hkv;
+    const int k = (int)(r % a.max_nodes);
+    r /= a.max_nodes;
+    const int b = (int)(r % a.B);
+    r /= a.B;
+    const int kv = (int)(r % 2);
+    const int l = (int)(r / 2);
+    const int acc = a.accept_len[b];
+    if (k > acc) continue;
+    const int node0 = a.cu_nodes[b];
+    const int nn = a.cu_nodes[b + 1] - node0;
+    const int node = a.path[(size_t)b * a.max_nodes + k];
+    if (node0 < 0 || node0 + nn > a.T || node < 0 || node >= nn) {
+      flag_error(a.err, PF_DEVERR_BOUNDS);
+      continue;
+    }
+    const int pos = a.prefix_len[b] + k;
+    long long dst_row;
+    if (a.layout == PF_KV_CONTIGUOUS) {
+      if (pos >= a.max_seq) {
+        flag_error(a.err, PF_DEVERR_CAPACITY);
+        continue;
+      }
+      dst_row = ((long long)b * a.Hkv + g) * a.max_seq + pos;
+    } else {
+      const int pi = pos / PF_PAGE_SIZE;
+      const int page = pi < a.pages_per_seq ? a.page_table[(size_t)b * a.pages_per_seq + pi] : -1;
+      if (page < 0 || page >= a.num_pages) {
+        flag_error(a.err, PF_DEVERR_CAPACITY);
+        continue;
+      }
+      dst_row = ((long long)page * a.Hkv + g) * PF_PAGE_SIZE + pos % PF_PAGE_SIZE;
+    }
+    const char* src = (kv ? a.tree_v : a.tree_k) + l * a.tree_layer_bytes +
+                      (((long long)(node0 + node) * a.Hkv + g) * a.row_bytes) + c * 16;
+    char* dst = (kv ? a.cache_v : a.cache_k) + l * a.cache_layer_bytes +
+                dst_row * a.row_bytes + c * 16;
+    *reinterpret_cast<uint4*>(dst) = __ldg(reinterpret_cast<const uint4*>(src));
+  }
+  if (blockIdx.x == 0)
+    for (int b = threadIdx.x; b < a.B; b += blockDim.x)
+      a.new_len[b] = a.prefix_len[b] + a.accept_len[b] + 1;
+  pdl_launch_dependents();
+}
+
+}  // namespace
+
+cudaError_t launch_kv_commit(const CommitArgs& a, cudaStream_t s, int num_sms, bool pdl) {
+  const long long total =
+      (long long)a.B * a.max_nodes * a.Hkv * (a.row_bytes / 16) * 2 * a.L;
+  long long blocks = (total + 255) / 256;
+  const long long cap = (long long)num_sms * 8;
+  if (blocks > cap) blocks = cap;
+  if (blocks < 1) blocks = 1;
+  return launch_ex(kv_commit_kernel, dim3((unsigned)blocks), dim3(256), 0, s, 1, pdl, a);
+}
+
+}  // namespace pf

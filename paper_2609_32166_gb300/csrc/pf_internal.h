@@ -1,0 +1,147 @@
+// Internal interface between the C-ABI layer (api.cu) and the kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <utility>
+
+#include "pf_verify.h"
+
+namespace pf {
+
+// ------------------------------------------------------------ attention
+struct AttnArgs {
+  int B, Hq, Hkv, D, G;
+  int T, max_nodes, max_prefix;
+  int nb;          // proposal nodes per row block (bf16: floor(128 / G))
+  int rb_count;    // row blocks per (sequence, KV head)
+  int splits;      // CTAs of one cluster, each taking a slice of the KV tiles
+  float scale_log2;  // softmax scale * log2(e)
+  float scale;
+  const int32_t* cu_nodes;
+  const int32_t* prefix_len;
+  const uint64_t* mask;
+  void* out;
+  int layout;
+  int max_seq;
+  const int32_t* page_table;
+  int pages_per_seq;
+  int num_pages;
+  int32_t* err;
+  // raw pointers (fp32 path; the bf16 path reads through tensor maps)
+  const void* q;
+  const void* tk;
+  const void* tv;
+  const void* ck;
+  const void* cv;
+};
+
+struct AttnMaps {
+  CUtensorMap q, tk, tv, ck, cv;
+};
+
+cudaError_t launch_attention_bf16(const AttnArgs& a, const AttnMaps& m, cudaStream_t s,
+                                  int num_sms, bool pdl);
+cudaError_t launch_attention_f32(const AttnArgs& a, cudaStream_t s, bool pdl);
+int attention_bf16_smem_bytes(int D);
+
+// ------------------------------------------------------------ LM head
+struct LmArgs {
+  int T, H, V, B, max_nodes;
+  int npad;        // T rounded up to a multiple of 16 (UMMA N)
+  int num_tiles;   // ceil(V / 128)
+  int nk;          // ceil(H / 64)
+  int stages;      // TMA pipeline depth
+  const int32_t* cu_nodes;
+  const int32_t* tokens;
+  const int32_t* parent;
+  int32_t* argmax;
+  float* max_logit;
+  int32_t* accept_len;
+  int32_t* path;
+  int32_t* out_tokens;
+  int32_t* last_node;
+  unsigned long long* best;  // workspace [PF_MAX_LM_ROWS]
+  unsigned int* ticket;      // workspace
+  int32_t* err;
+  const float* hidden_f32;
+  const float* weight_f32;
+};
+
+cudaError_t launch_lmhead_bf16(const LmArgs& a, const CUtensorMap& w_map,
+                               const CUtensorMap& h_map, cudaStream_t s, int num_sms, bool pdl);
+cudaError_t launch_lmhead_f32(const LmArgs& a, cudaStream_t s, int num_sms, bool pdl);
+int lmhead_bf16_stages(int npad);
+int lmhead_bf16_smem_bytes(int npad, int stages);
+
+constexpr size_t kLmWorkspaceBytes = 8 * PF_MAX_LM_ROWS + 64;
+
+// ------------------------------------------------------------ commit
+struct CommitArgs {
+  int B, L, Hkv, row_bytes, max_nodes, T;
+  const int32_t* cu_nodes;
+  const int32_t* prefix_len;
+  const int32_t* accept_len;
+  const int32_t* path;
+  const char* tree_k;
+  const char* tree_v;
+  long long tree_layer_bytes;
+  char* cache_k;
+  char* cache_v;
+  long long cache_layer_bytes;
+  int layout;
+  int max_seq;
+  int Hkv_rows;  // rows per (page or sequence) per head: PF_PAGE_SIZE or max_seq
+  const int32_t* page_table;
+  int pages_per_seq;
+  int num_pages;
+  int32_t* new_len;
+  int32_t* err;
+};
+
+cudaError_t launch_kv_commit(const CommitArgs& a, cudaStream_t s, int num_sms, bool pdl);
+
+// Raise a kernel's dynamic shared-memory limit once per device (never while
+// a stream is being captured after the first call on that device).
+inline cudaError_t ensure_smem_limit(const void* func, int bytes, int* per_device) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev >= 0 && dev < 64 && per_device[dev] >= bytes) return cudaSuccess;
+  e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess && dev >= 0 && dev < 64) per_device[dev] = bytes;
+  return e;
+}
+
+// Shared launch helper: optional cluster dimension and programmatic
+// dependent launch.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_ex(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                      cudaStream_t s, int cluster_x, bool pdl, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attrs[2];
+  int na = 0;
+  if (cluster_x > 1) {
+    attrs[na].id = cudaLaunchAttributeClusterDimension;
+    attrs[na].val.clusterDim.x = cluster_x;
+    attrs[na].val.clusterDim.y = 1;
+    attrs[na].val.clusterDim.z = 1;
+    ++na;
+  }
+  if (pdl) {
+    attrs[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attrs[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
+  cfg.attrs = attrs;
+  cfg.numAttrs = na;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+}  // namespace pf

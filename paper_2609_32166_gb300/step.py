@@ -1,0 +1,204 @@
+"""Device buffers and call sequence of one verify step.
+
+``VerifyStep`` owns the device tensors of one workload (queries, proposal
+K/V and prefix caches of every layer, hidden states, LM-head weight, tree
+structure, outputs) and issues the three C-ABI calls of the step:
+``pf_verify_attention`` once per layer, ``pf_lmhead_accept`` once, and
+``pf_kv_commit`` once for all layers.  torch provides device memory and
+streams only; nothing here computes any part of the step.
+
+Layouts (row-major):
+  q, attn_out     [L, T, Hq, D]
+  tree_k, tree_v  [L, T, Hkv, D]
+  cache_k/v       [L, B, Hkv, S, D] (contiguous) or [L, pages, Hkv, 16, D] (paged)
+  mask            [T, 2] uint64 ancestor bitmaps (pf_tree_prepare)
+  hidden          [T, H];  weight [V, H]
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import binding as pb
+from . import inputs as I
+
+
+def _dev(arr: np.ndarray, dtype: str, device) -> torch.Tensor:
+    """Host array (bf16 bit patterns or float32/ints) -> device tensor."""
+    if dtype == "bf16":
+        t = torch.from_numpy(np.ascontiguousarray(arr).view(np.int16)).view(torch.bfloat16)
+    else:
+        t = torch.from_numpy(np.ascontiguousarray(arr))
+    return t.to(device)
+
+
+def _torch_dtype(dtype: str):
+    return torch.bfloat16 if dtype == "bf16" else torch.float32
+
+
+def host_bits(t: torch.Tensor) -> np.ndarray:
+    """Device tensor -> host numpy of the same bits (uint16 for bf16)."""
+    t = t.detach().cpu().contiguous()
+    if t.dtype == torch.bfloat16:
+        return t.view(torch.int16).numpy().view(np.uint16)
+    return t.numpy()
+
+
+class VerifyStep:
+    """One workload's device state.  ``layers`` may restrict the layer count
+    (parity tests use a few layers of a full-size workload)."""
+
+    def __init__(self, w: I.Workload, batch: I.Batch, tokens: np.ndarray, layers: int = None,
+                 device: str = "cuda", weight: np.ndarray = None, hidden: np.ndarray = None):
+        self.w, self.batch = w, batch
+        self.L = layers if layers is not None else w.layers
+        self.device = device
+        td = _torch_dtype(w.dtype)
+        T, B = batch.total_nodes, w.batch
+        self.T = T
+        self.max_nodes = max(len(p) for p in batch.parents)
+        self.max_prefix = int(batch.prefix_lens.max())
+
+        masks = []
+        for p in batch.parents:
+            _, m = pb.pf_tree_prepare(p)
+            masks.append(m)
+        mask = np.concatenate(masks, axis=0).astype(np.uint64)
+        self.mask = torch.from_numpy(mask.view(np.int64)).to(device)
+        self.cu_nodes = torch.from_numpy(batch.cu_nodes).to(device)
+        self.prefix_len = torch.from_numpy(batch.prefix_lens.astype(np.int32)).to(device)
+        self.parent = torch.from_numpy(batch.parent_flat).to(device)
+        self.tokens = torch.from_numpy(np.asarray(tokens, dtype=np.int32)).to(device)
+        self.page_table = (torch.from_numpy(batch.page_table).to(device)
+                           if batch.page_table is not None else None)
+
+        shp = I.cache_shape(w, batch)
+        self.q = torch.empty((self.L, T, w.hq, w.d), dtype=td, device=device)
+        self.tree_k = torch.empty((self.L, T, w.hkv, w.d), dtype=td, device=device)
+        self.tree_v = torch.empty_like(self.tree_k)
+        self.cache_k = torch.zeros((self.L,) + shp, dtype=td, device=device)
+        self.cache_v = torch.zeros_like(self.cache_k)
+        for l in range(self.L):
+            self.q[l] = _dev(I.layer_q(w, batch, l), w.dtype, device)
+            tk, tv = I.layer_tree_kv(w, batch, l)
+            self.tree_k[l] = _dev(tk, w.dtype, device)
+            self.tree_v[l] = _dev(tv, w.dtype, device)
+            ck = np.zeros(shp, dtype=np.uint16 if w.dtype == "bf16" else np.float32)
+            cv = np.zeros_like(ck)
+            for s in range(B):
+                pk, pv = I.layer_prefix_kv(w, batch, l, s)
+                I.place_prefix(w, batch, ck, s, pk)
+                I.place_prefix(w, batch, cv, s, pv)
+            self.cache_k[l] = _dev(ck, w.dtype, device)
+            self.cache_v[l] = _dev(cv, w.dtype, device)
+        self.attn_out = torch.zeros_like(self.q)
+        if hidden is None:
+            hidden = I.hidden_states(w, batch)
+        if weight is None:
+            weight = I.lm_weight(w, batch.seed)
+        self.hidden = _dev(hidden, w.dtype, device)
+        self.weight = _dev(weight, w.dtype, device)
+
+        i32 = dict(dtype=torch.int32, device=device)
+        self.argmax = torch.full((T,), -1, **i32)
+        self.max_logit = torch.zeros((T,), dtype=torch.float32, device=device)
+        self.accept_len = torch.full((B,), -1, **i32)
+        self.path = torch.full((B, self.max_nodes), -1, **i32)
+        self.out_tokens = torch.full((B, self.max_nodes), -1, **i32)
+        self.last_node = torch.full((B,), -1, **i32)
+        self.new_len = torch.zeros((B,), **i32)
+        self.err = torch.zeros((1,), **i32)
+        self.ws_bytes = pb.pf_lmhead_accept_workspace_size()
+        self.workspace = torch.zeros((self.ws_bytes,), dtype=torch.uint8, device=device)
+        self._build_descs()
+
+    # ------------------------------------------------------------------ descs
+    def _view(self, l: int) -> pb.pf_kv_view:
+        w, b = self.w, self.batch
+        v = pb.pf_kv_view()
+        v.layout = pb.PF_KV_PAGED if w.layout == "paged" else pb.PF_KV_CONTIGUOUS
+        v.k = self.cache_k[l].data_ptr()
+        v.v = self.cache_v[l].data_ptr()
+        v.max_seq = b.max_seq if w.layout == "contiguous" else 0
+        if w.layout == "paged":
+            v.num_pages = b.num_pages
+            v.page_table = self.page_table.data_ptr()
+            v.pages_per_seq = int(b.page_table.shape[1])
+        return v
+
+    def _build_descs(self):
+        w = self.w
+        dt = pb.PF_BF16 if w.dtype == "bf16" else pb.PF_F32
+        self.attn_descs = []
+        for l in range(self.L):
+            d = pb.pf_attn_desc()
+            d.dtype, d.batch = dt, w.batch
+            d.n_q_heads, d.n_kv_heads, d.head_dim = w.hq, w.hkv, w.d
+            d.scale = 0.0
+            d.total_nodes, d.max_nodes, d.max_prefix_len = self.T, self.max_nodes, self.max_prefix
+            d.cu_nodes, d.prefix_len = self.cu_nodes.data_ptr(), self.prefix_len.data_ptr()
+            d.q = self.q[l].data_ptr()
+            d.tree_k, d.tree_v = self.tree_k[l].data_ptr(), self.tree_v[l].data_ptr()
+            d.mask = self.mask.data_ptr()
+            d.cache = self._view(l)
+            d.out = self.attn_out[l].data_ptr()
+            d.error_flag = self.err.data_ptr()
+            self.attn_descs.append(d)
+        d = pb.pf_lm_desc()
+        d.dtype, d.batch, d.hidden, d.vocab = dt, w.batch, w.hidden, w.vocab
+        d.total_nodes, d.max_nodes = self.T, self.max_nodes
+        d.cu_nodes = self.cu_nodes.data_ptr()
+        d.hidden_states, d.weight = self.hidden.data_ptr(), self.weight.data_ptr()
+        d.tokens, d.parent = self.tokens.data_ptr(), self.parent.data_ptr()
+        d.argmax, d.max_logit = self.argmax.data_ptr(), self.max_logit.data_ptr()
+        d.accept_len, d.path = self.accept_len.data_ptr(), self.path.data_ptr()
+        d.out_tokens, d.last_node = self.out_tokens.data_ptr(), self.last_node.data_ptr()
+        d.error_flag = self.err.data_ptr()
+        self.lm_desc = d
+        c = pb.pf_commit_desc()
+        c.dtype, c.batch, c.n_layers = dt, w.batch, self.L
+        c.n_kv_heads, c.head_dim = w.hkv, w.d
+        c.total_nodes, c.max_nodes, c.max_prefix_len = self.T, self.max_nodes, self.max_prefix
+        c.cu_nodes, c.prefix_len = self.cu_nodes.data_ptr(), self.prefix_len.data_ptr()
+        c.accept_len, c.path = self.accept_len.data_ptr(), self.path.data_ptr()
+        c.tree_k, c.tree_v = self.tree_k.data_ptr(), self.tree_v.data_ptr()
+        c.tree_layer_stride = self.tree_k[0].numel()
+        c.cache = self._view(0)
+        c.cache_layer_stride = self.cache_k[0].numel()
+        c.new_len = self.new_len.data_ptr()
+        c.error_flag = self.err.data_ptr()
+        self.commit_desc = c
+
+    # ------------------------------------------------------------------ calls
+    @staticmethod
+    def _stream(stream):
+        return torch.cuda.current_stream().cuda_stream if stream is None else int(stream)
+
+    def attention(self, layer: int, stream=None):
+        pb.pf_verify_attention(self.attn_descs[layer], self._stream(stream))
+
+    def lmhead(self, stream=None):
+        pb.pf_lmhead_accept(self.lm_desc, self.workspace.data_ptr(), self.ws_bytes,
+                            self._stream(stream))
+
+    def commit(self, stream=None):
+        pb.pf_kv_commit(self.commit_desc, self._stream(stream))
+
+    def step(self, stream=None):
+        s = self._stream(stream)
+        for l in range(self.L):
+            pb.pf_verify_attention(self.attn_descs[l], s)
+        pb.pf_lmhead_accept(self.lm_desc, self.workspace.data_ptr(), self.ws_bytes, s)
+        pb.pf_kv_commit(self.commit_desc, s)
+
+    def launches_per_step(self) -> int:
+        return self.L + 2
+
+    # ------------------------------------------------------------------ results
+    def results(self) -> dict:
+        torch.cuda.synchronize()
+        return dict(argmax=self.argmax.cpu().numpy(), max_logit=self.max_logit.cpu().numpy(),
+                    accept_len=self.accept_len.cpu().numpy(), path=self.path.cpu().numpy(),
+                    out_tokens=self.out_tokens.cpu().numpy(),
+                    last_node=self.last_node.cpu().numpy(), new_len=self.new_len.cpu().numpy(),
+                    err=int(self.err.item()))

@@ -1,0 +1,560 @@
+"""Benchmark of the verify step (tree attention x L layers, LM head with
+greedy acceptance, KV commit) on seeded synthetic inputs.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+    python bench.py --impl reference ...      # the fp64 CPU oracle, timed
+
+Prints one JSON line.  The metric is accepted tokens/s of whole verify steps
+(sum over sequences of accepted drafts + 1 bonus token, divided by the step
+time), with the attention time per layer and the step's achieved HBM
+bandwidth alongside.  Every step is one CUDA-graph segment: L attention
+launches, one LM-head launch, one commit launch.  Between steps a 256 MB
+memset evicts L2; each step is bracketed by its own CUDA events, so the
+flush is outside the measured time.  Multi-GPU runs are independent
+replicas (one process per GPU under torchrun); the value is the sum of
+tokens over ranks divided by the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "verify-step µs/layer & accepted tokens/s; achieved HBM GB/s vs ~8 TB/s peak"
+DEFAULT_WORKLOAD = "2b-bf16-chain16"
+L2_FLUSH_BYTES = 256 << 20
+PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "lmhead_traffic.txt")
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=400)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    p.add_argument("--seed", type=int, default=0)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--cpu-worker", default=None, help=argparse.SUPPRESS)
+    return p.parse_args()
+
+
+# ---------------------------------------------------------------------------
+# algorithmic bytes
+# ---------------------------------------------------------------------------
+def step_bytes(w, batch, accept_lens):
+    es = 2 if w.dtype == "bf16" else 4
+    T = batch.total_nodes
+    prefix = int(np.sum(batch.prefix_lens))
+    attn = (2 * prefix * w.hkv * w.d + 2 * T * w.hkv * w.d + 2 * T * w.hq * w.d) * es + T * 16
+    lm = (w.vocab * w.hidden + T * w.hidden) * es + T * 4 * 4
+    rows = int(np.sum(np.asarray(accept_lens) + 1))
+    commit = 2 * rows * w.hkv * w.d * es * 2 * w.layers
+    return attn, lm, commit
+
+
+def lmhead_source_fingerprint():
+    h = hashlib.sha256()
+    for f in ("lmhead.cu", "pf_ptx.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2609_32166_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload):
+    """dram bytes per LM-head launch from the committed ncu summary, if it was
+    taken on the current kernel source for this workload; else None."""
+    if not os.path.exists(PROFILE_TRAFFIC):
+        return None
+    kv = {}
+    for line in open(PROFILE_TRAFFIC):
+        if ":" in line and not line.startswith("#"):
+            k, v = line.split(":", 1)
+            kv[k.strip()] = v.strip()
+    if kv.get("source_fingerprint") != lmhead_source_fingerprint():
+        return None
+    if kv.get("workload") != workload:
+        return None
+    try:
+        return float(kv["dram_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
+# ---------------------------------------------------------------------------
+# clocks
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append(dict(sm=float(parts[1]), max=float(parts[2]),
+                                 power=float(parts[3]) if parts[3] not in ("[N/A]", "N/A") else 0.0,
+                                 hw=parts[5], hwt=parts[6], swt=parts[7], pcap=parts[8]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        pmax = max(r["power"] for r in rows)
+        load = [r for r in rows if r["power"] >= 0.5 * pmax] or rows
+        reasons = set()
+        for r in rows:
+            for key, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"),
+                              ("swt", "sw_thermal_slowdown"), ("pcap", "sw_power_cap")):
+                if r[key].lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(r["sm"] for r in load),
+                "sm_max_mhz": max(r["max"] for r in rows), "reasons": sorted(reasons),
+                "samples": len(rows), "samples_under_load": len(load),
+                "power_w_max": pmax}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (cpu_baseline and --impl reference); runs in a fresh
+# interpreter so its BLAS thread count is set before numpy loads
+# ---------------------------------------------------------------------------
+def cpu_worker(spec: dict) -> dict:
+    from oracle import accept as OAcc
+    from oracle import attention as OA
+    from oracle import commit as OC
+    from oracle import lmhead as OL
+    from paper_2609_32166_gb300 import inputs as I
+
+    w = I.WORKLOADS[spec["workload"]]
+    batch = I.make_batch(w, spec["seed"])
+    f = (lambda x: I.bf16_bits_to_f32(x)) if w.dtype == "bf16" else (lambda x: x)
+    hidden = f(I.hidden_states(w, batch))
+    weight = f(I.lm_weight(w, batch.seed))
+    nl = spec["layers_sample"]
+    layers = []
+    for l in range(nl):
+        q = f(I.layer_q(w, batch, l))
+        tk, tv = (f(x) for x in I.layer_tree_kv(w, batch, l))
+        pre = [tuple(f(x) for x in I.layer_prefix_kv(w, batch, l, s)) for s in range(w.batch)]
+        layers.append((q, tk, tv, pre))
+    cu = batch.cu_nodes
+    ends = I.step_forced_ends(batch, 50)
+    counter = [0]
+
+    def one_step():
+        g = counter[0] % len(ends)
+        counter[0] += 1
+        t0 = time.perf_counter()
+        for (q, tk, tv, pre) in layers:
+            for s in range(w.batch):
+                c0, c1 = int(cu[s]), int(cu[s + 1])
+                OA.tree_attention(q[c0:c1], pre[s][0], pre[s][1], tk[c0:c1], tv[c0:c1],
+                                  batch.parents[s])
+        t_attn = time.perf_counter() - t0
+        t1 = time.perf_counter()
+        am, _, _ = OL.greedy(OL.logits(hidden, weight))
+        tokens = I.plant_tokens(batch, am, ends[g], salt=g)   # this step's proposal
+        acc = []
+        for s in range(w.batch):
+            c0, c1 = int(cu[s]), int(cu[s + 1])
+            acc.append(OAcc.accept_walk(batch.parents[s], tokens[c0:c1], am[c0:c1]))
+        t_lm = time.perf_counter() - t1
+        t2 = time.perf_counter()
+        for (q, tk, tv, pre) in layers:
+            for s in range(w.batch):
+                c0, c1 = int(cu[s]), int(cu[s + 1])
+                P = int(batch.prefix_lens[s])
+                rows = np.zeros((w.hkv, P + w.nodes, w.d), dtype=np.float32)
+                OC.commit_rows(rows, P, acc[s][1], tk[c0:c1])
+                OC.commit_rows(rows, P, acc[s][1], tv[c0:c1])
+        t_commit = time.perf_counter() - t2
+        scale = w.layers / nl
+        est = (t_attn + t_commit) * scale + t_lm
+        return est, sum(a[0] + 1 for a in acc)
+
+    times, toks = [], []
+    n = spec.get("steps")
+    if n is None:   # time-bounded sample for cpu_baseline
+        t_start = time.perf_counter()
+        while (time.perf_counter() - t_start < spec["budget_s"] or not times) and len(times) < 50:
+            est, tok = one_step()
+            times.append(est)
+            toks.append(tok)
+    else:
+        for _ in range(spec["warmup"]):
+            one_step()
+        counter[0] = 0
+        for _ in range(n):
+            est, tok = one_step()
+            times.append(est)
+            toks.append(tok)
+    return dict(step_s=float(np.mean(times)), steps=len(times),
+                tokens_per_step=float(np.mean(toks)))
+
+
+def run_cpu_worker(spec: dict) -> dict:
+    cores = os.cpu_count() or 1
+    env = dict(os.environ)
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        env[k] = str(cores)
+    env["CUDA_VISIBLE_DEVICES"] = ""
+    r = subprocess.run([sys.executable, os.path.abspath(__file__), "--cpu-worker", json.dumps(spec)],
+                       capture_output=True, text=True, env=env, cwd=ROOT)
+    if r.returncode != 0:
+        raise RuntimeError("CPU oracle worker failed:\n" + r.stderr[-2000:])
+    out = json.loads(r.stdout.strip().splitlines()[-1])
+    out["cores"] = cores
+    return out
+
+
+def cpu_sample_text(w, nl):
+    return (f"whole verify steps of {w.name} in fp64 numpy: attention of {nl} of {w.layers} "
+            f"layers (time scaled by {w.layers}/{nl}), full LM head ({w.vocab}x{w.hidden}), "
+            f"acceptance, commit")
+
+
+# ---------------------------------------------------------------------------
+# reference arm: the oracle as it stands, on the host cores
+# ---------------------------------------------------------------------------
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from paper_2609_32166_gb300 import inputs as I
+    w = I.WORKLOADS[args.workload]
+    nl = 1
+    spec = dict(workload=args.workload, seed=args.seed, layers_sample=nl, steps=args.steps,
+                warmup=args.warmup)
+    t0 = time.perf_counter()
+    r = run_cpu_worker(spec)
+    wall = time.perf_counter() - t0
+    value = r["tokens_per_step"] / r["step_s"]
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": r["step_s"] * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded generator)",
+        "config": config_dict(w, args),
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": r["cores"],
+                         "kind": "oracle", "sample": cpu_sample_text(w, nl)},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+        "wall_s": wall,
+    }
+    print(json.dumps(line))
+
+
+def config_dict(w, args):
+    return {"workload": w.name, "layers": w.layers, "batch": w.batch, "q_heads": w.hq,
+            "kv_heads": w.hkv, "head_dim": w.d, "hidden": w.hidden, "vocab": w.vocab,
+            "prefix": list(w.prefix), "nodes": w.nodes, "tree": w.tree, "kv_layout": w.layout,
+            "seed": args.seed,
+            "l2": "256 MB memset between steps (outside the per-step events); "
+                  "step inputs also exceed the 129 MB L2"}
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+def main():
+    args = parse()
+    if args.cpu_worker is not None:
+        print(json.dumps(cpu_worker(json.loads(args.cpu_worker))))
+        return
+    if args.impl == "reference":
+        run_reference(args)
+        return
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    cpu_base = None
+    from paper_2609_32166_gb300 import inputs as I
+    w = I.WORKLOADS[args.workload]
+    nl_cpu = 1
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        # before any CUDA call in this process
+        cpu_base = run_cpu_worker(dict(workload=args.workload, seed=args.seed,
+                                       layers_sample=nl_cpu, budget_s=12.0))
+
+    import torch
+    import torch.distributed as dist
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl")
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_32166_gb300.step import VerifyStep
+
+    batch = I.make_batch(w, args.seed)
+    vs = VerifyStep(w, batch, np.zeros(batch.total_nodes, np.int32))
+    # plant the draft tokens from the model's own greedy predictions so the
+    # accepted length is the planted one
+    vs.lmhead()
+    torch.cuda.synchronize()
+    greedy = vs.argmax.cpu().numpy()
+    # every step verifies a new proposal: the planted accepted path of step k
+    # follows the workload's rule, drawn from a seeded per-step stream
+    K = args.steps
+    G = max(d for d in range(1, min(K, 50) + 1) if K % d == 0)
+    ends = I.step_forced_ends(batch, G)
+    depth = [I.node_depths(p) for p in batch.parents]
+    planned = [int(sum(depth[b][e[b]] + 1 for b in range(w.batch))) for e in ends]
+    tok_table = torch.from_numpy(np.stack([I.plant_tokens(batch, greedy, e, salt=g)
+                                           for g, e in enumerate(ends)])).cuda()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+
+    stream = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        for k in range(max(args.warmup, 3)):
+            flush.zero_()
+            vs.tokens.copy_(tok_table[k % G])
+            vs.step()
+            stream.synchronize()
+            got = int((vs.accept_len + 1).sum().item())
+            assert got == planned[k % G], (k, got, planned[k % G])
+    accepted_steps = [planned[k % G] for k in range(K)]
+
+    # one graph = G steps; each step: flush, tokens | e0 attention e1 lmhead e2 commit e3
+    per_step, attn_t, lm_t, commit_t = [], [], [], []
+
+    def collect(e):
+        per_step.append(e[0].elapsed_time(e[3]))
+        attn_t.append(e[0].elapsed_time(e[1]))
+        lm_t.append(e[1].elapsed_time(e[2]))
+        commit_t.append(e[2].elapsed_time(e[3]))
+
+    try:
+        torch.cuda.Event(enable_timing=True, external=True)
+        graph_events = True
+    except TypeError:
+        graph_events = False
+    clocks = ClockSampler(torch.cuda.current_device())
+    if graph_events:
+        R = K // G
+        ev = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(4)]
+              for _ in range(G)]
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            s = torch.cuda.current_stream()
+            for g in range(G):
+                flush.zero_()
+                vs.tokens.copy_(tok_table[g])
+                ev[g][0].record(s)
+                for l in range(vs.L):
+                    vs.attention(l, s.cuda_stream)
+                ev[g][1].record(s)
+                vs.lmhead(s.cuda_stream)
+                ev[g][2].record(s)
+                vs.commit(s.cuda_stream)
+                ev[g][3].record(s)
+        with torch.cuda.stream(stream):
+            graph.replay()   # untimed: uploads the graph
+        stream.synchronize()
+        clocks.start()
+        time.sleep(0.3)
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        with torch.cuda.stream(stream):
+            for r in range(R):
+                graph.replay()
+                # the event nodes hold this replay's timestamps: read them
+                # before the next replay overwrites them
+                stream.synchronize()
+                for g in range(G):
+                    collect(ev[g])
+    else:
+        # torch without external graph events: one graph per part, events
+        # recorded between graph launches
+        parts = []
+        for fn in (lambda st: [vs.attention(l, st) for l in range(vs.L)],
+                   lambda st: vs.lmhead(st), lambda st: vs.commit(st)):
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr, stream=stream):
+                fn(torch.cuda.current_stream().cuda_stream)
+            parts.append(gr)
+        with torch.cuda.stream(stream):
+            for gr in parts:
+                gr.replay()
+        stream.synchronize()
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
+        clocks.start()
+        time.sleep(0.3)
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        with torch.cuda.stream(stream):
+            for k in range(K):
+                flush.zero_()
+                vs.tokens.copy_(tok_table[k % G])
+                ev[k][0].record(stream)
+                parts[0].replay()
+                ev[k][1].record(stream)
+                parts[1].replay()
+                ev[k][2].record(stream)
+                parts[2].replay()
+                ev[k][3].record(stream)
+        stream.synchronize()
+        for k in range(K):
+            collect(ev[k])
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    assert len(per_step) == K
+    t_total_ms = float(np.sum(per_step))
+    if world > 1:
+        tt = torch.tensor([t_total_ms], device="cuda")
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        t_total_ms = float(tt.item())
+    res = vs.results()
+    assert res["err"] == 0, f"device error flag {res['err']}"
+    assert int(np.sum(res["accept_len"] + 1)) == accepted_steps[-1]
+
+    ms_step = t_total_ms / K
+    accepted = float(np.mean(accepted_steps))
+    value = world * float(np.sum(accepted_steps)) / (t_total_ms / 1e3)
+    attn_b, lm_b, commit_b = step_bytes(w, batch, res["accept_len"])
+    attn_b_layer = attn_b
+    step_b = attn_b * w.layers + lm_b + commit_b
+    lm_ms = float(np.mean(lm_t))
+    attn_ms = float(np.mean(attn_t))
+    peaks = {}
+    pk = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(pk):
+        peaks = json.load(open(pk))
+    hbm_peak = peaks.get("hbm_gbs", 6800.0)
+    peak_src = "measured" if "hbm_gbs" in peaks else "fallback"
+    lm_gbs = lm_b / (lm_ms * 1e-3) / 1e9
+
+    e2e = None if args.no_e2e else run_e2e(vs, w, batch, K, stream, flush, world, tok_table,
+                                           planned)
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
+        "data": "synthetic (seeded generator, shapes of the named workload)",
+        "config": config_dict(w, args),
+        "accepted_tokens_per_step": accepted,
+        "us_per_layer_attention": attn_ms * 1e3 / w.layers,
+        "us_lmhead": lm_ms * 1e3, "us_commit": float(np.mean(commit_t)) * 1e3,
+        "step_hbm_gbs": step_b / (ms_step * 1e-3) / 1e9,
+        "step_hbm_frac": step_b / (ms_step * 1e-3) / 1e9 / hbm_peak,
+        "step_bytes": step_b,
+        "roofline": {"kernel": "pf_lmhead_accept", "bound": "hbm", "achieved": lm_gbs,
+                     "peak": hbm_peak, "unit": "GB/s", "frac": lm_gbs / hbm_peak,
+                     "peak_source": f"{peak_src} (copy bandwidth)",
+                     "algorithmic_bytes": lm_b,
+                     "traffic": profiled_traffic(w.name)},
+        "attention_roofline": {"achieved": attn_b_layer * w.layers / (attn_ms * 1e-3) / 1e9,
+                               "unit": "GB/s", "frac": attn_b_layer * w.layers /
+                               (attn_ms * 1e-3) / 1e9 / hbm_peak},
+        "gpu_launches": K * vs.launches_per_step(),
+        "timing": ("CUDA graph of G steps, external event nodes around each step's parts"
+                   if graph_events else "one CUDA graph per part, events between graph launches"),
+        "clocks": clk,
+        "e2e": e2e,
+    }
+    if cpu_base is not None:
+        line["cpu_baseline"] = {"value": cpu_base["tokens_per_step"] / cpu_base["step_s"],
+                                "unit": "tokens/s", "cores": cpu_base["cores"], "kind": "oracle",
+                                "sample": cpu_sample_text(w, nl_cpu) +
+                                f"; {cpu_base['steps']} step(s) timed"}
+    print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def run_e2e(vs, w, batch, K, stream, flush, world, tok_table, planned):
+    """Same metric through host buffers: every step copies its inputs from
+    pinned host memory, runs the step and reads the accepted tokens back."""
+    import torch
+    names = ["q", "tree_k", "tree_v", "hidden", "tokens", "parent", "mask", "cu_nodes",
+             "prefix_len"]
+    host = {n: getattr(vs, n).detach().cpu().pin_memory() for n in names}
+    host_tokens = [t.cpu().pin_memory() for t in tok_table]
+    outs = {n: torch.empty_like(getattr(vs, n), device="cpu").pin_memory()
+            for n in ("accept_len", "out_tokens", "new_len")}
+    h2d = sum(t.numel() * t.element_size() for t in host.values())
+    d2h = sum(t.numel() * t.element_size() for t in outs.values())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        vs.step(torch.cuda.current_stream().cuda_stream)
+    with torch.cuda.stream(stream):
+        g.replay()
+    stream.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    times = []
+    tok = 0
+    n = min(K, 200)
+    with torch.cuda.stream(stream):
+        for k in range(n):
+            flush.zero_()
+            host["tokens"] = host_tokens[k % len(host_tokens)]
+            e0.record(stream)
+            for name, t in host.items():
+                getattr(vs, name).copy_(t, non_blocking=True)
+            g.replay()
+            for name, t in outs.items():
+                t.copy_(getattr(vs, name), non_blocking=True)
+            e1.record(stream)
+            stream.synchronize()
+            times.append(e0.elapsed_time(e1))
+            got = int((outs["accept_len"] + 1).sum())
+            assert got == planned[k % len(planned)]
+            tok += got
+    t = float(np.sum(times))
+    return {"value": world * tok / (t * 1e-3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "steps": n, "ms_per_step": t / n}
+
+
+if __name__ == "__main__":
+    main()

@@ -146,7 +146,18 @@ typedef struct pf_attn_desc {
   pf_kv_view cache;            /* this layer's prefix cache                  */
   void* out;                   /* device [T][Hq][D]                          */
   int32_t* error_flag;         /* optional device int32                      */
+  int32_t flags;               /* PF_ATTN_* bits, 0 = none                   */
 } pf_attn_desc;
+
+/* PF_ATTN_EARLY_PREFETCH: the prefix cache, page_table, cu_nodes, prefix_len
+ * and mask were all written before the kernel that precedes this call in the
+ * stream started (for example: layers after the first of one verify step,
+ * whose cache only the previous step's pf_kv_commit wrote).  The kernel then
+ * requests its cache tiles before waiting for that preceding kernel to
+ * finish (programmatic dependent launch); q, tree_k and tree_v are still
+ * read only after it finishes.  Leave it clear when the preceding kernel may
+ * write any of those inputs. */
+#define PF_ATTN_EARLY_PREFETCH 1
 
 PF_API pf_status pf_verify_attention(const pf_attn_desc* d, void* stream);
 

@@ -11,6 +11,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
+#include <algorithm>
 #include <string>
 
 #include "pf_internal.h"
@@ -106,6 +107,56 @@ pf_status check_cache_view(const pf_kv_view& c, int need_rows, const char* who) 
     return fail(PF_ERR_SHAPE, "%s: unknown cache layout %d", who, c.layout);
   }
   return PF_OK;
+}
+
+// Launch shape of the bf16 attention: query rows per CTA (32, 64 or 128)
+// and KV splits per cluster (<= 16).  Small problems take small row blocks
+// and wide clusters so that enough SMs stream the cache; large ones keep
+// 128-row blocks so each K/V tile serves more rows.  A cluster wider than 8
+// is used only if the device can schedule it.
+int max_cluster_for(int bm, int D, int want) {
+  static int cache[64][3][2][17];
+  int dev = 0;
+  cudaGetDevice(&dev);
+  const int bi = bm == 32 ? 0 : bm == 64 ? 1 : 2, di = D == 64 ? 0 : 1;
+  int w = want;
+  while (w > 8) {
+    int& c = cache[dev & 63][bi][di][w];
+    if (c == 0) c = pf::attention_cluster_fits(D, bm, w) ? 1 : -1;
+    if (c > 0) break;
+    --w;
+  }
+  return w;
+}
+
+void choose_attention_shape(pf::AttnArgs& a, int max_prefix_len, int sms) {
+  const int max_tiles = (max_prefix_len + 63) / 64 + (a.max_nodes + 63) / 64;
+  const int bms[3] = {128, 64, 32};
+  int pick = 32;
+  for (int bm : bms) {
+    if (a.G > bm) break;
+    const int rb = (a.max_nodes + bm / a.G - 1) / (bm / a.G);
+    const int base = a.B * a.Hkv * rb;
+    const int per_sm = bm == 128 ? 1 : 2;
+    if (base * std::min(16, max_tiles) >= sms * per_sm || bm == 32) {
+      pick = bm;
+      break;
+    }
+  }
+  if (a.G > pick) pick = 128;
+  if (const char* e = getenv("PF_ATTN_BM")) pick = atoi(e);
+  a.bm = pick;
+  a.nb = pick / a.G;
+  a.rb_count = (a.max_nodes + a.nb - 1) / a.nb;
+  const int base = a.B * a.Hkv * a.rb_count;
+  const int per_sm = pick == 128 ? 1 : 2;
+  int splits = (sms * per_sm) / base;
+  if (const char* e = getenv("PF_ATTN_SPLITS")) splits = atoi(e);
+  if (splits > 16) splits = 16;
+  if (splits > max_tiles) splits = max_tiles;
+  if (splits < 1) splits = 1;
+  if (splits > 8) splits = max_cluster_for(pick, a.D, splits);
+  a.splits = splits;
 }
 
 }  // namespace
@@ -210,23 +261,16 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
     return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
   }
 
-  a.nb = 128 / G;
-  a.rb_count = (d->max_nodes + a.nb - 1) / a.nb;
-  const int base = a.B * a.Hkv * a.rb_count;
-  const int max_tiles = (d->max_prefix_len + 63) / 64 + (d->max_nodes + 63) / 64;
-  int splits = sms / base;
-  if (const char* e = getenv("PF_ATTN_SPLITS")) splits = atoi(e);
-  if (splits > 8) splits = 8;
-  if (splits > max_tiles) splits = max_tiles;
-  if (splits < 1) splits = 1;
-  a.splits = splits;
-
+  if (d->flags & ~PF_ATTN_EARLY_PREFETCH)
+    return fail(PF_ERR_SHAPE, "%s: unknown flags 0x%x", who, d->flags);
+  a.flags = d->flags;
+  choose_attention_shape(a, d->max_prefix_len, sms);
   pf::AttnMaps m;
   const cuuint64_t es = 2;
   {
     cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)a.Hq, (cuuint64_t)a.T};
     cuuint64_t str[2] = {D * es, (cuuint64_t)a.Hq * D * es};
-    cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)a.nb};
+    cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)a.nb};  // nb * G <= bm rows
     if ((st = make_map(&m.q, 3, d->q, dims, str, box, "q")) != PF_OK) return st;
   }
   {

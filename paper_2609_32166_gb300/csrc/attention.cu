@@ -25,34 +25,34 @@ namespace pf {
 namespace {
 
 constexpr int kBN = 64;         // tokens per KV tile
-constexpr int kRows = 128;      // query rows per CTA (8 warps x 16)
-constexpr int kThreads = 256;
 constexpr int kStages = 3;
 
-template <int D>
+// Shared-memory plan of one CTA with BM query rows (BM / 16 warps).
+template <int D, int BM>
 struct AttnSmem {
+  static constexpr int kThreads = BM * 2;
   static constexpr int kHalves = D / 64;
   static constexpr int kTileBytes = kBN * D * 2;       // one K or V tile
   static constexpr int kStageBytes = 2 * kTileBytes;   // K + V
-  static constexpr int kQBytes = kRows * D * 2;
+  static constexpr int kQBytes = BM * D * 2;
   static constexpr int kRedOff = kStages * kStageBytes + kQBytes;
-  static constexpr int kBarOff = kRedOff + 2 * kRows * 4;
+  static constexpr int kBarOff = kRedOff + 2 * BM * 4;
   static constexpr int kTotal = kBarOff + (kStages + 1) * 8 + 16;
   static constexpr int kOStride = D + 4;               // fp32 partial-O row pitch
-  static_assert(kRows * kOStride * 4 <= kRedOff, "partial O must fit the staging area");
+  static_assert(BM * kOStride * 4 <= kStages * kStageBytes, "partial O must fit the KV ring");
 };
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
 }
 
-template <int D>
+template <int D, int BM>
 __device__ __forceinline__ void issue_kv_tile(const AttnArgs& a, const CUtensorMap* tm_ck,
                                               const CUtensorMap* tm_cv, const CUtensorMap* tm_tk,
                                               const CUtensorMap* tm_tv, uint8_t* stage,
                                               uint32_t bar, int t, int n_ptiles, int b, int g,
                                               int node0, int P) {
-  using S = AttnSmem<D>;
+  using S = AttnSmem<D, BM>;
   uint8_t* sk = stage;
   uint8_t* sv = stage + S::kTileBytes;
   if (t < n_ptiles) {
@@ -90,14 +90,15 @@ __device__ __forceinline__ void issue_kv_tile(const AttnArgs& a, const CUtensorM
   }
 }
 
-template <int D>
-__global__ void __launch_bounds__(kThreads, 1)
+template <int D, int BM>
+__global__ void __launch_bounds__(BM * 2, 1)
     attn_bf16_kernel(const __grid_constant__ CUtensorMap tm_q,
                      const __grid_constant__ CUtensorMap tm_tk,
                      const __grid_constant__ CUtensorMap tm_tv,
                      const __grid_constant__ CUtensorMap tm_ck,
                      const __grid_constant__ CUtensorMap tm_cv, const AttnArgs a) {
-  using S = AttnSmem<D>;
+  using S = AttnSmem<D, BM>;
+  constexpr int kThreads = S::kThreads;
   constexpr int KS = D / 16;   // k-steps of QK^T
   constexpr int NT = D / 8;    // n8 tiles of O
   extern __shared__ uint8_t smem_raw[];
@@ -105,9 +106,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* sKV = smem;
   uint8_t* sQ = smem + kStages * S::kStageBytes;
   float* sM = reinterpret_cast<float*>(smem + S::kRedOff);
-  float* sL = sM + kRows;
+  float* sL = sM + BM;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S::kBarOff);
-  float* sO = reinterpret_cast<float*>(smem);  // reused after the KV loop
+  float* sO = reinterpret_cast<float*>(smem);  // reuses the KV ring after the loop
 
   cg::cluster_group cluster = cg::this_cluster();
   const int nsplit = a.splits;
@@ -119,7 +120,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int b = cid / a.Hkv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
-  pdl_wait();
+  // With PF_ATTN_EARLY_PREFETCH the tree structure, prefix lengths and the
+  // prefix cache were complete before the preceding kernel started, so they
+  // are read, and the cache tiles requested, before waiting for that kernel
+  // (programmatic dependent launch); q and the proposal K/V are read after.
+  const bool early = (a.flags & PF_ATTN_EARLY_PREFETCH) != 0;
+  if (!early) pdl_wait();
 
   const int node0 = a.cu_nodes[b];
   const int nn = a.cu_nodes[b + 1] - node0;
@@ -136,19 +142,28 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int ntiles = n_ptiles + (nn + kBN - 1) / kBN;
   const int t_begin = (int)((long long)ntiles * split / nsplit);
   const int my_tiles = (int)((long long)ntiles * (split + 1) / nsplit) - t_begin;
+  const int first = min(kStages, my_tiles);
 
   const uint32_t qbar = smem_u32(&bars[kStages]);
   if (tid == 0) {
     for (int i = 0; i < kStages; ++i) mbar_init(smem_u32(&bars[i]), 1);
     mbar_init(qbar, 1);
     fence_mbar_init();
+    for (int i = 0; i < first; ++i)
+      if (t_begin + i < n_ptiles)
+        issue_kv_tile<D, BM>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
+                             smem_u32(&bars[i]), t_begin + i, n_ptiles, b, g, node0, P);
+  }
+  if (early) pdl_wait();
+  if (tid == 0) {
     mbar_arrive_expect_tx(qbar, S::kHalves * a.G * a.nb * 128);
 #pragma unroll
     for (int h = 0; h < S::kHalves; ++h)
-      tma_load_3d(smem_u32(sQ + h * kRows * 128), &tm_q, h * 64, g * a.G, node0 + nfirst, qbar);
-    for (int i = 0; i < min(kStages, my_tiles); ++i)
-      issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
-                       smem_u32(&bars[i]), t_begin + i, n_ptiles, b, g, node0, P);
+      tma_load_3d(smem_u32(sQ + h * BM * 128), &tm_q, h * 64, g * a.G, node0 + nfirst, qbar);
+    for (int i = 0; i < first; ++i)
+      if (t_begin + i >= n_ptiles)
+        issue_kv_tile<D, BM>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
+                             smem_u32(&bars[i]), t_begin + i, n_ptiles, b, g, node0, P);
   }
   __syncthreads();
   pdl_launch_dependents();
@@ -175,8 +190,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
     for (int kk = 0; kk < KS; ++kk) {
       const int col = kk * 16 + (lane >> 4) * 8;
-      const uint32_t addr =
-          smem_u32(sQ + (col >> 6) * kRows * 128) + sw128_off(qrow, col & 63);
+      const uint32_t addr = smem_u32(sQ + (col >> 6) * BM * 128) + sw128_off(qrow, col & 63);
       ldsm_x4(addr, qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3]);
     }
   }
@@ -198,12 +212,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       // Rows past the prefix end may hold anything (even NaN bit patterns):
       // zero their V so masked-out columns contribute exactly 0.
       uint8_t* sv = stage + S::kTileBytes;
-      const int chunks = (kBN - valid) * S::kHalves * 8;
-      for (int c = tid; c < chunks; c += kThreads) {
-        const int h = c / ((kBN - valid) * 8);
-        const int rem = c % ((kBN - valid) * 8);
-        const int row = valid + rem / 8;
-        *reinterpret_cast<uint4*>(sv + h * kBN * 128 + row * 128 + (rem % 8) * 16) =
+      const int per_half = (kBN - valid) * 8;
+      for (int c = tid; c < per_half * S::kHalves; c += kThreads) {
+        const int h = c / per_half;
+        const int rem = c % per_half;
+        *reinterpret_cast<uint4*>(sv + h * kBN * 128 + (valid + rem / 8) * 128 + (rem % 8) * 16) =
             make_uint4(0, 0, 0, 0);
       }
       fence_proxy_async_smem();
@@ -292,44 +305,34 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-    __syncthreads();  // every warp is done with this stage
-    if (tid == 0 && i + kStages < my_tiles)
-      issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, stage, smem_u32(&bars[st]),
-                       t + kStages, n_ptiles, b, g, node0, P);
+    if (i + kStages < my_tiles) {
+      __syncthreads();  // every warp is done with this stage before it is refilled
+      if (tid == 0)
+        issue_kv_tile<D, BM>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, stage, smem_u32(&bars[st]),
+                             t + kStages, n_ptiles, b, g, node0, P);
+    }
   }
 
-  // ---- merge the cluster's partials through distributed shared memory
+  // ---- merge the cluster's partials through distributed shared memory:
+  // every CTA publishes its row maxima m, sums l and unnormalised O; after
+  // one cluster barrier each CTA combines a slice of the rows from all peers.
   l_run[0] += __shfl_xor_sync(0xffffffffu, l_run[0], 1);
   l_run[0] += __shfl_xor_sync(0xffffffffu, l_run[0], 2);
   l_run[1] += __shfl_xor_sync(0xffffffffu, l_run[1], 1);
   l_run[1] += __shfl_xor_sync(0xffffffffu, l_run[1], 2);
+  __syncthreads();  // the KV ring is free: every warp has finished its last tile
   if ((lane & 3) == 0) {
     sM[r0] = m_run[0];
     sL[r0] = l_run[0];
     sM[r1] = m_run[1];
     sL[r1] = l_run[1];
   }
-  cluster.sync();
   if (warp_active) {
-    float sc[2];
-#pragma unroll
-    for (int rr = 0; rr < 2; ++rr) {
-      const int r = rr ? r1 : r0;
-      float M = -INFINITY;
-      for (int q = 0; q < nsplit; ++q) M = fmaxf(M, cluster.map_shared_rank(sM, q)[r]);
-      const float Mu = M == -INFINITY ? 0.f : M;
-      float Lsum = 0.f;
-      for (int q = 0; q < nsplit; ++q)
-        Lsum += cluster.map_shared_rank(sL, q)[r] * exp2f(cluster.map_shared_rank(sM, q)[r] - Mu);
-      sc[rr] = Lsum > 0.f ? exp2f(m_run[rr] - Mu) / Lsum : 0.f;
-    }
 #pragma unroll
     for (int j = 0; j < NT; ++j) {
       const int col = j * 8 + (lane & 3) * 2;
-      *reinterpret_cast<float2*>(&sO[r0 * S::kOStride + col]) =
-          make_float2(o[j][0] * sc[0], o[j][1] * sc[0]);
-      *reinterpret_cast<float2*>(&sO[r1 * S::kOStride + col]) =
-          make_float2(o[j][2] * sc[1], o[j][3] * sc[1]);
+      *reinterpret_cast<float2*>(&sO[r0 * S::kOStride + col]) = make_float2(o[j][0], o[j][1]);
+      *reinterpret_cast<float2*>(&sO[r1 * S::kOStride + col]) = make_float2(o[j][2], o[j][3]);
     }
   }
   cluster.sync();
@@ -341,20 +344,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int idx = tid; idx < (hi - lo) * C4; idx += kThreads) {
       const int r = lo + idx / C4;
       const int c = (idx % C4) * 4;
+      float M = -INFINITY;
+      for (int q = 0; q < nsplit; ++q) M = fmaxf(M, cluster.map_shared_rank(sM, q)[r]);
+      const float Mu = M == -INFINITY ? 0.f : M;
+      float Lsum = 0.f;
       float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
       for (int q = 0; q < nsplit; ++q) {
-        const float4 v =
-            *reinterpret_cast<const float4*>(cluster.map_shared_rank(sO, q) + r * S::kOStride + c);
-        acc.x += v.x;
-        acc.y += v.y;
-        acc.z += v.z;
-        acc.w += v.w;
+        const float wq = exp2f(cluster.map_shared_rank(sM, q)[r] - Mu);
+        Lsum += wq * cluster.map_shared_rank(sL, q)[r];
+        const float4 v = *reinterpret_cast<const float4*>(cluster.map_shared_rank(sO, q) +
+                                                          r * S::kOStride + c);
+        acc.x += wq * v.x;
+        acc.y += wq * v.y;
+        acc.z += wq * v.z;
+        acc.w += wq * v.w;
       }
+      const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
       const int node = node0 + nfirst + r / a.G;
       const int h = g * a.G + r % a.G;
       uint2 pk;
-      pk.x = pack_bf16(acc.x, acc.y);
-      pk.y = pack_bf16(acc.z, acc.w);
+      pk.x = pack_bf16(acc.x * inv, acc.y * inv);
+      pk.y = pack_bf16(acc.z * inv, acc.w * inv);
       *reinterpret_cast<uint2*>(out + ((size_t)node * a.Hq + h) * D + c) = pk;
     }
   }
@@ -505,21 +515,80 @@ __global__ void __launch_bounds__(256) attn_f32_kernel(const AttnArgs a) {
   }
 }
 
+template <int D, int BM>
+cudaError_t launch_bf16_t(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl) {
+  const int smem = AttnSmem<D, BM>::kTotal + 1024;
+  static int limit[64] = {};
+  static bool nonportable[64] = {};
+  cudaError_t e = ensure_smem_limit((const void*)attn_bf16_kernel<D, BM>, smem, limit);
+  if (e != cudaSuccess) return e;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (a.splits > 8 && dev >= 0 && dev < 64 && !nonportable[dev]) {
+    e = cudaFuncSetAttribute(attn_bf16_kernel<D, BM>,
+                             cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+    nonportable[dev] = true;
+  }
+  const dim3 grid(a.B * a.Hkv * a.rb_count * a.splits);
+  return launch_ex(attn_bf16_kernel<D, BM>, grid, dim3(AttnSmem<D, BM>::kThreads), smem, s,
+                   a.splits, pdl, m.q, m.tk, m.tv, m.ck, m.cv, a);
+}
+
 template <int D>
 cudaError_t launch_bf16_d(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl) {
-  const int smem = AttnSmem<D>::kTotal + 1024;
-  static int limit[64] = {};
-  cudaError_t e = ensure_smem_limit((const void*)attn_bf16_kernel<D>, smem, limit);
-  if (e != cudaSuccess) return e;
-  const dim3 grid(a.B * a.Hkv * a.rb_count * a.splits);
-  return launch_ex(attn_bf16_kernel<D>, grid, dim3(kThreads), smem, s, a.splits, pdl, m.q, m.tk,
-                   m.tv, m.ck, m.cv, a);
+  switch (a.bm) {
+    case 32: return launch_bf16_t<D, 32>(a, m, s, pdl);
+    case 64: return launch_bf16_t<D, 64>(a, m, s, pdl);
+    default: return launch_bf16_t<D, 128>(a, m, s, pdl);
+  }
 }
 
 }  // namespace
 
-int attention_bf16_smem_bytes(int D) {
-  return (D == 64 ? AttnSmem<64>::kTotal : AttnSmem<128>::kTotal) + 1024;
+int attention_bf16_smem_bytes(int D, int bm) {
+  if (D == 64)
+    return (bm == 32 ? AttnSmem<64, 32>::kTotal
+                     : bm == 64 ? AttnSmem<64, 64>::kTotal : AttnSmem<64, 128>::kTotal) + 1024;
+  return (bm == 32 ? AttnSmem<128, 32>::kTotal
+                   : bm == 64 ? AttnSmem<128, 64>::kTotal : AttnSmem<128, 128>::kTotal) + 1024;
+}
+
+template <int D, int BM>
+bool cluster_fits_t(int cluster) {
+  const int smem = AttnSmem<D, BM>::kTotal + 1024;
+  static int limit[64] = {};
+  if (ensure_smem_limit((const void*)attn_bf16_kernel<D, BM>, smem, limit) != cudaSuccess)
+    return false;
+  if (cluster > 8 && cudaFuncSetAttribute(attn_bf16_kernel<D, BM>,
+                                          cudaFuncAttributeNonPortableClusterSizeAllowed,
+                                          1) != cudaSuccess)
+    return false;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(cluster);
+  cfg.blockDim = dim3(AttnSmem<D, BM>::kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = cluster;
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, attn_bf16_kernel<D, BM>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return n > 0;
+}
+
+bool attention_cluster_fits(int D, int bm, int cluster) {
+  if (D == 64)
+    return bm == 32 ? cluster_fits_t<64, 32>(cluster)
+                    : bm == 64 ? cluster_fits_t<64, 64>(cluster) : cluster_fits_t<64, 128>(cluster);
+  return bm == 32 ? cluster_fits_t<128, 32>(cluster)
+                  : bm == 64 ? cluster_fits_t<128, 64>(cluster) : cluster_fits_t<128, 128>(cluster);
 }
 
 cudaError_t launch_attention_bf16(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, int,

@@ -15,9 +15,11 @@ namespace pf {
 struct AttnArgs {
   int B, Hq, Hkv, D, G;
   int T, max_nodes, max_prefix;
-  int nb;          // proposal nodes per row block (bf16: floor(128 / G))
+  int bm;          // query rows per CTA (bf16: 32, 64 or 128)
+  int nb;          // proposal nodes per row block (bf16: floor(bm / G))
   int rb_count;    // row blocks per (sequence, KV head)
   int splits;      // CTAs of one cluster, each taking a slice of the KV tiles
+  int flags;       // PF_ATTN_* flags
   float scale_log2;  // softmax scale * log2(e)
   float scale;
   const int32_t* cu_nodes;
@@ -45,7 +47,10 @@ struct AttnMaps {
 cudaError_t launch_attention_bf16(const AttnArgs& a, const AttnMaps& m, cudaStream_t s,
                                   int num_sms, bool pdl);
 cudaError_t launch_attention_f32(const AttnArgs& a, cudaStream_t s, bool pdl);
-int attention_bf16_smem_bytes(int D);
+int attention_bf16_smem_bytes(int D, int bm);
+// Whether a cluster of `cluster` CTAs of the bf16 attention kernel can be
+// resident at once on this device.
+bool attention_cluster_fits(int D, int bm, int cluster);
 
 // ------------------------------------------------------------ LM head
 struct LmArgs {

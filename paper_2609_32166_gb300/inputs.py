@@ -210,6 +210,24 @@ class Batch:
         return np.concatenate(self.parents).astype(np.int32)
 
 
+def _draw_end(w: Workload, parent: np.ndarray, rng: np.random.Generator) -> int:
+    """End node of the planted accepted path, by the workload's rule."""
+    if w.accept in ("chain", "uniform_node"):
+        return int(rng.integers(0, len(parent)))       # chain: a ~ U[0, nodes-1]
+    dep = node_depths(parent)
+    a = int(rng.integers(0, int(dep.max()) + 1))
+    cand = np.nonzero(dep == a)[0]
+    return int(cand[rng.integers(len(cand))])
+
+
+def step_forced_ends(batch: "Batch", count: int) -> List[np.ndarray]:
+    """Planted accepted-path ends for ``count`` successive verify steps over
+    the same trees (each step verifies a new proposal)."""
+    rng = _stream(batch.seed, "step_ends")
+    return [np.asarray([_draw_end(batch.workload, p, rng) for p in batch.parents], np.int32)
+            for _ in range(count)]
+
+
 def make_batch(w: Workload, seed: int = 0) -> Batch:
     rng = _stream(seed, "structure")
     parents, ends = [], []
@@ -222,15 +240,7 @@ def make_batch(w: Workload, seed: int = 0) -> Batch:
             p = chains_tree(w.nodes, w.max_depth, rng)
         else:
             p = random_tree(w.nodes, w.branching, rng)
-        dep = node_depths(p)
-        if w.accept == "chain":
-            end = int(rng.integers(0, w.nodes))           # a ~ U[0, nodes-1]
-        elif w.accept == "uniform_node":
-            end = int(rng.integers(0, w.nodes))
-        else:
-            a = int(rng.integers(0, int(dep.max()) + 1))
-            cand = np.nonzero(dep == a)[0]
-            end = int(cand[rng.integers(len(cand))])
+        end = _draw_end(w, p, rng)
         parents.append(p)
         ends.append(end)
     max_seq = int(prefix_lens.max()) + w.nodes
@@ -244,19 +254,20 @@ def make_batch(w: Workload, seed: int = 0) -> Batch:
                  page_table, num_pages, max_seq)
 
 
-def plant_tokens(batch: Batch, argmax: np.ndarray) -> np.ndarray:
+def plant_tokens(batch: Batch, argmax: np.ndarray, forced_end=None, salt: int = 0) -> np.ndarray:
     """Draft tokens for every node given each node's greedy token ``argmax``
     (flat over the batch).  Along the planted path the child's token is its
     parent's greedy token; every other child gets a token different from its
     parent's greedy token and from its siblings', so the accepted path is
     exactly the planted one.  The root's token (the current token) is random."""
     w = batch.workload
-    rng = _stream(batch.seed, "tokens")
+    rng = _stream(batch.seed, "tokens", salt)
+    ends = batch.forced_end if forced_end is None else forced_end
     out = np.empty(batch.total_nodes, dtype=np.int32)
     cu = batch.cu_nodes
     for b, parent in enumerate(batch.parents):
         off = int(cu[b])
-        on_path = set(root_path(parent, int(batch.forced_end[b])))
+        on_path = set(root_path(parent, int(ends[b])))
         used = {}
         out[off] = int(rng.integers(0, w.vocab))
         for j in range(1, len(parent)):

@@ -143,6 +143,10 @@ class VerifyStep:
             d.cache = self._view(l)
             d.out = self.attn_out[l].data_ptr()
             d.error_flag = self.err.data_ptr()
+            # Within one step only pf_kv_commit writes the cache, and it runs
+            # after the last layer: every layer but the first may request its
+            # cache tiles while the previous layer is still finishing.
+            d.flags = pb.PF_ATTN_EARLY_PREFETCH if l > 0 else 0
             self.attn_descs.append(d)
         d = pb.pf_lm_desc()
         d.dtype, d.batch, d.hidden, d.vocab = dt, w.batch, w.hidden, w.vocab

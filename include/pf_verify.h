@@ -207,6 +207,26 @@ PF_API pf_status pf_lmhead_accept(const pf_lm_desc* d, void* workspace, size_t w
                            void* stream);
 
 /*
+ * pf_lmhead_accept_noalloc -- pf_lmhead_accept without a workspace argument.
+ * The paper has no counterpart: this exists for callers that cannot
+ * allocate device memory where they verify, e.g. code running while a
+ * stream is being captured into a CUDA graph (cudaMalloc is not allowed
+ * there), plug-ins whose host framework owns every device allocation, and
+ * loops that must never reach the allocator.  The scratch lives in a
+ * file-scope device array of 2112 bytes (room for PF_MAX_LM_ROWS = 256
+ * proposal rows) that every GPU loading this library holds until exit;
+ * total_nodes above 256 is rejected with PF_ERR_SHAPE.  The first call on
+ * each device looks up that array's device address (cudaGetSymbolAddress),
+ * so make the first call on a device before any stream capture.  Every call
+ * clears the array (cudaMemsetAsync on the given stream) and then runs
+ * exactly pf_lmhead_accept; nothing is allocated or freed.  All calls share
+ * the one array, so calls that overlap on the GPU (other streams, other
+ * host threads) race: serialise them.  Same outputs and errors as
+ * pf_lmhead_accept otherwise.
+ */
+PF_API pf_status pf_lmhead_accept_noalloc(const pf_lm_desc* d, void* stream);
+
+/*
  * pf_kv_commit -- carry the accepted rows forward (Section 1 and Section
  * 3.4: accepted positions keep their K/V; Section 4: one contiguous cache).
  * For every layer l, K and V, sequence b and k = 0..accept_len[b]:

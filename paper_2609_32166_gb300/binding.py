@@ -108,6 +108,8 @@ def lib() -> C.CDLL:
     L.pf_lmhead_accept_workspace_size.argtypes = [C.POINTER(pf_lm_desc)]
     L.pf_lmhead_accept.restype = C.c_int
     L.pf_lmhead_accept.argtypes = [C.POINTER(pf_lm_desc), C.c_void_p, C.c_size_t, C.c_void_p]
+    L.pf_lmhead_accept_noalloc.restype = C.c_int
+    L.pf_lmhead_accept_noalloc.argtypes = [C.POINTER(pf_lm_desc), C.c_void_p]
     L.pf_kv_commit.restype = C.c_int
     L.pf_kv_commit.argtypes = [C.POINTER(pf_commit_desc), C.c_void_p]
     _lib = L
@@ -155,6 +157,12 @@ def pf_lmhead_accept(desc: pf_lm_desc, workspace: int, workspace_bytes: int,
                      stream: int = 0) -> None:
     _check(lib().pf_lmhead_accept(C.byref(desc), C.c_void_p(workspace),
                                   C.c_size_t(workspace_bytes), C.c_void_p(stream)))
+
+
+def pf_lmhead_accept_noalloc(desc: pf_lm_desc, stream: int = 0) -> None:
+    """pf_lmhead_accept with the scratch in the library's fixed device array
+    (for callers that cannot allocate; calls must not overlap on the GPU)."""
+    _check(lib().pf_lmhead_accept_noalloc(C.byref(desc), C.c_void_p(stream)))
 
 
 def pf_kv_commit(desc: pf_commit_desc, stream: int = 0) -> None:

@@ -161,6 +161,18 @@ void choose_attention_shape(pf::AttnArgs& a, int max_prefix_len, int sms) {
 
 }  // namespace
 
+namespace pf {
+pf_status set_error(pf_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return s;
+}
+}  // namespace pf
+
 extern "C" {
 
 const char* pf_last_error(void) { return g_last_error.c_str(); }

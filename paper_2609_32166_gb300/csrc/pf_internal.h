@@ -108,6 +108,9 @@ struct CommitArgs {
 
 cudaError_t launch_kv_commit(const CommitArgs& a, cudaStream_t s, int num_sms, bool pdl);
 
+// Record the message pf_last_error() returns on this thread; returns s.
+pf_status set_error(pf_status s, const char* fmt, ...);
+
 // Raise a kernel's dynamic shared-memory limit once per device (never while
 // a stream is being captured after the first call on that device).
 inline cudaError_t ensure_smem_limit(const void* func, int bytes, int* per_device) {

@@ -114,23 +114,51 @@ pf_status check_cache_view(const pf_kv_view& c, int need_rows, const char* who) 
 // and wide clusters so that enough SMs stream the cache; large ones keep
 // 128-row blocks so each K/V tile serves more rows.  A cluster wider than 8
 // is used only if the device can schedule it.
-int max_cluster_for(int bm, int D, int want) {
-  static int cache[64][3][2][17];
+// kernel index 0..2: mma.sync BM 32/64/128; 3: tcgen05
+int max_cluster_for(int kernel, int D, int want) {
+  static int cache[64][4][2][17];
   int dev = 0;
   cudaGetDevice(&dev);
-  const int bi = bm == 32 ? 0 : bm == 64 ? 1 : 2, di = D == 64 ? 0 : 1;
+  const int di = D == 64 ? 0 : 1;
   int w = want;
   while (w > 8) {
-    int& c = cache[dev & 63][bi][di][w];
-    if (c == 0) c = pf::attention_cluster_fits(D, bm, w) ? 1 : -1;
+    int& c = cache[dev & 63][kernel][di][w];
+    if (c == 0) {
+      const bool fits = kernel == 3 ? pf::attention_tc_cluster_fits(w)
+                                    : pf::attention_cluster_fits(D, 32 << kernel, w);
+      c = fits ? 1 : -1;
+    }
     if (c > 0) break;
-    --w;
+    w -= kernel == 3 ? 2 : 1;
   }
   return w;
 }
 
+// The tcgen05 kernel serves bf16 with D = 128 (PF_ATTN_IMPL=mma selects the
+// mma.sync kernel instead).
+bool use_tc_attention(const pf::AttnArgs& a) {
+  const char* e = getenv("PF_ATTN_IMPL");
+  return a.D == 128 && !(e && strcmp(e, "mma") == 0);
+}
+
 void choose_attention_shape(pf::AttnArgs& a, int max_prefix_len, int sms) {
   const int max_tiles = (max_prefix_len + 63) / 64 + (a.max_nodes + 63) / 64;
+  if (use_tc_attention(a)) {
+    a.bm = 128;
+    a.nb = 128 / a.G;
+    a.rb_count = (a.max_nodes + a.nb - 1) / a.nb;
+    const int base = a.B * a.Hkv * a.rb_count;
+    int splits = sms / base;
+    if (const char* e = getenv("PF_ATTN_SPLITS")) splits = atoi(e);
+    splits = std::max(1, std::min({splits, 16, max_tiles}));
+    // even cluster sizes: clusters are placed on pairs of SMs, so an odd
+    // cluster of one-CTA-per-SM blocks strands an SM and can push the grid
+    // into a second wave
+    if (splits > 1) splits &= ~1;
+    if (splits > 8) splits = max_cluster_for(3, a.D, splits);
+    a.splits = splits;
+    return;
+  }
   const int bms[3] = {128, 64, 32};
   int pick = 32;
   for (int bm : bms) {
@@ -155,7 +183,7 @@ void choose_attention_shape(pf::AttnArgs& a, int max_prefix_len, int sms) {
   if (splits > 16) splits = 16;
   if (splits > max_tiles) splits = max_tiles;
   if (splits < 1) splits = 1;
-  if (splits > 8) splits = max_cluster_for(pick, a.D, splits);
+  if (splits > 8) splits = max_cluster_for(pick == 32 ? 0 : pick == 64 ? 1 : 2, a.D, splits);
   a.splits = splits;
 }
 
@@ -306,7 +334,8 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
     if ((st = make_map(&m.ck, 4, d->cache.k, dims, str, box, "cache.k")) != PF_OK) return st;
     if ((st = make_map(&m.cv, 4, d->cache.v, dims, str, box, "cache.v")) != PF_OK) return st;
   }
-  cudaError_t e = pf::launch_attention_bf16(a, m, s, sms, pdl_enabled());
+  cudaError_t e = use_tc_attention(a) ? pf::launch_attention_tc(a, m, s, pdl_enabled())
+                                      : pf::launch_attention_bf16(a, m, s, sms, pdl_enabled());
   return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
 }
 
@@ -399,6 +428,8 @@ pf_status pf_kv_commit(const pf_commit_desc* d, void* stream) {
   if (d->max_nodes < 1 || d->max_nodes > PF_MAX_NODES)
     return fail(PF_ERR_SHAPE, "%s: max_nodes outside 1..%d", who, PF_MAX_NODES);
   if (d->max_prefix_len < 0) return fail(PF_ERR_SHAPE, "%s: max_prefix_len < 0", who);
+  if ((long long)d->n_layers * d->batch * 2 > 65535)
+    return fail(PF_ERR_SHAPE, "%s: n_layers * batch must be <= 32767", who);
   const int es = elem_size(d->dtype);
   const int row_bytes = d->head_dim * es;
   if (row_bytes % 16 != 0)

@@ -15,8 +15,7 @@
 // no workspace and no second launch are needed.
 #include <cooperative_groups.h>
 
-#include "pf_internal.h"
-#include "pf_ptx.cuh"
+#include "attn_common.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -24,7 +23,6 @@ namespace pf {
 
 namespace {
 
-constexpr int kBN = 64;         // tokens per KV tile
 constexpr int kStages = 3;
 
 // Shared-memory plan of one CTA with BM query rows (BM / 16 warps).
@@ -41,54 +39,6 @@ struct AttnSmem {
   static constexpr int kOStride = D + 4;               // fp32 partial-O row pitch
   static_assert(BM * kOStride * 4 <= kStages * kStageBytes, "partial O must fit the KV ring");
 };
-
-__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
-  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
-}
-
-template <int D, int BM>
-__device__ __forceinline__ void issue_kv_tile(const AttnArgs& a, const CUtensorMap* tm_ck,
-                                              const CUtensorMap* tm_cv, const CUtensorMap* tm_tk,
-                                              const CUtensorMap* tm_tv, uint8_t* stage,
-                                              uint32_t bar, int t, int n_ptiles, int b, int g,
-                                              int node0, int P) {
-  using S = AttnSmem<D, BM>;
-  uint8_t* sk = stage;
-  uint8_t* sv = stage + S::kTileBytes;
-  if (t < n_ptiles) {
-    const int tok0 = t * kBN;
-    if (a.layout == PF_KV_CONTIGUOUS) {
-      mbar_arrive_expect_tx(bar, 2 * S::kTileBytes);
-#pragma unroll
-      for (int h = 0; h < S::kHalves; ++h) {
-        tma_load_3d(smem_u32(sk + h * kBN * 128), tm_ck, h * 64, tok0, b * a.Hkv + g, bar);
-        tma_load_3d(smem_u32(sv + h * kBN * 128), tm_cv, h * 64, tok0, b * a.Hkv + g, bar);
-      }
-    } else {
-      const int left = P - tok0;
-      const int npages = min(kBN / PF_PAGE_SIZE, (left + PF_PAGE_SIZE - 1) / PF_PAGE_SIZE);
-      mbar_arrive_expect_tx(bar, 2 * S::kHalves * npages * PF_PAGE_SIZE * 128);
-      const int32_t* pt = a.page_table + (size_t)b * a.pages_per_seq + tok0 / PF_PAGE_SIZE;
-      for (int p = 0; p < npages; ++p) {
-        const int page = pt[p];
-#pragma unroll
-        for (int h = 0; h < S::kHalves; ++h) {
-          const int off = h * kBN * 128 + p * PF_PAGE_SIZE * 128;
-          tma_load_4d(smem_u32(sk + off), tm_ck, h * 64, 0, g, page, bar);
-          tma_load_4d(smem_u32(sv + off), tm_cv, h * 64, 0, g, page, bar);
-        }
-      }
-    }
-  } else {
-    const int j = t - n_ptiles;
-    mbar_arrive_expect_tx(bar, 2 * S::kTileBytes);
-#pragma unroll
-    for (int h = 0; h < S::kHalves; ++h) {
-      tma_load_3d(smem_u32(sk + h * kBN * 128), tm_tk, h * 64, g, node0 + j * kBN, bar);
-      tma_load_3d(smem_u32(sv + h * kBN * 128), tm_tv, h * 64, g, node0 + j * kBN, bar);
-    }
-  }
-}
 
 template <int D, int BM>
 __global__ void __launch_bounds__(BM * 2, 1)
@@ -151,7 +101,7 @@ __global__ void __launch_bounds__(BM * 2, 1)
     fence_mbar_init();
     for (int i = 0; i < first; ++i)
       if (t_begin + i < n_ptiles)
-        issue_kv_tile<D, BM>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
+        issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
                              smem_u32(&bars[i]), t_begin + i, n_ptiles, b, g, node0, P);
   }
   if (early) pdl_wait();
@@ -162,7 +112,7 @@ __global__ void __launch_bounds__(BM * 2, 1)
       tma_load_3d(smem_u32(sQ + h * BM * 128), &tm_q, h * 64, g * a.G, node0 + nfirst, qbar);
     for (int i = 0; i < first; ++i)
       if (t_begin + i >= n_ptiles)
-        issue_kv_tile<D, BM>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
+        issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
                              smem_u32(&bars[i]), t_begin + i, n_ptiles, b, g, node0, P);
   }
   __syncthreads();
@@ -308,67 +258,33 @@ __global__ void __launch_bounds__(BM * 2, 1)
     if (i + kStages < my_tiles) {
       __syncthreads();  // every warp is done with this stage before it is refilled
       if (tid == 0)
-        issue_kv_tile<D, BM>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, stage, smem_u32(&bars[st]),
+        issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, stage, smem_u32(&bars[st]),
                              t + kStages, n_ptiles, b, g, node0, P);
     }
   }
 
-  // ---- merge the cluster's partials through distributed shared memory:
-  // every CTA publishes its row maxima m, sums l and unnormalised O; after
-  // one cluster barrier each CTA combines a slice of the rows from all peers.
+  __syncthreads();  // the KV ring is free: every warp has finished its last tile
+  if ((lane & 3) == 0) {
+    sM[r0] = m_run[0];
+    sM[r1] = m_run[1];
+  }
   l_run[0] += __shfl_xor_sync(0xffffffffu, l_run[0], 1);
   l_run[0] += __shfl_xor_sync(0xffffffffu, l_run[0], 2);
   l_run[1] += __shfl_xor_sync(0xffffffffu, l_run[1], 1);
   l_run[1] += __shfl_xor_sync(0xffffffffu, l_run[1], 2);
-  __syncthreads();  // the KV ring is free: every warp has finished its last tile
   if ((lane & 3) == 0) {
-    sM[r0] = m_run[0];
     sL[r0] = l_run[0];
-    sM[r1] = m_run[1];
     sL[r1] = l_run[1];
   }
   if (warp_active) {
 #pragma unroll
     for (int j = 0; j < NT; ++j) {
       const int col = j * 8 + (lane & 3) * 2;
-      *reinterpret_cast<float2*>(&sO[r0 * S::kOStride + col]) = make_float2(o[j][0], o[j][1]);
-      *reinterpret_cast<float2*>(&sO[r1 * S::kOStride + col]) = make_float2(o[j][2], o[j][3]);
+      *reinterpret_cast<float2*>(&sO[r0 * (D + 4) + col]) = make_float2(o[j][0], o[j][1]);
+      *reinterpret_cast<float2*>(&sO[r1 * (D + 4) + col]) = make_float2(o[j][2], o[j][3]);
     }
   }
-  cluster.sync();
-  {
-    const int per = (rows + nsplit - 1) / nsplit;
-    const int lo = split * per, hi = min(rows, lo + per);
-    constexpr int C4 = D / 4;
-    __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.out);
-    for (int idx = tid; idx < (hi - lo) * C4; idx += kThreads) {
-      const int r = lo + idx / C4;
-      const int c = (idx % C4) * 4;
-      float M = -INFINITY;
-      for (int q = 0; q < nsplit; ++q) M = fmaxf(M, cluster.map_shared_rank(sM, q)[r]);
-      const float Mu = M == -INFINITY ? 0.f : M;
-      float Lsum = 0.f;
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int q = 0; q < nsplit; ++q) {
-        const float wq = exp2f(cluster.map_shared_rank(sM, q)[r] - Mu);
-        Lsum += wq * cluster.map_shared_rank(sL, q)[r];
-        const float4 v = *reinterpret_cast<const float4*>(cluster.map_shared_rank(sO, q) +
-                                                          r * S::kOStride + c);
-        acc.x += wq * v.x;
-        acc.y += wq * v.y;
-        acc.z += wq * v.z;
-        acc.w += wq * v.w;
-      }
-      const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
-      const int node = node0 + nfirst + r / a.G;
-      const int h = g * a.G + r % a.G;
-      uint2 pk;
-      pk.x = pack_bf16(acc.x * inv, acc.y * inv);
-      pk.y = pack_bf16(acc.z * inv, acc.w * inv);
-      *reinterpret_cast<uint2*>(out + ((size_t)node * a.Hq + h) * D + c) = pk;
-    }
-  }
-  cluster.sync();  // keep this CTA's shared memory alive until every peer has read it
+  cluster_merge<D, kThreads>(a, cluster, sM, sL, sO, rows, split, nsplit, node0 + nfirst, g, tid);
 }
 
 // ---------------------------------------------------------------- fp32 path

@@ -1,0 +1,425 @@
+// Tree-masked GQA attention on the 5th-generation tensor cores (tcgen05).
+// Same contract and work split as the mma.sync kernel in attention.cu (one
+// CTA = 128 query rows of one KV head x a slice of the 64-token KV tiles,
+// clusters merge the slices); the arithmetic moves to UMMA with TMEM
+// accumulators:
+//
+//   warp 0     TMA producer: Q once, then K/V tiles into a 3-stage ring
+//   warp 1     TMEM owner and MMA issuer (one thread):
+//                S_i  = Q K_i^T      M=128, N=64, K=D   -> TMEM S[i % 2]
+//                O   += P_i V_i      M=128, N=D,  K=64  -> TMEM O
+//              issued in the order S_0 S_1 PV_0 S_2 PV_1 ... so the tensor
+//              core computes S_{i+1} while the softmax warps work on S_i
+//   warps 2-5  one query row per thread (its TMEM lane): read S_i, mask
+//              (prefix length / ancestor bits), online softmax in the exp2
+//              domain, write P_i as bf16 into shared memory (K-major,
+//              128-byte swizzle); the running maximum is only moved (and O
+//              rescaled in TMEM) when it grows by more than 2^8, so the
+//              common case never touches O; at the end they read O back
+//              and publish (m, l, O) for the cluster merge.
+//
+// V is the B operand of PV in its natural token-major layout (an MN-major
+// UMMA operand), so no transpose is needed anywhere.
+#include <cuda_fp16.h>
+
+#include "attn_common.cuh"
+
+namespace cg = cooperative_groups;
+
+namespace pf {
+
+namespace {
+
+constexpr int kTcStages = 3;
+constexpr int kTcThreads = 192;
+constexpr float kRescaleLog2 = 8.f;   // move the reference max when it grows by > 2^8
+constexpr uint32_t kTmemCols = 256;   // S[0] 0..63, S[1] 64..127, O 128..128+D-1
+
+template <int D>
+struct TcSmem {
+  static constexpr int kHalves = D / 64;
+  static constexpr int kTileBytes = kBN * D * 2;         // one K or V tile
+  static constexpr int kStageBytes = 2 * kTileBytes;     // K + V
+  static constexpr int kQBytes = 128 * D * 2;
+  static constexpr int kPBytes = 128 * kBN * 2;          // one P tile (bf16)
+  static constexpr int kQOff = kTcStages * kStageBytes;
+  static constexpr int kPOff = kQOff + kQBytes;
+  // Merge inbox: one slot per (split, row) a CTA may receive, at most
+  // splits * ceil(rows / splits) <= 128 + 15 slots: the normalised partial
+  // O / l in fp16 (pitch D + 8 halves) and its log2-sum-exp.
+  static constexpr int kInboxSlots = 144;
+  static constexpr int kInboxPitch = D + 8;              // halves
+  static constexpr int kInboxOff = kPOff + 2 * kPBytes;
+  static constexpr int kLseOff = kInboxOff + kInboxSlots * kInboxPitch * 2;
+  static constexpr int kBarOff = kLseOff + kInboxSlots * 4;
+  // kv_full[3] kv_empty[3] q_full s_full[2] s_empty[2] p_full[2] pv_done[2]
+  static constexpr int kNumBars = 2 * kTcStages + 9;
+  static constexpr int kTotal = kBarOff + kNumBars * 8 + 16;
+  static_assert(kTotal + 1024 <= 232448, "shared memory budget");
+};
+
+template <int D>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
+                   const __grid_constant__ CUtensorMap tm_tk,
+                   const __grid_constant__ CUtensorMap tm_tv,
+                   const __grid_constant__ CUtensorMap tm_ck,
+                   const __grid_constant__ CUtensorMap tm_cv, const AttnArgs a) {
+  using S = TcSmem<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  uint8_t* sKV = smem;
+  uint8_t* sQ = smem + S::kQOff;
+  uint8_t* sP = smem + S::kPOff;
+  __half* sInbox = reinterpret_cast<__half*>(smem + S::kInboxOff);
+  float* sLse = reinterpret_cast<float*>(smem + S::kLseOff);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S::kBarOff);
+  uint64_t* kv_full = bars;
+  uint64_t* kv_empty = bars + kTcStages;
+  uint64_t* q_full = bars + 2 * kTcStages;
+  uint64_t* s_full = q_full + 1;
+  uint64_t* s_empty = s_full + 2;
+  uint64_t* p_full = s_empty + 2;
+  uint64_t* pv_done = p_full + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + S::kNumBars);
+
+  cg::cluster_group cluster = cg::this_cluster();
+  const int nsplit = a.splits;
+  const int split = (int)cluster.block_rank();
+  int cid = blockIdx.x / nsplit;
+  const int rb = cid % a.rb_count;
+  cid /= a.rb_count;
+  const int g = cid % a.Hkv;
+  const int b = cid / a.Hkv;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+  // With PF_ATTN_EARLY_PREFETCH the tree structure, prefix lengths and the
+  // prefix cache were complete before the preceding kernel started: read
+  // them and request cache tiles before waiting for it (programmatic
+  // dependent launch); q and the proposal K/V only after.
+  const bool early = (a.flags & PF_ATTN_EARLY_PREFETCH) != 0;
+  if (!early) pdl_wait();
+
+  const int node0 = a.cu_nodes[b];
+  const int nn = a.cu_nodes[b + 1] - node0;
+  const int P = a.prefix_len[b];
+  if (node0 < 0 || nn < 1 || nn > a.max_nodes || node0 + nn > a.T || P < 0 ||
+      P > a.max_prefix) {
+    if (tid == 0 && split == 0 && rb == 0) flag_error(a.err, PF_DEVERR_BOUNDS);
+    return;  // uniform over the cluster (same b)
+  }
+  const int nfirst = rb * a.nb;
+  if (nfirst >= nn) return;  // uniform over the cluster (same b, g, rb)
+  const int rows = min(a.nb, nn - nfirst) * a.G;
+  const int n_ptiles = (P + kBN - 1) / kBN;
+  const int ntiles = n_ptiles + (nn + kBN - 1) / kBN;
+  const int t_begin = (int)((long long)ntiles * split / nsplit);
+  const int my_tiles = (int)((long long)ntiles * (split + 1) / nsplit) - t_begin;
+  const int first = min(kTcStages, my_tiles);
+
+  if (tid == 0) {
+    for (int i = 0; i < kTcStages; ++i) {
+      mbar_init(smem_u32(&kv_full[i]), 1);
+      mbar_init(smem_u32(&kv_empty[i]), 1);
+    }
+    mbar_init(smem_u32(q_full), 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&s_full[i]), 1);
+      mbar_init(smem_u32(&s_empty[i]), 128);
+      mbar_init(smem_u32(&p_full[i]), 128);
+      mbar_init(smem_u32(&pv_done[i]), 1);
+    }
+    fence_mbar_init();
+    for (int i = 0; i < first; ++i)
+      if (t_begin + i < n_ptiles)
+        issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
+                         smem_u32(&kv_full[i]), t_begin + i, n_ptiles, b, g, node0, P);
+  }
+  if (early) pdl_wait();
+  if (tid == 0) {
+    mbar_arrive_expect_tx(smem_u32(q_full), S::kHalves * a.G * a.nb * 128);
+#pragma unroll
+    for (int h = 0; h < S::kHalves; ++h)
+      tma_load_3d(smem_u32(sQ + h * 128 * 128), &tm_q, h * 64, g * a.G, node0 + nfirst,
+                  smem_u32(q_full));
+    for (int i = 0; i < first; ++i)
+      if (t_begin + i >= n_ptiles)
+        issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
+                         smem_u32(&kv_full[i]), t_begin + i, n_ptiles, b, g, node0, P);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_launch_dependents();
+
+  float m_ref = -INFINITY, l = 0.f;   // softmax threads: running max (log2) and sum of their row
+  if (warp == 0) {
+    // ---------------- producer: refill the ring as PV releases stages
+    if (lane == 0) {
+      for (int i = kTcStages; i < my_tiles; ++i) {
+        const int st = i % kTcStages;
+        if (!mbar_wait(smem_u32(&kv_empty[st]), ((i / kTcStages) & 1) ^ 1, a.err)) break;
+        issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + st * S::kStageBytes,
+                         smem_u32(&kv_full[st]), t_begin + i, n_ptiles, b, g, node0, P);
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer
+    if (lane == 0) {
+      const uint32_t id_s = umma_idesc_bf16(128, kBN);
+      const uint32_t id_o = umma_idesc_bf16_bmn(128, D);
+      bool ok = mbar_wait(smem_u32(q_full), 0, a.err);
+      const uint32_t q0 = smem_u32(sQ);
+      for (int i = 0; i <= my_tiles && ok; ++i) {
+        if (i < my_tiles) {
+          const int st = i % kTcStages, sb = i & 1;
+          ok = mbar_wait(smem_u32(&kv_full[st]), (i / kTcStages) & 1, a.err) &&
+               mbar_wait(smem_u32(&s_empty[sb]), ((i >> 1) & 1) ^ 1, a.err);
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t k0 = smem_u32(sKV + st * S::kStageBytes);
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t qa = q0 + (kk >> 2) * (128 * 128) + (kk & 3) * 32;
+            const uint32_t kb = k0 + (kk >> 2) * (kBN * 128) + (kk & 3) * 32;
+            umma_bf16(tmem + sb * kBN, umma_desc_sw128(qa), umma_desc_sw128(kb), id_s, kk > 0);
+          }
+          umma_commit(smem_u32(&s_full[sb]));
+        }
+        if (i >= 1) {
+          const int j = i - 1, pb = j & 1, stj = j % kTcStages;
+          ok = mbar_wait(smem_u32(&p_full[pb]), (j >> 1) & 1, a.err);
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t p0 = smem_u32(sP + pb * S::kPBytes);
+          const uint32_t v0 = smem_u32(sKV + stj * S::kStageBytes + S::kTileBytes);
+#pragma unroll
+          for (int kt = 0; kt < kBN / 16; ++kt)
+            umma_bf16(tmem + 2 * kBN, umma_desc_sw128(p0 + kt * 32),
+                      umma_desc_sw128_lbo(v0 + kt * 16 * 128, kBN * 128, 1024), id_o,
+                      (j > 0 || kt > 0) ? 1u : 0u);
+          umma_commit(smem_u32(&pv_done[pb]));
+          umma_commit(smem_u32(&kv_empty[stj]));
+        }
+      }
+    }
+  } else {
+    // ---------------- softmax / correction / epilogue: one row per thread
+    const int quad = warp & 3;
+    const int r = quad * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+    uint64_t mk0 = 0, mk1 = 0;
+    if (r < rows) {
+      const int node = node0 + nfirst + r / a.G;
+      mk0 = a.mask[2 * node];
+      mk1 = a.mask[2 * node + 1];
+    }
+    bool ok = true;
+    for (int i = 0; i < my_tiles && ok; ++i) {
+      const int sb = i & 1;
+      const int st = i % kTcStages;
+      ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&s_full[sb]), (i >> 1) & 1, a.err));
+      if (!ok) break;  // warp-uniform
+      tc_fence_after();
+      uint32_t lo[32], hi[32];
+      tmem_ld_32(tmem + lane_base + sb * kBN, lo);
+      tmem_ld_32(tmem + lane_base + sb * kBN + 32, hi);
+      tmem_ld_wait();
+      tc_fence_before();
+      mbar_arrive(smem_u32(&s_empty[sb]));
+
+      const int t = t_begin + i;
+      const bool is_prefix = t < n_ptiles;
+      const int valid = is_prefix ? min(kBN, P - t * kBN) : kBN;
+      float sv[64];
+#pragma unroll
+      for (int c = 0; c < 64; ++c) sv[c] = __uint_as_float(c < 32 ? lo[c] : hi[c - 32]);
+      if (!is_prefix || valid < kBN) {
+        // masked tile: prefix columns past the end, or proposal columns
+        // that are not ancestors of this row's node
+        const uint64_t vis = is_prefix ? (valid >= 64 ? ~0ull : ((1ull << valid) - 1ull))
+                                       : ((t - n_ptiles) ? mk1 : mk0);
+#pragma unroll
+        for (int c = 0; c < 64; ++c)
+          if (!((vis >> c) & 1ull)) sv[c] = -INFINITY;
+      }
+      // row maximum of the raw scores (scale > 0 commutes with max), as a
+      // tree so that the dependent chain is 6 deep rather than 64
+      float mxs[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        float m2 = fmaxf(fmaxf(sv[k], sv[k + 8]), fmaxf(sv[k + 16], sv[k + 24]));
+        float m3 = fmaxf(fmaxf(sv[k + 32], sv[k + 40]), fmaxf(sv[k + 48], sv[k + 56]));
+        mxs[k] = fmaxf(m2, m3);
+      }
+      const float mx = fmaxf(fmaxf(fmaxf(mxs[0], mxs[1]), fmaxf(mxs[2], mxs[3])),
+                             fmaxf(fmaxf(mxs[4], mxs[5]), fmaxf(mxs[6], mxs[7]))) *
+                       a.scale_log2;
+      const float m_new = fmaxf(m_ref, mx);
+      const bool resc = m_ref != -INFINITY && m_new > m_ref + kRescaleLog2;
+      if (m_ref == -INFINITY) m_ref = m_new;
+      if (__any_sync(0xffffffffu, resc)) {
+        // O must hold exactly the tiles before i: wait for PV_{i-1}.
+        if (i >= 1) mbar_wait(smem_u32(&pv_done[(i - 1) & 1]), ((i - 1) >> 1) & 1, a.err);
+        tc_fence_after();
+        const float alpha = resc ? ex2_approx(m_ref - m_new) : 1.f;
+#pragma unroll
+        for (int c0 = 0; c0 < D; c0 += 32) {
+          uint32_t ov[32];
+          tmem_ld_32(tmem + lane_base + 2 * kBN + c0, ov);
+          tmem_ld_wait();
+#pragma unroll
+          for (int c = 0; c < 32; ++c) ov[c] = __float_as_uint(__uint_as_float(ov[c]) * alpha);
+          tmem_st_32(tmem + lane_base + 2 * kBN + c0, ov);
+        }
+        tmem_st_wait();
+        if (resc) {
+          l *= alpha;
+          m_ref = m_new;
+        }
+      }
+      // p = 2^(s * scale_log2 - m): one FFMA and one MUFU per score
+      const float neg_mu = m_ref == -INFINITY ? 0.f : -m_ref;
+      float rs[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      uint32_t pk[32];
+#pragma unroll
+      for (int c = 0; c < 32; ++c) {
+        const float p0 = ex2_approx(fmaf(sv[2 * c], a.scale_log2, neg_mu));
+        const float p1 = ex2_approx(fmaf(sv[2 * c + 1], a.scale_log2, neg_mu));
+        rs[c & 7] += p0 + p1;
+        pk[c] = pack_bf16(p0, p1);
+      }
+      l += ((rs[0] + rs[1]) + (rs[2] + rs[3])) + ((rs[4] + rs[5]) + (rs[6] + rs[7]));
+      // P buffer sb was last read by PV_{i-2}.
+      if (i >= 2) mbar_wait(smem_u32(&pv_done[sb]), ((i - 2) >> 1) & 1, a.err);
+      uint8_t* prow = sP + sb * S::kPBytes + r * 128;
+#pragma unroll
+      for (int c = 0; c < 8; ++c)
+        *reinterpret_cast<uint4*>(prow + ((c ^ (r & 7)) << 4)) =
+            make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+      if (valid < kBN) {
+        // Cache rows past the prefix end may hold anything (even NaN bit
+        // patterns): zero their V so masked columns contribute exactly 0.
+        uint8_t* sv = sKV + st * S::kStageBytes + S::kTileBytes;
+        const int per_half = (kBN - valid) * 8;
+        for (int c = r; c < per_half * S::kHalves; c += 128) {
+          const int h = c / per_half, rem = c % per_half;
+          *reinterpret_cast<uint4*>(sv + h * kBN * 128 + (valid + rem / 8) * 128 + (rem % 8) * 16) =
+              make_uint4(0, 0, 0, 0);
+        }
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(smem_u32(&p_full[sb]));
+    }
+    // O of this row is complete once the last PV has landed
+    if (my_tiles > 0)
+      mbar_wait(smem_u32(&pv_done[(my_tiles - 1) & 1]), ((my_tiles - 1) >> 1) & 1, a.err);
+  }
+  __syncwarp();  // the producer and MMA lanes rejoin their warps before the barriers
+
+  // ---- split-KV merge, push style.  Each row's partial result, normalised
+  // (O / l, fp16) with its log2-sum-exp lse = m + log2(l), is stored straight
+  // into a dedicated inbox in the shared memory of the CTA that merges that
+  // row (posted remote stores; the inbox is never touched by the KV loop, so
+  // no barrier is needed before them).  One cluster barrier makes them
+  // visible; each CTA then merges its rows from local shared memory:
+  //   out = sum_s 2^(lse_s - M) (O/l)_s / sum_s 2^(lse_s - M),  M = max_s lse_s
+  const int per = (rows + nsplit - 1) / nsplit;
+  if (warp >= 2) {
+    const int quad = warp & 3;
+    const int r = quad * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+    const bool valid_row = r < rows;
+    const int owner = valid_row ? r / per : 0;
+    const int slot = split * per + (r - owner * per);
+    const float inv_l = (my_tiles > 0 && l > 0.f) ? 1.f / l : 0.f;
+    __half* dst = cluster.map_shared_rank(sInbox, owner) + slot * S::kInboxPitch;
+#pragma unroll
+    for (int c0 = 0; c0 < D; c0 += 32) {
+      uint32_t ov[32];
+      tmem_ld_32(tmem + lane_base + 2 * kBN + c0, ov);
+      tmem_ld_wait();
+      if (valid_row) {
+#pragma unroll
+        for (int c = 0; c < 32; c += 8) {
+          uint4 pk;
+          pk.x = pack_half(__uint_as_float(ov[c]) * inv_l, __uint_as_float(ov[c + 1]) * inv_l);
+          pk.y = pack_half(__uint_as_float(ov[c + 2]) * inv_l, __uint_as_float(ov[c + 3]) * inv_l);
+          pk.z = pack_half(__uint_as_float(ov[c + 4]) * inv_l, __uint_as_float(ov[c + 5]) * inv_l);
+          pk.w = pack_half(__uint_as_float(ov[c + 6]) * inv_l, __uint_as_float(ov[c + 7]) * inv_l);
+          *reinterpret_cast<uint4*>(dst + c0 + c) = pk;
+        }
+      }
+    }
+    if (valid_row)
+      cluster.map_shared_rank(sLse, owner)[slot] =
+          inv_l > 0.f ? m_ref + __log2f(l) : -INFINITY;
+  }
+  tc_fence_before();
+  cluster.sync();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+  inbox_merge<D, kTcThreads, S::kInboxPitch>(a, sLse, sInbox, rows, split, per, nsplit,
+                                             node0 + nfirst, g, tid);
+}
+
+}  // namespace
+
+int attention_tc_smem_bytes() { return TcSmem<128>::kTotal + 1024; }
+
+bool attention_tc_cluster_fits(int cluster) {
+  const int smem = TcSmem<128>::kTotal + 1024;
+  static int limit[64] = {};
+  if (ensure_smem_limit((const void*)attn_tc_kernel<128>, smem, limit) != cudaSuccess)
+    return false;
+  if (cluster > 8 && cudaFuncSetAttribute(attn_tc_kernel<128>,
+                                          cudaFuncAttributeNonPortableClusterSizeAllowed,
+                                          1) != cudaSuccess)
+    return false;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(cluster);
+  cfg.blockDim = dim3(kTcThreads);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = cluster;
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<128>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return n > 0;
+}
+
+cudaError_t launch_attention_tc(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl) {
+  const int smem = TcSmem<128>::kTotal + 1024;
+  static int limit[64] = {};
+  static bool nonportable[64] = {};
+  cudaError_t e = ensure_smem_limit((const void*)attn_tc_kernel<128>, smem, limit);
+  if (e != cudaSuccess) return e;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (a.splits > 8 && dev >= 0 && dev < 64 && !nonportable[dev]) {
+    e = cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeNonPortableClusterSizeAllowed,
+                             1);
+    if (e != cudaSuccess) return e;
+    nonportable[dev] = true;
+  }
+  const dim3 grid(a.B * a.Hkv * a.rb_count * a.splits);
+  return launch_ex(attn_tc_kernel<128>, grid, dim3(kTcThreads), smem, s, a.splits, pdl, m.q, m.tk,
+                   m.tv, m.ck, m.cv, a);
+}
+
+}  // namespace pf

@@ -1,0 +1,206 @@
+// Pieces shared by the two bf16 tree-attention kernels: the TMA loader of
+// one 64-token K/V tile (prefix cache, contiguous or paged, or the proposal's
+// own K/V) and the merge of split-KV partials across a thread-block cluster.
+#pragma once
+
+#include <cooperative_groups.h>
+#include <cuda_fp16.h>
+
+#include "pf_internal.h"
+#include "pf_ptx.cuh"
+
+namespace pf {
+
+constexpr int kBN = 64;  // tokens per KV tile
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+}
+
+template <int D>
+__device__ __forceinline__ void issue_kv_tile(const AttnArgs& a, const CUtensorMap* tm_ck,
+                                              const CUtensorMap* tm_cv, const CUtensorMap* tm_tk,
+                                              const CUtensorMap* tm_tv, uint8_t* stage,
+                                              uint32_t bar, int t, int n_ptiles, int b, int g,
+                                              int node0, int P) {
+  constexpr int kHalves = D / 64;
+  constexpr int kTileBytes = kBN * D * 2;
+  uint8_t* sk = stage;
+  uint8_t* sv = stage + kTileBytes;
+  if (t < n_ptiles) {
+    const int tok0 = t * kBN;
+    if (a.layout == PF_KV_CONTIGUOUS) {
+      mbar_arrive_expect_tx(bar, 2 * kTileBytes);
+#pragma unroll
+      for (int h = 0; h < kHalves; ++h) {
+        tma_load_3d(smem_u32(sk + h * kBN * 128), tm_ck, h * 64, tok0, b * a.Hkv + g, bar);
+        tma_load_3d(smem_u32(sv + h * kBN * 128), tm_cv, h * 64, tok0, b * a.Hkv + g, bar);
+      }
+    } else {
+      const int left = P - tok0;
+      const int npages = min(kBN / PF_PAGE_SIZE, (left + PF_PAGE_SIZE - 1) / PF_PAGE_SIZE);
+      mbar_arrive_expect_tx(bar, 2 * kHalves * npages * PF_PAGE_SIZE * 128);
+      const int32_t* pt = a.page_table + (size_t)b * a.pages_per_seq + tok0 / PF_PAGE_SIZE;
+      for (int p = 0; p < npages; ++p) {
+        const int page = pt[p];
+#pragma unroll
+        for (int h = 0; h < kHalves; ++h) {
+          const int off = h * kBN * 128 + p * PF_PAGE_SIZE * 128;
+          tma_load_4d(smem_u32(sk + off), tm_ck, h * 64, 0, g, page, bar);
+          tma_load_4d(smem_u32(sv + off), tm_cv, h * 64, 0, g, page, bar);
+        }
+      }
+    }
+  } else {
+    const int j = t - n_ptiles;
+    mbar_arrive_expect_tx(bar, 2 * kTileBytes);
+#pragma unroll
+    for (int h = 0; h < kHalves; ++h) {
+      tma_load_3d(smem_u32(sk + h * kBN * 128), tm_tk, h * 64, g, node0 + j * kBN, bar);
+      tma_load_3d(smem_u32(sv + h * kBN * 128), tm_tv, h * 64, g, node0 + j * kBN, bar);
+    }
+  }
+}
+
+// Merge of split-KV partials.  Every CTA of the cluster has published, for
+// its rows, the running maximum m (log2 domain), the sum l of exp2(s - m)
+// and the unnormalised O (fp32, row pitch D + 4) in its shared memory.  After
+// one cluster barrier, CTA `split` combines rows [split*per, (split+1)*per):
+//   M = max_q m_q,  w_q = exp2(m_q - M),  out = sum_q w_q O_q / sum_q w_q l_q
+// reading its peers' shared memory, one warp per row: lane q fetches peer
+// q's (m, l), shuffles reduce them, and each lane owns D/32 output columns,
+// issuing all of its peers' loads before accumulating.  A second barrier
+// keeps every CTA's shared memory alive until its peers are done.
+template <int D, int kThreads>
+__device__ __forceinline__ void cluster_merge(const AttnArgs& a,
+                                              cooperative_groups::cluster_group& cluster,
+                                              float* sM, float* sL, float* sO, int rows, int split,
+                                              int nsplit, int node_base, int g, int tid) {
+  constexpr int kOStride = D + 4;
+  constexpr int kMaxSplit = 16;
+  constexpr int CPL = D / 32;  // output columns per lane
+  static_assert(CPL == 2 || CPL == 4, "head_dim 64 or 128");
+  cluster.sync();
+  const int warp = tid >> 5, lane = tid & 31;
+  const int per = (rows + nsplit - 1) / nsplit;
+  const int lo = split * per, hi = min(rows, lo + per);
+  __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.out);
+  for (int r = lo + warp; r < hi; r += kThreads / 32) {
+    float mq = -INFINITY, lq = 0.f;
+    if (lane < nsplit) {
+      mq = cluster.map_shared_rank(sM, lane)[r];
+      lq = cluster.map_shared_rank(sL, lane)[r];
+    }
+    float M = mq;
+#pragma unroll
+    for (int off = 16; off; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    const float Mu = M == -INFINITY ? 0.f : M;
+    const float wq = lane < nsplit ? exp2f(mq - Mu) : 0.f;
+    float L = wq * lq;
+#pragma unroll
+    for (int off = 16; off; off >>= 1) L += __shfl_xor_sync(0xffffffffu, L, off);
+    float v[kMaxSplit][CPL];
+#pragma unroll
+    for (int q = 0; q < kMaxSplit; ++q) {
+      if (q < nsplit) {
+        const float* src = cluster.map_shared_rank(sO, q) + r * kOStride + lane * CPL;
+        if constexpr (CPL == 4) {
+          const float4 t = *reinterpret_cast<const float4*>(src);
+          v[q][0] = t.x;
+          v[q][1] = t.y;
+          v[q][2] = t.z;
+          v[q][3] = t.w;
+        } else {
+          const float2 t = *reinterpret_cast<const float2*>(src);
+          v[q][0] = t.x;
+          v[q][1] = t.y;
+        }
+      }
+    }
+    float acc[CPL];
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) acc[c] = 0.f;
+#pragma unroll
+    for (int q = 0; q < kMaxSplit; ++q) {
+      const float w = __shfl_sync(0xffffffffu, wq, q);
+      if (q < nsplit) {
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) acc[c] = fmaf(w, v[q][c], acc[c]);
+      }
+    }
+    const float inv = L > 0.f ? 1.f / L : 0.f;
+    const int node = node_base + r / a.G;
+    const int h = g * a.G + r % a.G;
+    __nv_bfloat16* dst = out + ((size_t)node * a.Hq + h) * D + lane * CPL;
+    if constexpr (CPL == 4) {
+      uint2 pk;
+      pk.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+      pk.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+      *reinterpret_cast<uint2*>(dst) = pk;
+    } else {
+      *reinterpret_cast<uint32_t*>(dst) = pack_bf16(acc[0] * inv, acc[1] * inv);
+    }
+  }
+  cluster.sync();
+}
+
+// Local half of the push-style merge: this CTA (rank `split`) owns rows
+// [split*per, split*per + cnt); peer s stored, for local row i, its
+// normalised partial (O / l, fp16, pitch kPitch halves) at inbox slot
+// s*per + i and its log2-sum-exp at lse[s*per + i].
+//   M = max_s lse_s,  w_s = 2^(lse_s - M),  out = sum_s w_s (O/l)_s / sum_s w_s
+// One thread per (row, 8 output columns); all loads are issued before use.
+template <int D, int kThreads, int kPitch>
+__device__ __forceinline__ void inbox_merge(const AttnArgs& a, const float* lse,
+                                            const __half* inbox, int rows, int split, int per,
+                                            int nsplit, int node_base, int g, int tid) {
+  constexpr int kMaxSplit = 16;
+  constexpr int C8 = D / 8;
+  const int cnt = min(per, rows - split * per);
+  __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.out);
+  for (int it = tid; it < cnt * C8; it += kThreads) {
+    const int i = it / C8, c8 = it - (it / C8) * C8;
+    float ls[kMaxSplit];
+    uint4 v[kMaxSplit];
+#pragma unroll
+    for (int q = 0; q < kMaxSplit; ++q) {
+      if (q < nsplit) {
+        ls[q] = lse[q * per + i];
+        v[q] = *reinterpret_cast<const uint4*>(inbox + (q * per + i) * kPitch + c8 * 8);
+      } else {
+        ls[q] = -INFINITY;
+      }
+    }
+    float M = -INFINITY;
+#pragma unroll
+    for (int q = 0; q < kMaxSplit; ++q) M = fmaxf(M, ls[q]);
+    const float Mu = M == -INFINITY ? 0.f : M;
+    float W = 0.f, acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int q = 0; q < kMaxSplit; ++q) {
+      if (q < nsplit) {
+        const float w = ls[q] == -INFINITY ? 0.f : exp2f(ls[q] - Mu);
+        W += w;
+        const __half2* h2 = reinterpret_cast<const __half2*>(&v[q]);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const float2 f = __half22float2(h2[c]);
+          acc[2 * c] = fmaf(w, f.x, acc[2 * c]);
+          acc[2 * c + 1] = fmaf(w, f.y, acc[2 * c + 1]);
+        }
+      }
+    }
+    const float inv = W > 0.f ? 1.f / W : 0.f;
+    const int r = split * per + i;
+    const int node = node_base + r / a.G;
+    const int h = g * a.G + r % a.G;
+    uint4 pk;
+    pk.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+    pk.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+    pk.z = pack_bf16(acc[4] * inv, acc[5] * inv);
+    pk.w = pack_bf16(acc[6] * inv, acc[7] * inv);
+    *reinterpret_cast<uint4*>(out + ((size_t)node * a.Hq + h) * D + c8 * 8) = pk;
+  }
+}
+
+}  // namespace pf

@@ -251,6 +251,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       mbar_arrive(smem_u32(&tempty[acc]));
     }
   }
+  __syncwarp();  // the producer and MMA lanes rejoin their warps before the barrier
 
   __syncthreads();
   if (threadIdx.x == 0 && s_misc[1] > s_misc[2]) {

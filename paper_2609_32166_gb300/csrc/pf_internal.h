@@ -51,6 +51,10 @@ int attention_bf16_smem_bytes(int D, int bm);
 // Whether a cluster of `cluster` CTAs of the bf16 attention kernel can be
 // resident at once on this device.
 bool attention_cluster_fits(int D, int bm, int cluster);
+// tcgen05 variant (bf16, D = 128, 128 query rows per CTA).
+cudaError_t launch_attention_tc(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl);
+bool attention_tc_cluster_fits(int cluster);
+int attention_tc_smem_bytes();
 
 // ------------------------------------------------------------ LM head
 struct LmArgs {

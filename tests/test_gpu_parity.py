@@ -86,6 +86,19 @@ def test_edge_cases(name):
     c.check_commit(res)
 
 
+@pytest.mark.parametrize("name", ["7b-tree64-small", "7b-batch8-paged-small"])
+def test_mma_sync_kernel(name, monkeypatch):
+    """The mma.sync attention kernel (selected with PF_ATTN_IMPL=mma) stays
+    correct at D = 128, where the tcgen05 kernel is the default."""
+    monkeypatch.setenv("PF_ATTN_IMPL", "mma")
+    c = Case(SMALL[name], seed=6)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for s in range(c.w.batch):
+        c.check_attention(0, s)
+
+
 def test_mixed_tree_sizes():
     """Sequences of 1, 17 and 128 nodes in one batch (variable cu_nodes)."""
     w = I.scaled(W["7b-bf16-batch8-paged"], layers=1, batch=3, prefix=(50, 400), nodes=128,

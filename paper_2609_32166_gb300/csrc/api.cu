@@ -124,14 +124,22 @@ int max_cluster_for(int kernel, int D, int want) {
   while (w > 8) {
     int& c = cache[dev & 63][kernel][di][w];
     if (c == 0) {
-      const bool fits = kernel == 3 ? pf::attention_tc_cluster_fits(w)
-                                    : pf::attention_cluster_fits(D, 32 << kernel, w);
+      const bool fits = pf::attention_cluster_fits(D, 32 << kernel, w);
       c = fits ? 1 : -1;
     }
     if (c > 0) break;
     w -= kernel == 3 ? 2 : 1;
   }
   return w;
+}
+
+int tc_max_active_clusters(int cluster) {
+  static int cache[64][17];
+  int dev = 0;
+  cudaGetDevice(&dev);
+  int& c = cache[dev & 63][cluster];
+  if (c == 0) c = std::max(1, pf::attention_tc_max_active_clusters(cluster)) + 1;
+  return c - 1;
 }
 
 // The tcgen05 kernel serves bf16 with D = 128 (PF_ATTN_IMPL=mma selects the
@@ -147,16 +155,16 @@ void choose_attention_shape(pf::AttnArgs& a, int max_prefix_len, int sms) {
     a.bm = 128;
     a.nb = 128 / a.G;
     a.rb_count = (a.max_nodes + a.nb - 1) / a.nb;
-    const int base = a.B * a.Hkv * a.rb_count;
-    int splits = sms / base;
-    if (const char* e = getenv("PF_ATTN_SPLITS")) splits = atoi(e);
-    splits = std::max(1, std::min({splits, 16, max_tiles}));
-    // even cluster sizes: clusters are placed on pairs of SMs, so an odd
-    // cluster of one-CTA-per-SM blocks strands an SM and can push the grid
-    // into a second wave
+    // One CTA per SM (shared memory), clusters must be co-resident: take the
+    // widest even split whose clusters all fit on the GPU at once, so the
+    // grid runs in one wave (odd cluster sizes strand SMs of an SM pair).
+    const int groups = a.B * a.Hkv * a.rb_count;
+    int splits = std::min(16, max_tiles);
     if (splits > 1) splits &= ~1;
-    if (splits > 8) splits = max_cluster_for(3, a.D, splits);
-    a.splits = splits;
+    for (; splits > 1; splits -= 2)
+      if (tc_max_active_clusters(splits) >= groups) break;
+    if (const char* e = getenv("PF_ATTN_SPLITS")) splits = std::max(1, std::min(16, atoi(e)));
+    a.splits = std::max(1, splits);
     return;
   }
   const int bms[3] = {128, 64, 32};

@@ -375,15 +375,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
 int attention_tc_smem_bytes() { return TcSmem<128>::kTotal + 1024; }
 
-bool attention_tc_cluster_fits(int cluster) {
+int attention_tc_max_active_clusters(int cluster) {
   const int smem = TcSmem<128>::kTotal + 1024;
   static int limit[64] = {};
-  if (ensure_smem_limit((const void*)attn_tc_kernel<128>, smem, limit) != cudaSuccess)
-    return false;
+  if (ensure_smem_limit((const void*)attn_tc_kernel<128>, smem, limit) != cudaSuccess) return 0;
   if (cluster > 8 && cudaFuncSetAttribute(attn_tc_kernel<128>,
                                           cudaFuncAttributeNonPortableClusterSizeAllowed,
                                           1) != cudaSuccess)
-    return false;
+    return 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(cluster);
   cfg.blockDim = dim3(kTcThreads);
@@ -398,9 +397,9 @@ bool attention_tc_cluster_fits(int cluster) {
   int n = 0;
   if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<128>, &cfg) != cudaSuccess) {
     cudaGetLastError();
-    return false;
+    return 0;
   }
-  return n > 0;
+  return n;
 }
 
 cudaError_t launch_attention_tc(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl) {

@@ -62,6 +62,46 @@ __device__ __forceinline__ void issue_kv_tile(const AttnArgs& a, const CUtensorM
   }
 }
 
+// TMA load of one 64-token tile of ONE matrix (K or V): from the prefix
+// cache (contiguous: one 3-D box per 64-column half; paged: one 4-D box per
+// 16-token page, only the pages that hold prefix rows) or, past the prefix,
+// from the proposal's own rows.  Arms `bar` with the bytes it will bring.
+template <int D>
+__device__ __forceinline__ void issue_one_tile(const AttnArgs& a, const CUtensorMap* tm_cache,
+                                               const CUtensorMap* tm_tree, uint8_t* dst,
+                                               uint32_t bar, int t, int n_ptiles, int b, int g,
+                                               int node0, int P) {
+  constexpr int kHalves = D / 64;
+  constexpr int kTileBytes = kBN * D * 2;
+  if (t < n_ptiles) {
+    const int tok0 = t * kBN;
+    if (a.layout == PF_KV_CONTIGUOUS) {
+      mbar_arrive_expect_tx(bar, kTileBytes);
+#pragma unroll
+      for (int h = 0; h < kHalves; ++h)
+        tma_load_3d(smem_u32(dst + h * kBN * 128), tm_cache, h * 64, tok0, b * a.Hkv + g, bar);
+    } else {
+      const int left = P - tok0;
+      const int npages = min(kBN / PF_PAGE_SIZE, (left + PF_PAGE_SIZE - 1) / PF_PAGE_SIZE);
+      mbar_arrive_expect_tx(bar, kHalves * npages * PF_PAGE_SIZE * 128);
+      const int32_t* pt = a.page_table + (size_t)b * a.pages_per_seq + tok0 / PF_PAGE_SIZE;
+      for (int p = 0; p < npages; ++p) {
+        const int page = pt[p];
+#pragma unroll
+        for (int h = 0; h < kHalves; ++h)
+          tma_load_4d(smem_u32(dst + h * kBN * 128 + p * PF_PAGE_SIZE * 128), tm_cache, h * 64, 0,
+                      g, page, bar);
+      }
+    }
+  } else {
+    const int j = t - n_ptiles;
+    mbar_arrive_expect_tx(bar, kTileBytes);
+#pragma unroll
+    for (int h = 0; h < kHalves; ++h)
+      tma_load_3d(smem_u32(dst + h * kBN * 128), tm_tree, h * 64, g, node0 + j * kBN, bar);
+  }
+}
+
 // Merge of split-KV partials.  Every CTA of the cluster has published, for
 // its rows, the running maximum m (log2 domain), the sum l of exp2(s - m)
 // and the unnormalised O (fp32, row pitch D + 4) in its shared memory.  After

@@ -53,7 +53,8 @@ int attention_bf16_smem_bytes(int D, int bm);
 bool attention_cluster_fits(int D, int bm, int cluster);
 // tcgen05 variant (bf16, D = 128, 128 query rows per CTA).
 cudaError_t launch_attention_tc(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl);
-bool attention_tc_cluster_fits(int cluster);
+// How many clusters of `cluster` CTAs of the tcgen05 kernel fit at once.
+int attention_tc_max_active_clusters(int cluster);
 int attention_tc_smem_bytes();
 
 // ------------------------------------------------------------ LM head

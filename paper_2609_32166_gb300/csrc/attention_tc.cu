@@ -45,15 +45,16 @@ struct TcSmem {
   static constexpr int kQOff = kTcStages * kStageBytes;
   static constexpr int kPOff = kQOff + kQBytes;
   // Merge inbox: one slot per (split, row) a CTA may receive, at most
-  // splits * ceil(rows / splits) <= 128 + 15 slots: the normalised partial
-  // O / l in fp16 (pitch D + 8 halves) and its log2-sum-exp.
+  // splits * ceil(rows / splits) <= 128 + 15 slots.  A slot holds the
+  // normalised partial O / l in fp16 (D halves) followed by its log2-sum-exp
+  // (one float) in the 16-byte pad; the same format is staged locally.
   static constexpr int kInboxSlots = 144;
   static constexpr int kInboxPitch = D + 8;              // halves
   static constexpr int kInboxOff = kPOff + 2 * kPBytes;
   static constexpr int kLseOff = kInboxOff + kInboxSlots * kInboxPitch * 2;
   static constexpr int kBarOff = kLseOff + kInboxSlots * 4;
-  // kv_full[3] kv_empty[3] q_full s_full[2] s_empty[2] p_full[2] pv_done[2]
-  static constexpr int kNumBars = 2 * kTcStages + 9;
+  // kv_full[3] kv_empty[3] q_full s_full[2] s_empty[2] p_full[2] pv_done[2] inbox
+  static constexpr int kNumBars = 2 * kTcStages + 10;
   static constexpr int kTotal = kBarOff + kNumBars * 8 + 16;
   static_assert(kTotal + 1024 <= 232448, "shared memory budget");
 };
@@ -72,7 +73,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   uint8_t* sQ = smem + S::kQOff;
   uint8_t* sP = smem + S::kPOff;
   __half* sInbox = reinterpret_cast<__half*>(smem + S::kInboxOff);
-  float* sLse = reinterpret_cast<float*>(smem + S::kLseOff);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S::kBarOff);
   uint64_t* kv_full = bars;
   uint64_t* kv_empty = bars + kTcStages;
@@ -81,6 +81,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   uint64_t* s_empty = s_full + 2;
   uint64_t* p_full = s_empty + 2;
   uint64_t* pv_done = p_full + 2;
+  uint64_t* inbox_full = pv_done + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + S::kNumBars);
 
   cg::cluster_group cluster = cg::this_cluster();
@@ -129,6 +130,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       mbar_init(smem_u32(&p_full[i]), 128);
       mbar_init(smem_u32(&pv_done[i]), 1);
     }
+    mbar_init(smem_u32(inbox_full), 1);
     fence_mbar_init();
     for (int i = 0; i < first; ++i)
       if (t_begin + i < n_ptiles)
@@ -155,6 +157,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // Peers may signal this CTA's inbox barrier only after it is initialised:
+  // arrive now, wait just before sending partials.  (A single split is
+  // launched without a cluster and uses no cluster feature at all.)
+  if (nsplit > 1) cluster_arrive_release();
   pdl_launch_dependents();
 
   float m_ref = -INFINITY, l = 0.f;   // softmax threads: running max (log2) and sum of their row
@@ -323,52 +329,103 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   }
   __syncwarp();  // the producer and MMA lanes rejoin their warps before the barriers
 
-  // ---- split-KV merge, push style.  Each row's partial result, normalised
-  // (O / l, fp16) with its log2-sum-exp lse = m + log2(l), is stored straight
-  // into a dedicated inbox in the shared memory of the CTA that merges that
-  // row (posted remote stores; the inbox is never touched by the KV loop, so
-  // no barrier is needed before them).  One cluster barrier makes them
-  // visible; each CTA then merges its rows from local shared memory:
+  // ---- split-KV merge.  Each row's partial result, normalised (O / l,
+  // fp16) with its log2-sum-exp lse = m + log2(l) in the row's pad, is
+  // staged in this CTA's (now idle) KV ring, row r at slot r, so the rows
+  // each peer merges are contiguous.  One bulk copy per peer moves them into
+  // the peer's inbox and completes on the peer's inbox barrier, which
+  // expects one block from every CTA of the cluster; the peer then merges
+  // from its own shared memory:
   //   out = sum_s 2^(lse_s - M) (O/l)_s / sum_s 2^(lse_s - M),  M = max_s lse_s
+  if (nsplit == 1) {
+    // ---- single split: O / l is the output
+    if (warp >= 2) {
+      const int quad = warp & 3;
+      const int r = quad * 32 + lane;
+      const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+      const float inv_l = (my_tiles > 0 && l > 0.f) ? 1.f / l : 0.f;
+      uint32_t ov[D];
+#pragma unroll
+      for (int c0 = 0; c0 < D; c0 += 32)
+        tmem_ld_32(tmem + lane_base + 2 * kBN + c0, *reinterpret_cast<uint32_t(*)[32]>(&ov[c0]));
+      tmem_ld_wait();
+      if (r < rows) {
+        const int node = node0 + nfirst + r / a.G;
+        const int h = g * a.G + r % a.G;
+        __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(a.out) + ((size_t)node * a.Hq + h) * D;
+#pragma unroll
+        for (int c = 0; c < D; c += 8) {
+          uint4 pk;
+          pk.x = pack_bf16(__uint_as_float(ov[c]) * inv_l, __uint_as_float(ov[c + 1]) * inv_l);
+          pk.y = pack_bf16(__uint_as_float(ov[c + 2]) * inv_l, __uint_as_float(ov[c + 3]) * inv_l);
+          pk.z = pack_bf16(__uint_as_float(ov[c + 4]) * inv_l, __uint_as_float(ov[c + 5]) * inv_l);
+          pk.w = pack_bf16(__uint_as_float(ov[c + 6]) * inv_l, __uint_as_float(ov[c + 7]) * inv_l);
+          *reinterpret_cast<uint4*>(dst + c) = pk;
+        }
+      }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+      tc_fence_after();
+      tmem_dealloc(tmem, kTmemCols);
+    }
+    return;
+  }
   const int per = (rows + nsplit - 1) / nsplit;
+  const int cnt_mine = max(0, min(per, rows - split * per));
+  constexpr int kRowBytes = S::kInboxPitch * 2;
+  __half* stage_rows = reinterpret_cast<__half*>(sKV);
+  if (tid == 0)
+    mbar_arrive_expect_tx(smem_u32(inbox_full), (uint32_t)(nsplit * cnt_mine * kRowBytes));
   if (warp >= 2) {
     const int quad = warp & 3;
     const int r = quad * 32 + lane;
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
-    const bool valid_row = r < rows;
-    const int owner = valid_row ? r / per : 0;
-    const int slot = split * per + (r - owner * per);
     const float inv_l = (my_tiles > 0 && l > 0.f) ? 1.f / l : 0.f;
-    __half* dst = cluster.map_shared_rank(sInbox, owner) + slot * S::kInboxPitch;
+    uint32_t ov[D];  // the whole O row: all TMEM loads in flight behind one wait
 #pragma unroll
-    for (int c0 = 0; c0 < D; c0 += 32) {
-      uint32_t ov[32];
-      tmem_ld_32(tmem + lane_base + 2 * kBN + c0, ov);
-      tmem_ld_wait();
-      if (valid_row) {
+    for (int c0 = 0; c0 < D; c0 += 32)
+      tmem_ld_32(tmem + lane_base + 2 * kBN + c0, *reinterpret_cast<uint32_t(*)[32]>(&ov[c0]));
+    tmem_ld_wait();
+    if (r < rows) {
+      __half* dst = stage_rows + r * S::kInboxPitch;
 #pragma unroll
-        for (int c = 0; c < 32; c += 8) {
-          uint4 pk;
-          pk.x = pack_half(__uint_as_float(ov[c]) * inv_l, __uint_as_float(ov[c + 1]) * inv_l);
-          pk.y = pack_half(__uint_as_float(ov[c + 2]) * inv_l, __uint_as_float(ov[c + 3]) * inv_l);
-          pk.z = pack_half(__uint_as_float(ov[c + 4]) * inv_l, __uint_as_float(ov[c + 5]) * inv_l);
-          pk.w = pack_half(__uint_as_float(ov[c + 6]) * inv_l, __uint_as_float(ov[c + 7]) * inv_l);
-          *reinterpret_cast<uint4*>(dst + c0 + c) = pk;
-        }
+      for (int c = 0; c < D; c += 8) {
+        uint4 pk;
+        pk.x = pack_half(__uint_as_float(ov[c]) * inv_l, __uint_as_float(ov[c + 1]) * inv_l);
+        pk.y = pack_half(__uint_as_float(ov[c + 2]) * inv_l, __uint_as_float(ov[c + 3]) * inv_l);
+        pk.z = pack_half(__uint_as_float(ov[c + 4]) * inv_l, __uint_as_float(ov[c + 5]) * inv_l);
+        pk.w = pack_half(__uint_as_float(ov[c + 6]) * inv_l, __uint_as_float(ov[c + 7]) * inv_l);
+        *reinterpret_cast<uint4*>(dst + c) = pk;
       }
+      *reinterpret_cast<float*>(dst + D) = inv_l > 0.f ? m_ref + __log2f(l) : -INFINITY;
     }
-    if (valid_row)
-      cluster.map_shared_rank(sLse, owner)[slot] =
-          inv_l > 0.f ? m_ref + __log2f(l) : -INFINITY;
   }
+  fence_proxy_async_smem();  // staged rows are read by the bulk-copy engine
   tc_fence_before();
-  cluster.sync();
+  __syncthreads();
+  cluster_wait_acquire();    // every peer's inbox barrier is initialised
+  if (tid < nsplit) {
+    const int q = tid;
+    const int cnt = min(per, rows - q * per);
+    if (cnt > 0) {
+      const uint32_t src = smem_u32(stage_rows + q * per * S::kInboxPitch);
+      const uint32_t dst = mapa_cluster(smem_u32(sInbox + split * per * S::kInboxPitch), q);
+      bulk_copy_s2cluster(dst, src, (uint32_t)(cnt * kRowBytes),
+                          mapa_cluster(smem_u32(inbox_full), q));
+      bulk_commit_group();
+    }
+  }
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
-  inbox_merge<D, kTcThreads, S::kInboxPitch>(a, sLse, sInbox, rows, split, per, nsplit,
-                                             node0 + nfirst, g, tid);
+  if (cnt_mine > 0) mbar_wait(smem_u32(inbox_full), 0, a.err);
+  inbox_merge<D, kTcThreads, S::kInboxPitch>(a, sInbox, rows, split, per, nsplit, node0 + nfirst,
+                                             g, tid);
+  // this CTA's staged rows must stay readable until its copies have left
+  if (tid < nsplit) bulk_wait_read_all();
 }
 
 }  // namespace

@@ -184,16 +184,16 @@ __device__ __forceinline__ void cluster_merge(const AttnArgs& a,
   cluster.sync();
 }
 
-// Local half of the push-style merge: this CTA (rank `split`) owns rows
-// [split*per, split*per + cnt); peer s stored, for local row i, its
-// normalised partial (O / l, fp16, pitch kPitch halves) at inbox slot
-// s*per + i and its log2-sum-exp at lse[s*per + i].
+// Local half of the split-KV merge: this CTA (rank `split`) owns rows
+// [split*per, split*per + cnt); peer s delivered, for local row i, its
+// normalised partial (O / l, fp16) followed by its log2-sum-exp (a float in
+// the row's pad) at inbox slot s*per + i (pitch kPitch halves).
 //   M = max_s lse_s,  w_s = 2^(lse_s - M),  out = sum_s w_s (O/l)_s / sum_s w_s
 // One thread per (row, 8 output columns); all loads are issued before use.
 template <int D, int kThreads, int kPitch>
-__device__ __forceinline__ void inbox_merge(const AttnArgs& a, const float* lse,
-                                            const __half* inbox, int rows, int split, int per,
-                                            int nsplit, int node_base, int g, int tid) {
+__device__ __forceinline__ void inbox_merge(const AttnArgs& a, const __half* inbox, int rows,
+                                            int split, int per, int nsplit, int node_base, int g,
+                                            int tid) {
   constexpr int kMaxSplit = 16;
   constexpr int C8 = D / 8;
   const int cnt = min(per, rows - split * per);
@@ -205,8 +205,9 @@ __device__ __forceinline__ void inbox_merge(const AttnArgs& a, const float* lse,
 #pragma unroll
     for (int q = 0; q < kMaxSplit; ++q) {
       if (q < nsplit) {
-        ls[q] = lse[q * per + i];
-        v[q] = *reinterpret_cast<const uint4*>(inbox + (q * per + i) * kPitch + c8 * 8);
+        const __half* slot = inbox + (q * per + i) * kPitch;
+        ls[q] = *reinterpret_cast<const float*>(slot + D);
+        v[q] = *reinterpret_cast<const uint4*>(slot + c8 * 8);
       } else {
         ls[q] = -INFINITY;
       }
@@ -219,7 +220,7 @@ __device__ __forceinline__ void inbox_merge(const AttnArgs& a, const float* lse,
 #pragma unroll
     for (int q = 0; q < kMaxSplit; ++q) {
       if (q < nsplit) {
-        const float w = ls[q] == -INFINITY ? 0.f : exp2f(ls[q] - Mu);
+        const float w = ex2_approx(ls[q] - Mu);  // -inf -> 0
         W += w;
         const __half2* h2 = reinterpret_cast<const __half2*>(&v[q]);
 #pragma unroll
@@ -230,7 +231,7 @@ __device__ __forceinline__ void inbox_merge(const AttnArgs& a, const float* lse,
         }
       }
     }
-    const float inv = W > 0.f ? 1.f / W : 0.f;
+    const float inv = W > 0.f ? __fdividef(1.f, W) : 0.f;
     const int r = split * per + i;
     const int node = node_base + r / a.G;
     const int h = g * a.G + r % a.G;

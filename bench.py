@@ -360,11 +360,12 @@ def main():
     # one graph = G steps; each step: flush, tokens | e0 attention e1 lmhead e2 commit e3
     per_step, attn_t, lm_t, commit_t = [], [], [], []
 
-    def collect(e):
+    def collect(e, parts=True):
         per_step.append(e[0].elapsed_time(e[3]))
-        attn_t.append(e[0].elapsed_time(e[1]))
-        lm_t.append(e[1].elapsed_time(e[2]))
-        commit_t.append(e[2].elapsed_time(e[3]))
+        if parts:
+            attn_t.append(e[0].elapsed_time(e[1]))
+            lm_t.append(e[1].elapsed_time(e[2]))
+            commit_t.append(e[2].elapsed_time(e[3]))
 
     try:
         torch.cuda.Event(enable_timing=True, external=True)
@@ -374,6 +375,10 @@ def main():
     clocks = ClockSampler(torch.cuda.current_device())
     if graph_events:
         R = K // G
+        # step boundaries carry events in every step; the part boundaries
+        # (which break the programmatic-dependent-launch chain between the
+        # last layer, the LM head and the commit) only in the first step of
+        # each graph, which provides the per-kernel breakdown
         ev = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(4)]
               for _ in range(G)]
         graph = torch.cuda.CUDAGraph()
@@ -385,9 +390,11 @@ def main():
                 ev[g][0].record(s)
                 for l in range(vs.L):
                     vs.attention(l, s.cuda_stream)
-                ev[g][1].record(s)
+                if g == 0:
+                    ev[g][1].record(s)
                 vs.lmhead(s.cuda_stream)
-                ev[g][2].record(s)
+                if g == 0:
+                    ev[g][2].record(s)
                 vs.commit(s.cuda_stream)
                 ev[g][3].record(s)
         with torch.cuda.stream(stream):
@@ -405,7 +412,7 @@ def main():
                 # before the next replay overwrites them
                 stream.synchronize()
                 for g in range(G):
-                    collect(ev[g])
+                    collect(ev[g], parts=(g == 0))
     else:
         # torch without external graph events: one graph per part, events
         # recorded between graph launches
@@ -497,7 +504,9 @@ def main():
                                "unit": "GB/s", "frac": attn_b_layer * w.layers /
                                (attn_ms * 1e-3) / 1e9 / hbm_peak},
         "gpu_launches": K * vs.launches_per_step(),
-        "timing": ("CUDA graph of G steps, external event nodes around each step's parts"
+        "timing": ("CUDA graphs of %d steps; event nodes at every step boundary, and around "
+                   "the attention / LM-head / commit parts of the first step of each graph "
+                   "(those give the per-part times)" % G
                    if graph_events else "one CUDA graph per part, events between graph launches"),
         "clocks": clk,
         "e2e": e2e,

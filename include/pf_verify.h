@@ -200,7 +200,15 @@ typedef struct pf_lm_desc {
   int32_t* out_tokens;         /* out device [B][max_nodes]                  */
   int32_t* last_node;          /* out device [B], optional                   */
   int32_t* error_flag;         /* optional device int32                      */
+  int32_t flags;               /* PF_LM_* bits, 0 = none                     */
 } pf_lm_desc;
+
+/* PF_LM_EARLY_WEIGHT: the weight was written before the kernel that precedes
+ * this call in the stream started (model weights normally are).  The kernel
+ * then starts streaming its first weight tiles before waiting for that
+ * preceding kernel to finish (programmatic dependent launch); the hidden
+ * states, tokens and tree are read only after it finishes. */
+#define PF_LM_EARLY_WEIGHT 1
 
 PF_API size_t pf_lmhead_accept_workspace_size(const pf_lm_desc* d);
 PF_API pf_status pf_lmhead_accept(const pf_lm_desc* d, void* workspace, size_t workspace_bytes,

@@ -27,6 +27,7 @@ PF_KV_CONTIGUOUS, PF_KV_PAGED = 0, 1
 PF_MAX_NODES, PF_MASK_WORDS, PF_PAGE_SIZE, PF_MAX_LM_ROWS = 128, 2, 16, 256
 PF_DEVERR_TIMEOUT, PF_DEVERR_CAPACITY, PF_DEVERR_BOUNDS = 1, 2, 4
 PF_ATTN_EARLY_PREFETCH = 1
+PF_LM_EARLY_WEIGHT = 1
 
 STATUS_NAMES = {0: "PF_OK", 1: "PF_ERR_NULL", 2: "PF_ERR_SHAPE", 3: "PF_ERR_DTYPE",
                 4: "PF_ERR_TREE", 5: "PF_ERR_CAPACITY", 6: "PF_ERR_ALIGN", 7: "PF_ERR_CUDA",
@@ -67,7 +68,7 @@ class pf_lm_desc(C.Structure):
                 ("argmax", C.c_void_p), ("max_logit", C.c_void_p),
                 ("accept_len", C.c_void_p), ("path", C.c_void_p),
                 ("out_tokens", C.c_void_p), ("last_node", C.c_void_p),
-                ("error_flag", C.c_void_p)]
+                ("error_flag", C.c_void_p), ("flags", C.c_int32)]
 
 
 class pf_commit_desc(C.Structure):

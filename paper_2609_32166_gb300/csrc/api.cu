@@ -393,6 +393,8 @@ pf_status pf_lmhead_accept(const pf_lm_desc* d, void* workspace, size_t workspac
   a.best = static_cast<unsigned long long*>(workspace);
   a.ticket = reinterpret_cast<unsigned int*>(static_cast<char*>(workspace) + 8 * PF_MAX_LM_ROWS);
   a.err = d->error_flag;
+  if (d->flags & ~PF_LM_EARLY_WEIGHT) return fail(PF_ERR_SHAPE, "%s: unknown flags", who);
+  a.flags = d->flags;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int sms = num_sms();
   if (sms <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);

@@ -156,6 +156,22 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     s_misc[1] = 0;
     s_misc[2] = 0;
   }
+  // With PF_LM_EARLY_WEIGHT the first `pre` stages of weight tiles are
+  // requested before waiting for the preceding kernel (programmatic
+  // dependent launch); their hidden-state halves follow after the wait.
+  const int my_tiles = blockIdx.x < a.num_tiles
+                           ? (a.num_tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1
+                           : 0;
+  const int pre = (a.flags & PF_LM_EARLY_WEIGHT) ? min(ns, my_tiles * a.nk) : 0;
+  if (threadIdx.x == 0) {
+    const uint64_t pol = l2_policy_evict_first();
+    for (int it = 0; it < pre; ++it) {
+      const int tile = blockIdx.x + (it / a.nk) * gridDim.x, kc = it % a.nk;
+      const uint32_t fb = smem_u32(&full[it]);
+      mbar_arrive_expect_tx(fb, kABytes + b_bytes);
+      tma_load_2d_hint(smem_u32(sA + it * kABytes), &tm_w, kc * kBK, tile * kBM, fb, pol);
+    }
+  }
   for (int i = threadIdx.x; i < PF_MAX_LM_ROWS; i += blockDim.x) s_best[i] = 0ull;
 
   // Wait for whatever produced the hidden states (programmatic dependent
@@ -179,13 +195,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       for (int tile = blockIdx.x; tile < a.num_tiles && ok; tile += gridDim.x) {
         for (int kc = 0; kc < a.nk; ++kc, ++it) {
           const int st = it % ns;
-          if (!mbar_wait(smem_u32(&empty[st]), ((it / ns) & 1) ^ 1, a.err)) {
-            ok = false;
-            break;
-          }
           const uint32_t fb = smem_u32(&full[st]);
-          mbar_arrive_expect_tx(fb, kABytes + b_bytes);
-          tma_load_2d_hint(smem_u32(sA + st * kABytes), &tm_w, kc * kBK, tile * kBM, fb, pol);
+          if (it >= pre) {
+            if (!mbar_wait(smem_u32(&empty[st]), ((it / ns) & 1) ^ 1, a.err)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(fb, kABytes + b_bytes);
+            tma_load_2d_hint(smem_u32(sA + st * kABytes), &tm_w, kc * kBK, tile * kBM, fb, pol);
+          }
           tma_load_2d(smem_u32(sB + st * b_bytes), &tm_h, kc * kBK, 0, fb);
           s_misc[1] = it + 1;
         }

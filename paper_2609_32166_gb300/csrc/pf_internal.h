@@ -64,6 +64,7 @@ struct LmArgs {
   int num_tiles;   // ceil(V / 128)
   int nk;          // ceil(H / 64)
   int stages;      // TMA pipeline depth
+  int flags;       // PF_LM_* flags
   const int32_t* cu_nodes;
   const int32_t* tokens;
   const int32_t* parent;

@@ -158,6 +158,7 @@ class VerifyStep:
         d.accept_len, d.path = self.accept_len.data_ptr(), self.path.data_ptr()
         d.out_tokens, d.last_node = self.out_tokens.data_ptr(), self.last_node.data_ptr()
         d.error_flag = self.err.data_ptr()
+        d.flags = pb.PF_LM_EARLY_WEIGHT  # nothing in the step writes the weight
         self.lm_desc = d
         c = pb.pf_commit_desc()
         c.dtype, c.batch, c.n_layers = dt, w.batch, self.L

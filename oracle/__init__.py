@@ -12,8 +12,10 @@ Modules
   accept     greedy descent of the proposal tree (accepted length, tokens, path)
   commit     copy of the accepted path's K/V rows into the cache
   step       one whole verify step for one sequence, built from the above
+  rope       rolling-image carryover: keys re-rotated to a new position
+  retrieval  decoding-memory lookup: int8 query key, token-filtered cosine top-1
 
 Every function is pinned by tests under ``tests/`` against brute force,
 library special cases, closed forms and hand-derived fixtures.
 """
-from . import tree, attention, lmhead, accept, commit, step  # noqa: F401
+from . import tree, attention, lmhead, accept, commit, step, rope, retrieval  # noqa: F401

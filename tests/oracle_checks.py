@@ -336,3 +336,141 @@ def check_tree_structure(validate, depths, ancestors):
     assert ancestors(parent, 5) == {0, 2, 5}
     assert ancestors(parent, 0) == {0}
 
+
+
+# ----------------------------------------------------------------------------
+# rotary re-rotation (rolling-image carryover)
+# ----------------------------------------------------------------------------
+def _complex_rope(x, position, base):
+    """Rotary embedding written as complex multiplication: pair i is the
+    complex number x_i + 1j * x_{i+D/2}, turned by exp(1j * position * theta_i)."""
+    x = np.asarray(x, dtype=np.float64)
+    D = x.shape[-1]
+    theta = np.array([base ** (-(2.0 * i) / D) for i in range(D // 2)])
+    z = (x[..., : D // 2] + 1j * x[..., D // 2:]) * np.exp(1j * position * theta)
+    return np.concatenate([z.real, z.imag], axis=-1)
+
+
+def check_rope_golden(carry):
+    g = read_kv("rope_worked.txt")
+    out = carry(np.array(_nums(g["key"])), float(g["m"]), float(g["m_new"]), float(g["base"]))
+    np.testing.assert_allclose(out, _nums(g["expect"]), rtol=0, atol=1e-9)
+
+
+def check_rope_carry_is_relative(carry, seed=10):
+    """Carrying a key rotated at m to m' equals embedding the raw key at m'
+    (complex-multiplication form), for several shifts, both directions."""
+    rng = np.random.default_rng(seed)
+    for D, base in ((8, 10000.0), (64, 1e6), (128, 1e6)):
+        k = rng.standard_normal((3, D))
+        for m, m_new in ((0, 7), (1300, 17), (5, 4096), (123, 123)):
+            got = carry(_complex_rope(k, m, base), m, m_new, base)
+            np.testing.assert_allclose(got, _complex_rope(k, m_new, base), rtol=0, atol=1e-9)
+            np.testing.assert_allclose(np.linalg.norm(got, axis=-1), np.linalg.norm(k, axis=-1),
+                                       rtol=1e-12)
+
+
+def check_rope_block_move(shift, carry, seed=11):
+    """shift_block: destination rows hold the re-rotated keys and the copied
+    values; every other row keeps its contents; left and right moves, with
+    and without overlap."""
+    rng = np.random.default_rng(seed)
+    Hkv, S, D, base = 2, 40, 8, 10000.0
+    for src, dst, n in ((20, 5, 10), (5, 9, 12), (30, 2, 6), (0, 0, 4)):
+        K = rng.standard_normal((Hkv, S, D))
+        V = rng.standard_normal((Hkv, S, D))
+        K2, V2 = shift(K, V, src, dst, n, base)
+        for pos in range(S):
+            if dst <= pos < dst + n:
+                j = pos - dst
+                np.testing.assert_allclose(K2[:, pos], carry(K[:, src + j], src + j, pos, base),
+                                           rtol=0, atol=1e-12)
+                np.testing.assert_array_equal(V2[:, pos], V[:, src + j])
+            else:
+                np.testing.assert_array_equal(K2[:, pos], K[:, pos])
+                np.testing.assert_array_equal(V2[:, pos], V[:, pos])
+
+
+ROPE_CHECKS = [check_rope_golden, check_rope_carry_is_relative]
+
+
+# ----------------------------------------------------------------------------
+# decoding-memory retrieval
+# ----------------------------------------------------------------------------
+def _ints_rows(s):
+    return np.array([[int(x) for x in r.split()] for r in s.split("|")], dtype=np.int8)
+
+
+def check_retrieval_golden(top1):
+    g = read_kv("retrieval_worked.txt")
+    q = np.array([int(x) for x in g["q"].split()], dtype=np.int8)
+    best, sim = top1(q, _ints_rows(g["keys"]), _ints(g["entry_token"]), _ints(g["entry_pos"]),
+                     _ints(g["entry_bound"]), int(g["token"]))
+    assert best == int(g["best"]) and abs(sim - float(g["similarity"])) < 1e-12
+
+
+def check_retrieval_float_bruteforce(top1, seed=12):
+    """Random int8 keys without near ties: the exact selection equals numpy's
+    float64 cosine argmax over the eligible entries."""
+    rng = np.random.default_rng(seed)
+    for trial in range(20):
+        M, D = 200, 32
+        keys = rng.integers(-127, 128, size=(M, D)).astype(np.int8)
+        q = rng.integers(-127, 128, size=D).astype(np.int8)
+        tok = rng.integers(0, 4, size=M)
+        pos = rng.integers(0, 10, size=M)
+        bound = rng.integers(0, 10, size=M)
+        y = int(rng.integers(0, 4))
+        kf = keys.astype(np.float64)
+        cos = kf @ q.astype(np.float64) / (np.linalg.norm(kf, axis=1) * np.linalg.norm(q))
+        elig = (tok == y) & (pos < bound)
+        best, sim = top1(q, keys, tok, pos, bound, y)
+        if not elig.any():
+            assert best == -1
+            continue
+        c = np.where(elig, cos, -np.inf)
+        order = np.sort(c[elig])
+        if len(order) > 1 and order[-1] - order[-2] < 1e-9:
+            continue
+        assert best == int(np.argmax(c)) and abs(sim - c.max()) < 1e-12
+
+
+def check_retrieval_ties_and_ranges(top1):
+    q = np.array([5, -3, 2, 0], dtype=np.int8)
+    base = np.array([2, -1, 1, 0], dtype=np.int8)
+    keys = np.stack([base * 3, base, base * 2, -base, base * 3]).astype(np.int8)
+    tok = [1, 1, 1, 1, 1]
+    pos = [0, 0, 0, 0, 0]
+    bound = [1, 1, 1, 1, 1]
+    assert top1(q, keys, tok, pos, bound, 1)[0] == 0          # equal cosines: lowest index
+    assert top1(q, keys, tok, pos, bound, 1, lo=1)[0] == 1
+    assert top1(q, keys, tok, pos, bound, 1, lo=3, hi=4)[0] == 3  # only a negative cosine left
+    assert top1(q, keys, tok, pos, bound, 2)[0] == -1         # no entry with the token
+    assert top1(q, keys, tok, pos, [0, 0, 0, 0, 0], 1)[0] == -1  # every entry at its boundary
+
+
+def check_project_key(project):
+    rng = np.random.default_rng(13)
+    H = 96
+    proj = rng.standard_normal((256, H))
+    for _ in range(5):
+        h = rng.standard_normal(H)
+        key, x = project(h, proj)
+        assert key.dtype == np.int8 and key.shape == (256,)
+        assert np.abs(key).max() == 127
+        assert np.array_equal(project(3.5 * h, proj)[0], key)   # scale of h is irrelevant
+        z = proj @ (h / np.linalg.norm(h))
+        assert np.dot(key, z) / (np.linalg.norm(key.astype(float)) * np.linalg.norm(z)) > 0.999
+        assert np.all(np.abs(x - key) <= 0.5)
+    # half-way values round to even
+    proj2 = np.zeros((256, 4))
+    proj2[0, 0] = 254.0       # -> 127 (the maximum)
+    proj2[1, 0] = 5.0         # 127 * 5 / 254 = 2.5 -> 2
+    proj2[2, 0] = 7.0         # 3.5 -> 4
+    proj2[3, 0] = -3.0        # -1.5 -> -2
+    key, _ = project(np.array([1.0, 0, 0, 0]), proj2)
+    assert list(key[:4]) == [127, 2, 4, -2]
+
+
+RETRIEVAL_CHECKS = [check_retrieval_golden, check_retrieval_float_bruteforce,
+                    check_retrieval_ties_and_ranges]

@@ -202,3 +202,133 @@ def test_step_composes_the_parts():
     r = oracle.step.verify_step(layers, hidden, weight, parent, tokens, P)
     assert r["accept_len"] == 2 and r["path"] == [0, 1, 2] and r["new_len"] == P + 3
     np.testing.assert_array_equal(r["caches"][1][0][:, P + 2], layers[1]["tree_k"][2])
+
+
+# ----------------------------------------------------------------------------
+# rotary re-rotation (rolling-image carryover)
+# ----------------------------------------------------------------------------
+from oracle import rope as R
+
+
+@pytest.mark.parametrize("check", C.ROPE_CHECKS, ids=lambda f: f.__name__)
+def test_rope_pins(check):
+    check(R.carry_keys)
+
+
+def test_rope_block_move_pin():
+    C.check_rope_block_move(R.shift_block, R.carry_keys)
+
+
+def _rope_variant(sign=1.0, interleaved=False, exponent=2.0, skip_inverse=False):
+    def rotate(x, position, base):
+        x = np.asarray(x, dtype=np.float64)
+        D = x.shape[-1]
+        ang = sign * position * base ** (-exponent * np.arange(D // 2) / D)
+        c, s = np.cos(ang), np.sin(ang)
+        if interleaved:
+            x1, x2 = x[..., 0::2], x[..., 1::2]
+            out = np.empty_like(x)
+            out[..., 0::2] = x1 * c - x2 * s
+            out[..., 1::2] = x1 * s + x2 * c
+            return out
+        x1, x2 = x[..., : D // 2], x[..., D // 2:]
+        return np.concatenate([x1 * c - x2 * s, x1 * s + x2 * c], axis=-1)
+
+    def carry(k, m, m_new, base):
+        return rotate(k, m_new, base) if skip_inverse else rotate(rotate(k, -m, base), m_new, base)
+    return carry
+
+
+ROPE_MUTANTS = {
+    "inverse_direction": _rope_variant(sign=-1.0),
+    "interleaved_pairs": _rope_variant(interleaved=True),
+    "wrong_frequency": _rope_variant(exponent=1.0),
+    "no_inverse": _rope_variant(skip_inverse=True),
+}
+
+
+@pytest.mark.parametrize("name", sorted(ROPE_MUTANTS))
+def test_rope_mutants_caught(name):
+    assert _fails_some(C.ROPE_CHECKS, ROPE_MUTANTS[name]) > 0
+
+
+def test_rope_block_mutants_caught():
+    def values_rotated(K, V, src, dst, n, base):
+        K2, V2 = R.shift_block(K, V, src, dst, n, base)
+        for j in range(n):
+            V2[:, dst + j] = R.carry_keys(V[:, src + j], src + j, dst + j, base)
+        return K2, V2
+
+    def reads_after_write(K, V, src, dst, n, base):
+        K2 = np.array(K, dtype=np.float64, copy=True)
+        V2 = np.array(V, dtype=np.float64, copy=True)
+        for j in range(n):  # in-place without staging: overlapping sources get clobbered
+            K2[:, dst + j] = R.carry_keys(K2[:, src + j], src + j, dst + j, base)
+            V2[:, dst + j] = V2[:, src + j]
+        return K2, V2
+    for mut in (values_rotated, reads_after_write):
+        with pytest.raises(AssertionError):
+            C.check_rope_block_move(mut, R.carry_keys)
+
+
+# ----------------------------------------------------------------------------
+# decoding-memory retrieval
+# ----------------------------------------------------------------------------
+from oracle import retrieval as RV
+
+
+@pytest.mark.parametrize("check", C.RETRIEVAL_CHECKS, ids=lambda f: f.__name__)
+def test_retrieval_pins(check):
+    check(RV.cosine_top1)
+
+
+def test_project_key_pins():
+    C.check_project_key(RV.project_key)
+
+
+def _top1_variant(ties_high=False, no_boundary=False, no_token=False, raw_dot=False):
+    def fn(qkey, keys, tok, pos, bound, y, lo=0, hi=None):
+        hi = len(keys) if hi is None else hi
+        q = np.asarray(qkey, dtype=np.float64)
+        best, bestv = -1, None
+        for j in range(lo, hi):
+            if not no_token and int(tok[j]) != int(y):
+                continue
+            if not no_boundary and not int(pos[j]) < int(bound[j]):
+                continue
+            k = np.asarray(keys[j], dtype=np.float64)
+            v = k @ q if raw_dot else (k @ q) / (np.linalg.norm(k) * np.linalg.norm(q))
+            if best < 0 or v > bestv or (ties_high and v == bestv):
+                best, bestv = j, v
+        if best < 0:
+            return -1, float("nan")
+        k = np.asarray(keys[best], dtype=np.float64)
+        return best, float((k @ q) / (np.linalg.norm(k) * np.linalg.norm(q)))
+    return fn
+
+
+RETRIEVAL_MUTANTS = {
+    "ties_to_highest": _top1_variant(ties_high=True),
+    "ignores_boundary": _top1_variant(no_boundary=True),
+    "ignores_token": _top1_variant(no_token=True),
+    "raw_dot_product": _top1_variant(raw_dot=True),
+}
+
+
+@pytest.mark.parametrize("name", sorted(RETRIEVAL_MUTANTS))
+def test_retrieval_mutants_caught(name):
+    assert _fails_some(C.RETRIEVAL_CHECKS, RETRIEVAL_MUTANTS[name]) > 0
+
+
+def test_project_key_mutants_caught():
+    def round_half_up(h, proj):
+        key, x = RV.project_key(h, proj)
+        return np.floor(x + 0.5).astype(np.int8), x
+
+    def no_normalise(h, proj):
+        z = np.asarray(proj, dtype=np.float64) @ np.asarray(h, dtype=np.float64)
+        x = np.clip(z, -127, 127)
+        return np.rint(x).astype(np.int8), x
+    for mut in (round_half_up, no_normalise):
+        with pytest.raises(AssertionError):
+            C.check_project_key(mut)

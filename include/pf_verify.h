@@ -273,6 +273,96 @@ typedef struct pf_commit_desc {
 
 PF_API pf_status pf_kv_commit(const pf_commit_desc* d, void* stream);
 
+/*
+ * pf_kv_shift -- rolling-image KV carryover (Section 3.4): when the window
+ * of retained screenshots advances, a retained visual-token block moves to
+ * a new span of the prompt.  For every layer and KV head of sequence `seq`:
+ *   K[dst + j] = R(dst + j) R(src + j)^-1 K[src + j]   (rotary re-rotation)
+ *   V[dst + j] = V[src + j]                             j = 0 .. count-1
+ * R is the rotary embedding in the rotate-half layout: the pair
+ * (x_i, x_{i+D/2}) turns by position * rope_base^(-2i/D); for multi-axis
+ * rotary embeddings every axis moves by the same shift, so the same
+ * rotation applies.  The move is in place: source and destination spans may
+ * overlap (rows are staged in the right order), and rows of the source span
+ * outside the destination keep their contents.  The rotation angles are
+ * formed on the host in double precision.  Layout as pf_kv_view (layer l at
+ * cache.k/v + l * cache_layer_stride elements); D even, D * element size a
+ * multiple of 16.  The host checks both spans fit the cache; the kernel
+ * flags PF_DEVERR_CAPACITY for a page-table entry outside the pool.
+ */
+typedef struct pf_shift_desc {
+  int32_t dtype;               /* pf_dtype                                   */
+  int32_t n_layers;            /* L                                          */
+  int32_t n_kv_heads;          /* Hkv                                        */
+  int32_t head_dim;            /* D                                          */
+  int32_t seq;                 /* sequence of the cache to move within       */
+  int32_t batch;               /* sequences (page-table rows when paged)     */
+  int32_t src;                 /* first source position                      */
+  int32_t dst;                 /* first destination position                 */
+  int32_t count;               /* rows to move (>= 0)                        */
+  float rope_base;             /* rotary base, e.g. 10000 or 1e6             */
+  pf_kv_view cache;            /* layer 0's view                             */
+  int64_t cache_layer_stride;  /* elements between layers                    */
+  int32_t* error_flag;         /* optional device int32                      */
+} pf_shift_desc;
+
+PF_API pf_status pf_kv_shift(const pf_shift_desc* d, void* stream);
+
+/*
+ * pf_retrieval_key -- the int8 retrieval key of a final-layer state
+ * (Section 4 "Memory and retrieval": normalised final-layer states mapped
+ * to 256-dimensional int8 keys by a fixed random projection).
+ *   z = P h / |h|,  key = round_half_even(127 * z / max_i |z_i|)
+ * (the per-vector scale keeps every key at full int8 range; cosine
+ * similarity is scale invariant).  hidden_state [H] and projection [256][H]
+ * in dtype; key_out [256] int8.  Workspace: pf_retrieval_workspace_size()
+ * bytes, zero-filled before first use and left zero-filled.
+ */
+typedef struct pf_key_desc {
+  int32_t dtype;               /* pf_dtype of hidden_state and projection    */
+  int32_t hidden;              /* H                                          */
+  const void* hidden_state;    /* device [H]                                 */
+  const void* projection;      /* device [256][H]                            */
+  int8_t* key_out;             /* out device [256]                           */
+  int32_t* error_flag;         /* optional device int32                      */
+} pf_key_desc;
+
+#define PF_KEY_DIM 256
+
+/*
+ * pf_retrieve -- context-compatible retrieval (Section 3.2): among the
+ * stored entries j in [lo, hi) whose token equals `token` and whose
+ * position is before its output boundary (entry_pos[j] < entry_bound[j]),
+ * the entry whose int8 key has the highest cosine similarity with
+ * query_key.  The comparison is exact (integer dot products and squared
+ * norms compared in 128-bit arithmetic); ties go to the lowest index;
+ * all-zero keys are never selected.  Outputs: best[0] = index or -1,
+ * similarity[0] = its cosine (fp32).  keys [n_entries][256] int8;
+ * entry_token, entry_pos, entry_bound [n_entries] int32.  Workspace:
+ * pf_retrieval_workspace_size() bytes, zero-filled before first use and
+ * left zero-filled; calls sharing a workspace must not overlap.
+ */
+typedef struct pf_retrieval_desc {
+  int32_t n_entries;           /* M                                          */
+  int32_t lo;                  /* first entry scanned                        */
+  int32_t hi;                  /* one past the last entry scanned            */
+  int32_t token;               /* the query's current token                  */
+  const int8_t* query_key;     /* device [256]                               */
+  const int8_t* keys;          /* device [M][256]                            */
+  const int32_t* entry_token;  /* device [M]                                 */
+  const int32_t* entry_pos;    /* device [M]                                 */
+  const int32_t* entry_bound;  /* device [M]                                 */
+  int32_t* best;               /* out device [1]                             */
+  float* similarity;           /* out device [1]                             */
+  int32_t* error_flag;         /* optional device int32                      */
+} pf_retrieval_desc;
+
+PF_API size_t pf_retrieval_workspace_size(void);
+PF_API pf_status pf_retrieval_key(const pf_key_desc* d, void* workspace, size_t workspace_bytes,
+                                  void* stream);
+PF_API pf_status pf_retrieve(const pf_retrieval_desc* d, void* workspace, size_t workspace_bytes,
+                             void* stream);
+
 #ifdef __cplusplus
 }
 #endif

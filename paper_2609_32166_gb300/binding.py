@@ -83,6 +83,28 @@ class pf_commit_desc(C.Structure):
                 ("error_flag", C.c_void_p)]
 
 
+class pf_shift_desc(C.Structure):
+    _fields_ = [("dtype", C.c_int32), ("n_layers", C.c_int32), ("n_kv_heads", C.c_int32),
+                ("head_dim", C.c_int32), ("seq", C.c_int32), ("batch", C.c_int32),
+                ("src", C.c_int32), ("dst", C.c_int32), ("count", C.c_int32),
+                ("rope_base", C.c_float), ("cache", pf_kv_view),
+                ("cache_layer_stride", C.c_int64), ("error_flag", C.c_void_p)]
+
+
+class pf_key_desc(C.Structure):
+    _fields_ = [("dtype", C.c_int32), ("hidden", C.c_int32), ("hidden_state", C.c_void_p),
+                ("projection", C.c_void_p), ("key_out", C.c_void_p),
+                ("error_flag", C.c_void_p)]
+
+
+class pf_retrieval_desc(C.Structure):
+    _fields_ = [("n_entries", C.c_int32), ("lo", C.c_int32), ("hi", C.c_int32),
+                ("token", C.c_int32), ("query_key", C.c_void_p), ("keys", C.c_void_p),
+                ("entry_token", C.c_void_p), ("entry_pos", C.c_void_p),
+                ("entry_bound", C.c_void_p), ("best", C.c_void_p),
+                ("similarity", C.c_void_p), ("error_flag", C.c_void_p)]
+
+
 _lib = None
 
 
@@ -113,6 +135,15 @@ def lib() -> C.CDLL:
     L.pf_lmhead_accept_noalloc.argtypes = [C.POINTER(pf_lm_desc), C.c_void_p]
     L.pf_kv_commit.restype = C.c_int
     L.pf_kv_commit.argtypes = [C.POINTER(pf_commit_desc), C.c_void_p]
+    L.pf_kv_shift.restype = C.c_int
+    L.pf_kv_shift.argtypes = [C.POINTER(pf_shift_desc), C.c_void_p]
+    L.pf_retrieval_workspace_size.restype = C.c_size_t
+    L.pf_retrieval_workspace_size.argtypes = []
+    L.pf_retrieval_key.restype = C.c_int
+    L.pf_retrieval_key.argtypes = [C.POINTER(pf_key_desc), C.c_void_p, C.c_size_t, C.c_void_p]
+    L.pf_retrieve.restype = C.c_int
+    L.pf_retrieve.argtypes = [C.POINTER(pf_retrieval_desc), C.c_void_p, C.c_size_t,
+                              C.c_void_p]
     _lib = L
     return L
 
@@ -168,3 +199,23 @@ def pf_lmhead_accept_noalloc(desc: pf_lm_desc, stream: int = 0) -> None:
 
 def pf_kv_commit(desc: pf_commit_desc, stream: int = 0) -> None:
     _check(lib().pf_kv_commit(C.byref(desc), C.c_void_p(stream)))
+
+
+def pf_kv_shift(desc: pf_shift_desc, stream: int = 0) -> None:
+    _check(lib().pf_kv_shift(C.byref(desc), C.c_void_p(stream)))
+
+
+def pf_retrieval_workspace_size() -> int:
+    return int(lib().pf_retrieval_workspace_size())
+
+
+def pf_retrieval_key(desc: pf_key_desc, workspace: int, workspace_bytes: int,
+                     stream: int = 0) -> None:
+    _check(lib().pf_retrieval_key(C.byref(desc), C.c_void_p(workspace),
+                                  C.c_size_t(workspace_bytes), C.c_void_p(stream)))
+
+
+def pf_retrieve(desc: pf_retrieval_desc, workspace: int, workspace_bytes: int,
+                stream: int = 0) -> None:
+    _check(lib().pf_retrieve(C.byref(desc), C.c_void_p(workspace),
+                             C.c_size_t(workspace_bytes), C.c_void_p(stream)))

@@ -484,4 +484,119 @@ pf_status pf_kv_commit(const pf_commit_desc* d, void* stream) {
   return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
 }
 
+pf_status pf_kv_shift(const pf_shift_desc* d, void* stream) {
+  static const char* who = "pf_kv_shift";
+  if (!d) return fail(PF_ERR_NULL, "%s: desc is NULL", who);
+  if (d->dtype != PF_BF16 && d->dtype != PF_F32)
+    return fail(PF_ERR_DTYPE, "%s: dtype %d unsupported", who, d->dtype);
+  if (d->n_layers < 1 || d->n_kv_heads < 1)
+    return fail(PF_ERR_SHAPE, "%s: n_layers and n_kv_heads must be >= 1", who);
+  const int es = elem_size(d->dtype);
+  const int D = d->head_dim;
+  if (D < 2 || D % 2 || D > 256 || ((D / 2) * es) % 16)
+    return fail(PF_ERR_SHAPE, "%s: head_dim must be even, <= 256, half a row a multiple of 16 B",
+                who);
+  if (d->count < 0 || d->src < 0 || d->dst < 0)
+    return fail(PF_ERR_SHAPE, "%s: src, dst and count must be >= 0", who);
+  if (!(d->rope_base > 0.f)) return fail(PF_ERR_SHAPE, "%s: rope_base must be > 0", who);
+  if ((long long)d->n_layers * d->n_kv_heads > 65535)
+    return fail(PF_ERR_SHAPE, "%s: n_layers * n_kv_heads must be <= 65535", who);
+  if (d->seq < 0 || d->seq >= d->batch)
+    return fail(PF_ERR_SHAPE, "%s: seq outside 0..batch-1", who);
+  pf_status st = check_cache_view(d->cache, std::max(d->src, d->dst) + d->count, who);
+  if (st != PF_OK) return st;
+  if (d->n_layers > 1 && (d->cache_layer_stride * es) % 16 != 0)
+    return fail(PF_ERR_ALIGN, "%s: layer stride must be a multiple of 16 bytes", who);
+  if (d->count == 0 || d->src == d->dst) return PF_OK;  // nothing moves, nothing turns
+
+  pf::ShiftArgs a = {};
+  a.L = d->n_layers;
+  a.Hkv = d->n_kv_heads;
+  a.row_bytes = D * es;
+  a.elem_bytes = es;
+  a.seq = d->seq;
+  a.src = d->src;
+  a.dst = d->dst;
+  a.count = d->count;
+  a.layout = d->cache.layout;
+  a.max_seq = d->cache.max_seq;
+  a.pages_per_seq = d->cache.pages_per_seq;
+  a.num_pages = d->cache.num_pages;
+  a.page_table = d->cache.page_table;
+  a.cache_k = static_cast<char*>(d->cache.k);
+  a.cache_v = static_cast<char*>(d->cache.v);
+  a.layer_bytes = d->cache_layer_stride * es;
+  a.err = d->error_flag;
+  const double shift = (double)d->dst - (double)d->src;
+  for (int i = 0; i < D / 2; ++i) {
+    const double ang = shift * std::pow((double)d->rope_base, -2.0 * i / D);
+    a.cs[i] = make_float2((float)std::cos(ang), (float)std::sin(ang));
+  }
+  if (num_sms() <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
+  cudaError_t e = pf::launch_kv_shift(a, static_cast<cudaStream_t>(stream), pdl_enabled());
+  return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
+}
+
+size_t pf_retrieval_workspace_size(void) { return pf::kRetrievalWsBytes; }
+
+pf_status pf_retrieval_key(const pf_key_desc* d, void* workspace, size_t workspace_bytes,
+                           void* stream) {
+  static const char* who = "pf_retrieval_key";
+  if (!d) return fail(PF_ERR_NULL, "%s: desc is NULL", who);
+  if (!d->hidden_state || !d->projection || !d->key_out)
+    return fail(PF_ERR_NULL, "%s: a required pointer is NULL", who);
+  if (!workspace || workspace_bytes < pf::kRetrievalWsBytes)
+    return fail(PF_ERR_WORKSPACE, "%s: workspace needs %zu bytes", who, pf::kRetrievalWsBytes);
+  if (!aligned16(workspace)) return fail(PF_ERR_ALIGN, "%s: workspace must be 16-byte aligned", who);
+  if (d->dtype != PF_BF16 && d->dtype != PF_F32)
+    return fail(PF_ERR_DTYPE, "%s: dtype %d unsupported", who, d->dtype);
+  if (d->hidden < 1) return fail(PF_ERR_SHAPE, "%s: hidden must be >= 1", who);
+  pf::KeyArgs a = {};
+  a.H = d->hidden;
+  a.bf16 = d->dtype == PF_BF16;
+  a.hidden = d->hidden_state;
+  a.proj = d->projection;
+  a.key_out = d->key_out;
+  a.z = reinterpret_cast<float*>(static_cast<char*>(workspace) + pf::kRetrievalZOff);
+  a.ticket = reinterpret_cast<unsigned*>(static_cast<char*>(workspace) + pf::kRetrievalKeyTicketOff);
+  a.err = d->error_flag;
+  if (num_sms() <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
+  cudaError_t e = pf::launch_retrieval_key(a, static_cast<cudaStream_t>(stream), pdl_enabled());
+  return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
+}
+
+pf_status pf_retrieve(const pf_retrieval_desc* d, void* workspace, size_t workspace_bytes,
+                      void* stream) {
+  static const char* who = "pf_retrieve";
+  if (!d) return fail(PF_ERR_NULL, "%s: desc is NULL", who);
+  if (!d->query_key || !d->keys || !d->entry_token || !d->entry_pos || !d->entry_bound ||
+      !d->best || !d->similarity)
+    return fail(PF_ERR_NULL, "%s: a required pointer is NULL", who);
+  if (!workspace || workspace_bytes < pf::kRetrievalWsBytes)
+    return fail(PF_ERR_WORKSPACE, "%s: workspace needs %zu bytes", who, pf::kRetrievalWsBytes);
+  if (d->n_entries < 0 || d->lo < 0 || d->lo > d->hi || d->hi > d->n_entries)
+    return fail(PF_ERR_SHAPE, "%s: need 0 <= lo <= hi <= n_entries", who);
+  if (!aligned16(d->keys) || !aligned16(d->query_key) || !aligned16(workspace))
+    return fail(PF_ERR_ALIGN, "%s: keys, query_key and workspace must be 16-byte aligned", who);
+  pf::RetrievalArgs a = {};
+  a.lo = d->lo;
+  a.hi = d->hi;
+  a.token = d->token;
+  a.query_key = d->query_key;
+  a.keys = d->keys;
+  a.entry_token = d->entry_token;
+  a.entry_pos = d->entry_pos;
+  a.entry_bound = d->entry_bound;
+  a.best = d->best;
+  a.similarity = d->similarity;
+  a.block_best = reinterpret_cast<int4*>(static_cast<char*>(workspace) + pf::kRetrievalBestOff);
+  a.ticket =
+      reinterpret_cast<unsigned*>(static_cast<char*>(workspace) + pf::kRetrievalScanTicketOff);
+  a.err = d->error_flag;
+  const int sms = num_sms();
+  if (sms <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
+  cudaError_t e = pf::launch_retrieve(a, static_cast<cudaStream_t>(stream), sms, pdl_enabled());
+  return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
+}
+
 }  // extern "C"

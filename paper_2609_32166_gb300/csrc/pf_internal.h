@@ -5,6 +5,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <algorithm>
 #include <utility>
 
 #include "pf_verify.h"
@@ -113,6 +114,60 @@ struct CommitArgs {
 };
 
 cudaError_t launch_kv_commit(const CommitArgs& a, cudaStream_t s, int num_sms, bool pdl);
+
+// ------------------------------------------------------------ KV shift
+struct ShiftArgs {
+  int L, Hkv, row_bytes, elem_bytes;
+  int seq, src, dst, count;
+  int overlap;     // spans overlap: one CTA per (layer, head) walks every pass
+  int descending;  // move to higher positions: passes run from the end
+  int layout, max_seq, pages_per_seq, num_pages;
+  const int32_t* page_table;
+  char* cache_k;
+  char* cache_v;
+  long long layer_bytes;
+  int32_t* err;
+  float2 cs[128];  // cos / sin of shift * theta_i, i < D/2 (host, double precision)
+};
+
+cudaError_t launch_kv_shift(const ShiftArgs& a, cudaStream_t s, bool pdl);
+
+// ------------------------------------------------------------ retrieval
+constexpr int kRetrievalMaxBlocks = 1024;
+// workspace: [0, 1024) z floats | [1024, 1040) key ticket |
+// [1088, 1088 + 16 * kRetrievalMaxBlocks) per-CTA winners | then scan ticket
+constexpr size_t kRetrievalZOff = 0;
+constexpr size_t kRetrievalKeyTicketOff = 1024;
+constexpr size_t kRetrievalBestOff = 1088;
+constexpr size_t kRetrievalScanTicketOff = kRetrievalBestOff + 16 * kRetrievalMaxBlocks;
+constexpr size_t kRetrievalWsBytes = kRetrievalScanTicketOff + 64;
+
+struct KeyArgs {
+  int H, bf16;
+  const void* hidden;
+  const void* proj;
+  int8_t* key_out;
+  float* z;
+  unsigned int* ticket;
+  int32_t* err;
+};
+
+struct RetrievalArgs {
+  int lo, hi, token;
+  const int8_t* query_key;
+  const int8_t* keys;
+  const int32_t* entry_token;
+  const int32_t* entry_pos;
+  const int32_t* entry_bound;
+  int32_t* best;
+  float* similarity;
+  int4* block_best;
+  unsigned int* ticket;
+  int32_t* err;
+};
+
+cudaError_t launch_retrieval_key(const KeyArgs& a, cudaStream_t s, bool pdl);
+cudaError_t launch_retrieve(const RetrievalArgs& a, cudaStream_t s, int num_sms, bool pdl);
 
 // Record the message pf_last_error() returns on this thread; returns s.
 pf_status set_error(pf_status s, const char* fmt, ...);

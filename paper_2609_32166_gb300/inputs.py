@@ -348,3 +348,54 @@ def cache_rows(w: Workload, batch: Batch, cache: np.ndarray, seq: int,
         pos = start + i
         out[:, i, :] = cache[pt[pos // PAGE_SIZE], :, pos % PAGE_SIZE, :]
     return out
+
+
+# ----------------------------------------------------------------------------
+# rolling-image carryover and decoding-memory inputs
+# ----------------------------------------------------------------------------
+KEY_DIM = 256
+QWEN_VOCAB = 151936
+
+
+def page_table(n_seqs: int, pages_per_seq: int, seed: int, spare: int = 3):
+    """A random permutation of n_seqs * pages_per_seq + spare pages laid out
+    as page_table [n_seqs, pages_per_seq]; returns (table int32, num_pages)."""
+    num_pages = n_seqs * pages_per_seq + spare
+    perm = _stream(seed, "page_table").permutation(num_pages).astype(np.int32)
+    return perm[: n_seqs * pages_per_seq].reshape(n_seqs, pages_per_seq), num_pages
+
+
+def int8_keys(n: int, seed: int, tag: str = "memory_keys", index: int = 0) -> np.ndarray:
+    """[n, 256] int8: N(0, 40^2) rounded and clipped to [-127, 127] (the spread
+    of keys that use most of the int8 range)."""
+    rng = _stream(seed, tag, index)
+    x = rng.normal(0.0, 40.0, size=(n, KEY_DIM))
+    return np.clip(np.rint(x), -127, 127).astype(np.int8)
+
+
+@dataclasses.dataclass
+class Memory:
+    keys: np.ndarray    # [M, 256] int8
+    token: np.ndarray   # [M] int32, token of the shared array at the entry's position
+    pos: np.ndarray     # [M] int32, position of the entry in the shared token array
+    bound: np.ndarray   # [M] int32, last position of the entry's output sequence
+
+
+def decoding_memory(n_entries: int, seed: int, vocab: int = QWEN_VOCAB,
+                    mean_len: int = 80) -> Memory:
+    """A decoding-experience memory of n_entries: output sequences of
+    U[16, 2 * mean_len - 16] tokens appended to one shared token array, one
+    entry per position (the last position of each sequence is its boundary).
+    Tokens follow a Zipf(1.2) law over the vocabulary, so a query's token
+    matches anywhere from a handful to a few percent of the entries."""
+    rng = _stream(seed, "memory_layout")
+    bound = np.empty(n_entries, dtype=np.int32)
+    p = 0
+    while p < n_entries:
+        n = int(rng.integers(16, max(17, 2 * mean_len - 15)))
+        e = min(n_entries, p + n)
+        bound[p:e] = p + n - 1
+        p = e
+    token = ((rng.zipf(1.2, size=n_entries) - 1) % vocab).astype(np.int32)
+    pos = np.arange(n_entries, dtype=np.int32)
+    return Memory(int8_keys(n_entries, seed), token, pos, bound)

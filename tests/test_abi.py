@@ -21,7 +21,8 @@ def test_exports_every_declared_symbol():
     names = pb.header_functions()
     assert set(names) >= {"pf_tree_prepare", "pf_verify_attention", "pf_lmhead_accept",
                           "pf_lmhead_accept_workspace_size", "pf_kv_commit", "pf_last_error",
-                          "pf_version"}
+                          "pf_version", "pf_kv_shift", "pf_retrieval_key", "pf_retrieve",
+                          "pf_retrieval_workspace_size", "pf_lmhead_accept_noalloc"}
     L = pb.lib()
     for n in names:
         assert hasattr(L, n), n
@@ -41,6 +42,10 @@ int main(void) {
   printf("%zu %zu %zu %zu %zu %zu %zu\n", sizeof(pf_kv_view), sizeof(pf_attn_desc),
          sizeof(pf_lm_desc), sizeof(pf_commit_desc), offsetof(pf_attn_desc, cache),
          offsetof(pf_commit_desc, cache), offsetof(pf_commit_desc, new_len));
+  printf("%zu %zu %zu %zu %zu %zu %zu\n", sizeof(pf_shift_desc), offsetof(pf_shift_desc, cache),
+         offsetof(pf_shift_desc, cache_layer_stride), sizeof(pf_key_desc),
+         offsetof(pf_key_desc, key_out), sizeof(pf_retrieval_desc),
+         offsetof(pf_retrieval_desc, similarity));
   return 0;
 }
 '''
@@ -53,7 +58,11 @@ int main(void) {
                                               check=True).stdout.split()]
     want = [C.sizeof(pb.pf_kv_view), C.sizeof(pb.pf_attn_desc), C.sizeof(pb.pf_lm_desc),
             C.sizeof(pb.pf_commit_desc), pb.pf_attn_desc.cache.offset,
-            pb.pf_commit_desc.cache.offset, pb.pf_commit_desc.new_len.offset]
+            pb.pf_commit_desc.cache.offset, pb.pf_commit_desc.new_len.offset,
+            C.sizeof(pb.pf_shift_desc), pb.pf_shift_desc.cache.offset,
+            pb.pf_shift_desc.cache_layer_stride.offset, C.sizeof(pb.pf_key_desc),
+            pb.pf_key_desc.key_out.offset, C.sizeof(pb.pf_retrieval_desc),
+            pb.pf_retrieval_desc.similarity.offset]
     assert got == want
 
 
@@ -183,3 +192,87 @@ def test_commit_rejects_bad_arguments(kw, status):
     with pytest.raises(pb.PfError) as e:
         pb.pf_kv_commit(_commit_desc(**kw), 0)
     assert e.value.status == status
+
+
+def _shift_desc(**kw):
+    d = pb.pf_shift_desc()
+    d.dtype, d.n_layers, d.n_kv_heads, d.head_dim = pb.PF_BF16, 2, 2, 128
+    d.seq, d.batch, d.src, d.dst, d.count, d.rope_base = 0, 1, 10, 4, 20, 1e4
+    fake = 0x10000
+    d.cache_layer_stride = 2 * 64 * 128
+    d.cache.layout, d.cache.k, d.cache.v, d.cache.max_seq = pb.PF_KV_CONTIGUOUS, fake, fake, 64
+    for k, v in kw.items():
+        if k.startswith("cache_") and k != "cache_layer_stride":
+            setattr(d.cache, k[6:], v)
+        else:
+            setattr(d, k, v)
+    return d
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(cache_k=None), pb.PF_ERR_NULL),
+    (dict(dtype=5), pb.PF_ERR_DTYPE),
+    (dict(head_dim=130), pb.PF_ERR_SHAPE),
+    (dict(head_dim=8), pb.PF_ERR_SHAPE),          # half a bf16 row below 16 bytes
+    (dict(head_dim=512), pb.PF_ERR_SHAPE),
+    (dict(count=-1), pb.PF_ERR_SHAPE),
+    (dict(src=-3), pb.PF_ERR_SHAPE),
+    (dict(rope_base=0.0), pb.PF_ERR_SHAPE),
+    (dict(seq=1), pb.PF_ERR_SHAPE),
+    (dict(n_layers=0), pb.PF_ERR_SHAPE),
+    (dict(dst=50), pb.PF_ERR_CAPACITY),           # 50 + 20 rows > max_seq 64
+    (dict(cache_layout=1, cache_page_table=0x10000, cache_num_pages=8, cache_pages_per_seq=1),
+     pb.PF_ERR_CAPACITY),
+    (dict(cache_layer_stride=3), pb.PF_ERR_ALIGN),
+])
+def test_kv_shift_rejects_bad_arguments(kw, status):
+    with pytest.raises(pb.PfError) as e:
+        pb.pf_kv_shift(_shift_desc(**kw), 0)
+    assert e.value.status == status
+
+
+def test_kv_shift_nothing_to_move_is_ok_without_gpu():
+    """count = 0 and src = dst move nothing and launch nothing."""
+    pb.pf_kv_shift(_shift_desc(count=0), 0)
+    pb.pf_kv_shift(_shift_desc(dst=10), 0)
+
+
+def _key_desc(**kw):
+    d = pb.pf_key_desc()
+    d.dtype, d.hidden = pb.PF_BF16, 64
+    d.hidden_state, d.projection, d.key_out = 0x10000, 0x10000, 0x10000
+    for k, v in kw.items():
+        setattr(d, k, v)
+    return d
+
+
+def _retrieval_desc(**kw):
+    d = pb.pf_retrieval_desc()
+    d.n_entries, d.lo, d.hi, d.token = 100, 0, 100, 7
+    for f in ("query_key", "keys", "entry_token", "entry_pos", "entry_bound", "best",
+              "similarity"):
+        setattr(d, f, 0x10000)
+    for k, v in kw.items():
+        setattr(d, k, v)
+    return d
+
+
+def test_retrieval_rejects_bad_arguments():
+    ws = pb.pf_retrieval_workspace_size()
+    assert ws >= 1024 + 16 * 1024
+    cases = [
+        (lambda: pb.pf_retrieval_key(_key_desc(projection=None), 0x20000, ws), pb.PF_ERR_NULL),
+        (lambda: pb.pf_retrieval_key(_key_desc(), 0x20000, ws - 1), pb.PF_ERR_WORKSPACE),
+        (lambda: pb.pf_retrieval_key(_key_desc(dtype=4), 0x20000, ws), pb.PF_ERR_DTYPE),
+        (lambda: pb.pf_retrieval_key(_key_desc(hidden=0), 0x20000, ws), pb.PF_ERR_SHAPE),
+        (lambda: pb.pf_retrieval_key(_key_desc(), 0x20008, ws), pb.PF_ERR_ALIGN),
+        (lambda: pb.pf_retrieve(_retrieval_desc(best=None), 0x20000, ws), pb.PF_ERR_NULL),
+        (lambda: pb.pf_retrieve(_retrieval_desc(), 0, ws), pb.PF_ERR_WORKSPACE),
+        (lambda: pb.pf_retrieve(_retrieval_desc(hi=101), 0x20000, ws), pb.PF_ERR_SHAPE),
+        (lambda: pb.pf_retrieve(_retrieval_desc(lo=60, hi=50), 0x20000, ws), pb.PF_ERR_SHAPE),
+        (lambda: pb.pf_retrieve(_retrieval_desc(keys=0x10004), 0x20000, ws), pb.PF_ERR_ALIGN),
+    ]
+    for call, status in cases:
+        with pytest.raises(pb.PfError) as e:
+            call()
+        assert e.value.status == status, pb.pf_last_error()

@@ -48,6 +48,8 @@ def parse():
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-next-rows", action="store_true",
+                   help="skip the key re-rotation and retrieval measurements")
     p.add_argument("--cpu-worker", default=None, help=argparse.SUPPRESS)
     return p.parse_args()
 
@@ -483,6 +485,7 @@ def main():
         if world > 1:
             dist.destroy_process_group()
         return
+    next_rows = None if args.no_next_rows else measure_next_rows(stream, flush, hbm_peak)
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
@@ -510,6 +513,7 @@ def main():
                    if graph_events else "one CUDA graph per part, events between graph launches"),
         "clocks": clk,
         "e2e": e2e,
+        "next_rows": next_rows,
     }
     if cpu_base is not None:
         line["cpu_baseline"] = {"value": cpu_base["tokens_per_step"] / cpu_base["step_s"],
@@ -519,6 +523,135 @@ def main():
     print(json.dumps(line))
     if world > 1:
         dist.destroy_process_group()
+
+
+def _time_events(stream, flush, fn, iters, warmup=3):
+    """Mean device time (ms) of fn(i) over iters calls, L2 flushed before each
+    call outside the events.  The calls are captured in one CUDA graph with
+    event nodes (so host launch overhead stays out of the numbers) when this
+    torch supports graph events, else launched eagerly."""
+    import torch
+    with torch.cuda.stream(stream):
+        for i in range(warmup):
+            flush.zero_()
+            fn(i)
+    stream.synchronize()
+    try:
+        ev = [(torch.cuda.Event(enable_timing=True, external=True),
+               torch.cuda.Event(enable_timing=True, external=True)) for _ in range(iters)]
+    except TypeError:
+        ev = None
+    if ev is not None:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            s = torch.cuda.current_stream()
+            for i in range(iters):
+                flush.zero_()
+                ev[i][0].record(s)
+                fn(warmup + i)
+                ev[i][1].record(s)
+        with torch.cuda.stream(stream):
+            g.replay()   # untimed: uploads the graph
+            stream.synchronize()
+            g.replay()
+        stream.synchronize()
+    else:
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(iters)]
+        with torch.cuda.stream(stream):
+            for i in range(iters):
+                flush.zero_()
+                ev[i][0].record(stream)
+                fn(warmup + i)
+                ev[i][1].record(stream)
+        stream.synchronize()
+    return float(np.mean([a.elapsed_time(b) for a, b in ev]))
+
+
+def measure_next_rows(stream, flush, hbm_peak):
+    """Rolling-image key re-rotation and decoding-memory retrieval, each on a
+    workload of the paper's shape, timed with CUDA events on the launching
+    stream (L2 flushed between calls)."""
+    import torch
+    from paper_2609_32166_gb300 import binding as pb
+    from paper_2609_32166_gb300 import inputs as I
+    out = {}
+    sp = stream.cuda_stream
+    # --- pf_kv_shift: two retained 1300-token screenshots move down by one
+    # screenshot in every layer of a 7B-VLM-shaped cache, and back again
+    L, Hkv, D, S = 28, 4, 128, 4096
+    src, dst, count = 1400, 100, 2600
+    k = torch.empty((L, 1, Hkv, S, D), dtype=torch.bfloat16, device="cuda").normal_()
+    v = torch.empty_like(k).normal_()
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    descs = []
+    for a, b in ((src, dst), (dst, src)):
+        d = pb.pf_shift_desc()
+        d.dtype, d.n_layers, d.n_kv_heads, d.head_dim = pb.PF_BF16, L, Hkv, D
+        d.seq, d.batch, d.src, d.dst, d.count, d.rope_base = 0, 1, a, b, count, 1e6
+        d.cache.layout, d.cache.k, d.cache.v, d.cache.max_seq = (pb.PF_KV_CONTIGUOUS,
+                                                                 k.data_ptr(), v.data_ptr(), S)
+        d.cache_layer_stride = Hkv * S * D
+        d.error_flag = err.data_ptr()
+        descs.append(d)
+    ms = _time_events(stream, flush, lambda i: pb.pf_kv_shift(descs[i % 2], sp), 30)
+    assert int(err.item()) == 0
+    shift_bytes = count * L * Hkv * D * 2 * 2 * 2   # K and V rows, read once and written once
+    gbs = shift_bytes / (ms * 1e-3) / 1e9
+    out["kv_shift"] = {
+        "workload": "28 layers x 4 KV heads x D=128 bf16; 2600 rows shifted by 1300 "
+                    "(two 1300-token screenshots), rope base 1e6",
+        "us": ms * 1e3, "algorithmic_bytes": shift_bytes, "achieved_gbs": gbs,
+        "peak_gbs": hbm_peak, "frac": gbs / hbm_peak, "launches": 2}
+    del k, v
+    # --- pf_retrieval_key + pf_retrieve over a 290K-entry memory (74 MiB at
+    # 256 + 12 bytes per entry)
+    M, H = 290000, 3584
+    mem = I.decoding_memory(M, seed=11)
+    keys = torch.from_numpy(mem.keys).cuda()
+    etok = torch.from_numpy(mem.token).cuda()
+    epos = torch.from_numpy(mem.pos).cuda()
+    ebnd = torch.from_numpy(mem.bound).cuda()
+    h = torch.empty(H, dtype=torch.bfloat16, device="cuda").normal_()
+    P = torch.empty((I.KEY_DIM, H), dtype=torch.bfloat16, device="cuda").normal_()
+    qkey = torch.zeros(I.KEY_DIM, dtype=torch.int8, device="cuda")
+    best = torch.zeros(1, dtype=torch.int32, device="cuda")
+    sim = torch.zeros(1, dtype=torch.float32, device="cuda")
+    nws = pb.pf_retrieval_workspace_size()
+    ws = torch.zeros(nws, dtype=torch.uint8, device="cuda")
+    kd = pb.pf_key_desc()
+    kd.dtype, kd.hidden, kd.hidden_state, kd.projection = pb.PF_BF16, H, h.data_ptr(), P.data_ptr()
+    kd.key_out, kd.error_flag = qkey.data_ptr(), err.data_ptr()
+    tokens, counts = np.unique(mem.token, return_counts=True)
+    elig = (mem.pos < mem.bound)
+    res = {}
+    for label, tok in (("most frequent token", int(tokens[np.argmax(counts)])),
+                       ("token of a random entry", int(mem.token[M // 3]))):
+        rd = pb.pf_retrieval_desc()
+        rd.n_entries, rd.lo, rd.hi, rd.token = M, 0, M, tok
+        rd.query_key, rd.keys = qkey.data_ptr(), keys.data_ptr()
+        rd.entry_token, rd.entry_pos, rd.entry_bound = (etok.data_ptr(), epos.data_ptr(),
+                                                        ebnd.data_ptr())
+        rd.best, rd.similarity, rd.error_flag = best.data_ptr(), sim.data_ptr(), err.data_ptr()
+
+        def lookup(i, rd=rd):
+            pb.pf_retrieval_key(kd, ws.data_ptr(), nws, sp)
+            pb.pf_retrieve(rd, ws.data_ptr(), nws, sp)
+
+        ms_l = _time_events(stream, flush, lookup, 50)
+        ms_s = _time_events(stream, flush, lambda i, rd=rd: pb.pf_retrieve(rd, ws.data_ptr(),
+                                                                          nws, sp), 50)
+        n_elig = int(np.sum((mem.token == tok) & elig))
+        # token, position and boundary of every entry, the key of every eligible one
+        scan_bytes = 12 * M + I.KEY_DIM * n_elig
+        res[label] = {"eligible": n_elig, "us_lookup": ms_l * 1e3, "us_scan": ms_s * 1e3,
+                      "scan_algorithmic_bytes": scan_bytes,
+                      "scan_gbs": scan_bytes / (ms_s * 1e-3) / 1e9}
+    assert int(err.item()) == 0
+    out["retrieval"] = {
+        "workload": f"{M} entries (int8 256-d keys, Zipf(1.2) tokens), H={H} bf16 query state",
+        "lookup": "pf_retrieval_key + pf_retrieve", "queries": res}
+    return out
 
 
 def run_e2e(vs, w, batch, K, stream, flush, world, tok_table, planned):

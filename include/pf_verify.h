@@ -336,8 +336,9 @@ typedef struct pf_key_desc {
  * the entry whose int8 key has the highest cosine similarity with
  * query_key.  The comparison is exact (integer dot products and squared
  * norms compared in 128-bit arithmetic); ties go to the lowest index;
- * all-zero keys are never selected.  Outputs: best[0] = index or -1,
- * similarity[0] = its cosine (fp32).  keys [n_entries][256] int8;
+ * all-zero keys are never selected.  keys, query_key and the three entry
+ * arrays must be 16-byte aligned.  Outputs: best[0] = index or -1,
+ * similarity[0] = its cosine (fp32, relative error below 3e-7).  keys [n_entries][256] int8;
  * entry_token, entry_pos, entry_bound [n_entries] int32.  Workspace:
  * pf_retrieval_workspace_size() bytes, zero-filled before first use and
  * left zero-filled; calls sharing a workspace must not overlap.

@@ -554,6 +554,8 @@ pf_status pf_retrieval_key(const pf_key_desc* d, void* workspace, size_t workspa
   pf::KeyArgs a = {};
   a.H = d->hidden;
   a.bf16 = d->dtype == PF_BF16;
+  a.vec = (d->hidden * elem_size(d->dtype)) % 16 == 0 && aligned16(d->hidden_state) &&
+          aligned16(d->projection);
   a.hidden = d->hidden_state;
   a.proj = d->projection;
   a.key_out = d->key_out;
@@ -576,8 +578,10 @@ pf_status pf_retrieve(const pf_retrieval_desc* d, void* workspace, size_t worksp
     return fail(PF_ERR_WORKSPACE, "%s: workspace needs %zu bytes", who, pf::kRetrievalWsBytes);
   if (d->n_entries < 0 || d->lo < 0 || d->lo > d->hi || d->hi > d->n_entries)
     return fail(PF_ERR_SHAPE, "%s: need 0 <= lo <= hi <= n_entries", who);
-  if (!aligned16(d->keys) || !aligned16(d->query_key) || !aligned16(workspace))
-    return fail(PF_ERR_ALIGN, "%s: keys, query_key and workspace must be 16-byte aligned", who);
+  if (!aligned16(d->keys) || !aligned16(d->query_key) || !aligned16(d->entry_token) ||
+      !aligned16(d->entry_pos) || !aligned16(d->entry_bound) || !aligned16(workspace))
+    return fail(PF_ERR_ALIGN, "%s: keys, query_key, entry arrays and workspace must be 16-byte aligned",
+                who);
   pf::RetrievalArgs a = {};
   a.lo = d->lo;
   a.hi = d->hi;

@@ -58,6 +58,12 @@ __device__ __forceinline__ long long row_offset(const ShiftArgs& a, int g, int p
 
 template <typename T>
 __global__ void __launch_bounds__(kShiftThreads) kv_shift_kernel(const ShiftArgs a) {
+  // cos / sin of the frequencies in shared memory: threads index the table
+  // by their own chunk, which from the parameter bank would serialise
+  __shared__ float2 s_cs[128];
+  const int D = a.row_bytes / a.elem_bytes;
+  for (int i = threadIdx.x; i < D / 2; i += kShiftThreads) s_cs[i] = a.cs[i];
+  __syncthreads();
   pdl_wait();
   using V = Vec<T>;
   const int l = blockIdx.y / a.Hkv, g = blockIdx.y % a.Hkv;
@@ -104,7 +110,7 @@ __global__ void __launch_bounds__(kShiftThreads) kv_shift_kernel(const ShiftArgs
 #pragma unroll
       for (int e = 0; e < V::N; e += 2) {
         const int i0 = chunk[u] * V::N + e;  // frequency index of this pair
-        const float2 cs0 = a.cs[i0], cs1 = a.cs[i0 + 1];
+        const float2 cs0 = s_cs[i0], cs1 = s_cs[i0 + 1];
         const float x0 = V::get(k1[u], e), y0 = V::get(k2[u], e);
         const float x1 = V::get(k1[u], e + 1), y1 = V::get(k2[u], e + 1);
         V::set_pair(o1, e >> 1, x0 * cs0.x - y0 * cs0.y, x1 * cs1.x - y1 * cs1.y);

@@ -144,6 +144,7 @@ constexpr size_t kRetrievalWsBytes = kRetrievalScanTicketOff + 64;
 
 struct KeyArgs {
   int H, bf16;
+  int vec;  // rows and pointers allow 16-byte loads
   const void* hidden;
   const void* proj;
   int8_t* key_out;

@@ -271,6 +271,10 @@ def test_retrieval_rejects_bad_arguments():
         (lambda: pb.pf_retrieve(_retrieval_desc(hi=101), 0x20000, ws), pb.PF_ERR_SHAPE),
         (lambda: pb.pf_retrieve(_retrieval_desc(lo=60, hi=50), 0x20000, ws), pb.PF_ERR_SHAPE),
         (lambda: pb.pf_retrieve(_retrieval_desc(keys=0x10004), 0x20000, ws), pb.PF_ERR_ALIGN),
+        (lambda: pb.pf_retrieve(_retrieval_desc(entry_token=0x10008), 0x20000, ws),
+         pb.PF_ERR_ALIGN),
+        (lambda: pb.pf_retrieve(_retrieval_desc(entry_bound=0x10004), 0x20000, ws),
+         pb.PF_ERR_ALIGN),
     ]
     for call, status in cases:
         with pytest.raises(pb.PfError) as e:

@@ -472,5 +472,16 @@ def check_project_key(project):
     assert list(key[:4]) == [127, 2, 4, -2]
 
 
+def check_retrieval_zero_keys(top1):
+    """An all-zero key has no cosine: it is never selected, not even over
+    entries of negative cosine, and alone it leaves nothing to select."""
+    q = np.array([3, 1, -2, 4], dtype=np.int8)
+    keys = np.array([[0, 0, 0, 0], [-3, -1, 2, -4], [0, 0, 0, 0]], dtype=np.int8)
+    tok, pos, bound = [9, 9, 9], [0, 0, 0], [1, 1, 1]
+    assert top1(q, keys, tok, pos, bound, 9)[0] == 1
+    assert top1(q, keys, tok, pos, bound, 9, lo=2)[0] == -1
+    assert top1(q, keys, tok, pos, bound, 9, hi=1)[0] == -1
+
+
 RETRIEVAL_CHECKS = [check_retrieval_golden, check_retrieval_float_bruteforce,
-                    check_retrieval_ties_and_ranges]
+                    check_retrieval_ties_and_ranges, check_retrieval_zero_keys]

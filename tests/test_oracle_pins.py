@@ -286,7 +286,8 @@ def test_project_key_pins():
     C.check_project_key(RV.project_key)
 
 
-def _top1_variant(ties_high=False, no_boundary=False, no_token=False, raw_dot=False):
+def _top1_variant(ties_high=False, no_boundary=False, no_token=False, raw_dot=False,
+                  zero_is_orthogonal=False):
     def fn(qkey, keys, tok, pos, bound, y, lo=0, hi=None):
         hi = len(keys) if hi is None else hi
         q = np.asarray(qkey, dtype=np.float64)
@@ -297,12 +298,19 @@ def _top1_variant(ties_high=False, no_boundary=False, no_token=False, raw_dot=Fa
             if not no_boundary and not int(pos[j]) < int(bound[j]):
                 continue
             k = np.asarray(keys[j], dtype=np.float64)
-            v = k @ q if raw_dot else (k @ q) / (np.linalg.norm(k) * np.linalg.norm(q))
+            if not k.any():
+                if not zero_is_orthogonal:
+                    continue
+                v = 0.0
+            else:
+                v = k @ q if raw_dot else (k @ q) / (np.linalg.norm(k) * np.linalg.norm(q))
             if best < 0 or v > bestv or (ties_high and v == bestv):
                 best, bestv = j, v
         if best < 0:
             return -1, float("nan")
         k = np.asarray(keys[best], dtype=np.float64)
+        if not k.any():
+            return best, 0.0
         return best, float((k @ q) / (np.linalg.norm(k) * np.linalg.norm(q)))
     return fn
 
@@ -312,6 +320,7 @@ RETRIEVAL_MUTANTS = {
     "ignores_boundary": _top1_variant(no_boundary=True),
     "ignores_token": _top1_variant(no_token=True),
     "raw_dot_product": _top1_variant(raw_dot=True),
+    "zero_key_as_orthogonal": _top1_variant(zero_is_orthogonal=True),
 }
 
 

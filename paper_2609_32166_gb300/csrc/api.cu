@@ -532,8 +532,9 @@ pf_status pf_kv_shift(const pf_shift_desc* d, void* stream) {
     const double ang = shift * std::pow((double)d->rope_base, -2.0 * i / D);
     a.cs[i] = make_float2((float)std::cos(ang), (float)std::sin(ang));
   }
-  if (num_sms() <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
-  cudaError_t e = pf::launch_kv_shift(a, static_cast<cudaStream_t>(stream), pdl_enabled());
+  const int sms = num_sms();
+  if (sms <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
+  cudaError_t e = pf::launch_kv_shift(a, static_cast<cudaStream_t>(stream), sms, pdl_enabled());
   return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
 }
 

@@ -3,13 +3,14 @@
 // p + (dst - src) and copying values, for all layers and KV heads in one
 // launch.  HBM-bound: every row is read once and written once.
 //
-// One CTA row = (layer, KV head).  A pass stages a block of rows (K and V
-// halves in registers), synchronises, then writes them.  Disjoint spans take
-// one pass per CTA; in the overlapping mode one CTA walks every pass in the
-// order that keeps the in-place move safe (ascending for a move to lower
-// positions, descending for higher).  A thread owns one
-// 16-byte chunk of a row's first half and the matching chunk of the second
-// half, i.e. whole rotary pairs (x_i, x_{i+D/2}).
+// Disjoint spans run as one flat grid-stride range of independent items.
+// Overlapping spans are cut into disjoint segments (below); only a shift so
+// small that this would take many launches uses the ordered mode, where one
+// CTA per (layer, KV head) stages a block of rows, synchronises, writes it,
+// and walks the blocks in the order that keeps the in-place move safe
+// (ascending for a move to lower positions, descending for higher).  An
+// item is one 16-byte chunk of a row's first half and the matching chunk of
+// the second half, i.e. whole rotary pairs (x_i, x_{i+D/2}), of K and V.
 #include "pf_internal.h"
 #include "pf_ptx.cuh"
 
@@ -56,6 +57,89 @@ __device__ __forceinline__ long long row_offset(const ShiftArgs& a, int g, int p
   return (((long long)page * a.Hkv + g) * PF_PAGE_SIZE + pos % PF_PAGE_SIZE) * a.row_bytes;
 }
 
+// K halves (k1, k2) of one 16-byte chunk pair rotated by the table, then K
+// and V stored at the destination row.
+template <typename T>
+__device__ __forceinline__ void rotate_store(const float2* s_cs, int chunk, const uint4& k1,
+                                             const uint4& k2, const uint4& v1, const uint4& v2,
+                                             char* kdst, char* vdst, int half_bytes) {
+  using V = Vec<T>;
+  uint4 o1 = k1, o2 = k2;
+#pragma unroll
+  for (int e = 0; e < V::N; e += 2) {
+    const int i0 = chunk * V::N + e;  // frequency index of this pair
+    const float2 cs0 = s_cs[i0], cs1 = s_cs[i0 + 1];
+    const float x0 = V::get(k1, e), y0 = V::get(k2, e);
+    const float x1 = V::get(k1, e + 1), y1 = V::get(k2, e + 1);
+    V::set_pair(o1, e >> 1, x0 * cs0.x - y0 * cs0.y, x1 * cs1.x - y1 * cs1.y);
+    V::set_pair(o2, e >> 1, x0 * cs0.y + y0 * cs0.x, x1 * cs1.y + y1 * cs1.x);
+  }
+  *reinterpret_cast<uint4*>(kdst + chunk * 16) = o1;
+  *reinterpret_cast<uint4*>(kdst + half_bytes + chunk * 16) = o2;
+  *reinterpret_cast<uint4*>(vdst + chunk * 16) = v1;
+  *reinterpret_cast<uint4*>(vdst + half_bytes + chunk * 16) = v2;
+}
+
+// Disjoint spans: every (layer, head, row, chunk) item is independent, so
+// the items form one flat range walked grid-stride by a grid sized to the
+// resident CTAs; each thread keeps kItemsPerThread items (16 loads) in
+// flight and needs no barrier.
+template <typename T>
+__global__ void __launch_bounds__(kShiftThreads) kv_shift_flat_kernel(const ShiftArgs a) {
+  __shared__ float2 s_cs[128];
+  const int D = a.row_bytes / a.elem_bytes;
+  for (int i = threadIdx.x; i < D / 2; i += kShiftThreads) s_cs[i] = a.cs[i];
+  __syncthreads();
+  pdl_wait();
+  // a dependent launch (the next segment of an overlapping move) may take
+  // the slots of finished CTAs; it reads nothing before its own wait
+  pdl_launch_dependents();
+  const int hc = a.row_bytes / 32;  // 16-byte chunks per half row
+  const int half_bytes = a.row_bytes / 2;
+  const long long per_head = (long long)a.count * hc;
+  const long long total = per_head * a.L * a.Hkv;
+  const long long stride = (long long)gridDim.x * kShiftThreads;
+  for (long long i0 = (long long)blockIdx.x * kShiftThreads + threadIdx.x; i0 < total;
+       i0 += stride * kItemsPerThread) {
+    uint4 k1[kItemsPerThread], k2[kItemsPerThread], v1[kItemsPerThread], v2[kItemsPerThread];
+    char* kd[kItemsPerThread];
+    char* vd[kItemsPerThread];
+    int chunk[kItemsPerThread];
+#pragma unroll
+    for (int u = 0; u < kItemsPerThread; ++u) {
+      const long long item = i0 + u * stride;
+      kd[u] = nullptr;
+      if (item < total) {
+        const int lh = (int)(item / per_head);
+        const long long rem = item - (long long)lh * per_head;
+        const int j = (int)(rem / hc);
+        const int c = (int)(rem - (long long)j * hc);
+        const int l = lh / a.Hkv, g = lh - l * a.Hkv;
+        const long long so = row_offset(a, g, a.src + j);
+        const long long d = row_offset(a, g, a.dst + j);
+        if (so < 0 || d < 0) {
+          flag_error(a.err, PF_DEVERR_CAPACITY);
+          continue;
+        }
+        const char* kb = a.cache_k + (long long)l * a.layer_bytes + so + c * 16;
+        const char* vb = a.cache_v + (long long)l * a.layer_bytes + so + c * 16;
+        k1[u] = *reinterpret_cast<const uint4*>(kb);
+        k2[u] = *reinterpret_cast<const uint4*>(kb + half_bytes);
+        v1[u] = *reinterpret_cast<const uint4*>(vb);
+        v2[u] = *reinterpret_cast<const uint4*>(vb + half_bytes);
+        kd[u] = a.cache_k + (long long)l * a.layer_bytes + d;
+        vd[u] = a.cache_v + (long long)l * a.layer_bytes + d;
+        chunk[u] = c;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kItemsPerThread; ++u)
+      if (kd[u]) rotate_store<T>(s_cs, chunk[u], k1[u], k2[u], v1[u], v2[u], kd[u], vd[u], half_bytes);
+  }
+}
+
+// Overlapping spans with a small shift: one CTA per (layer, KV head) walks
+// the passes in the safe order.
 template <typename T>
 __global__ void __launch_bounds__(kShiftThreads) kv_shift_kernel(const ShiftArgs a) {
   // cos / sin of the frequencies in shared memory: threads index the table
@@ -65,17 +149,15 @@ __global__ void __launch_bounds__(kShiftThreads) kv_shift_kernel(const ShiftArgs
   for (int i = threadIdx.x; i < D / 2; i += kShiftThreads) s_cs[i] = a.cs[i];
   __syncthreads();
   pdl_wait();
-  using V = Vec<T>;
   const int l = blockIdx.y / a.Hkv, g = blockIdx.y % a.Hkv;
   const int half_chunks = a.row_bytes / 32;  // 16-byte chunks per half row
   const int rows_per_pass = kItemsPerThread * kShiftThreads / half_chunks;
   const int passes = (a.count + rows_per_pass - 1) / rows_per_pass;
-  const int p_begin = a.overlap ? 0 : blockIdx.x;
-  const int p_end = a.overlap ? passes : min(passes, (int)blockIdx.x + 1);
+
   char* kbase = a.cache_k + (long long)l * a.layer_bytes;
   char* vbase = a.cache_v + (long long)l * a.layer_bytes;
   const int half_bytes = a.row_bytes / 2;
-  for (int pi = p_begin; pi < p_end; ++pi) {
+  for (int pi = 0; pi < passes; ++pi) {
     const int p = a.descending ? passes - 1 - pi : pi;
     uint4 k1[kItemsPerThread], k2[kItemsPerThread], v1[kItemsPerThread], v2[kItemsPerThread];
     long long dst_off[kItemsPerThread];
@@ -104,23 +186,10 @@ __global__ void __launch_bounds__(kShiftThreads) kv_shift_kernel(const ShiftArgs
     }
     __syncthreads();  // every source row of this pass is read before any write
 #pragma unroll
-    for (int u = 0; u < kItemsPerThread; ++u) {
-      if (dst_off[u] < 0) continue;
-      uint4 o1 = k1[u], o2 = k2[u];
-#pragma unroll
-      for (int e = 0; e < V::N; e += 2) {
-        const int i0 = chunk[u] * V::N + e;  // frequency index of this pair
-        const float2 cs0 = s_cs[i0], cs1 = s_cs[i0 + 1];
-        const float x0 = V::get(k1[u], e), y0 = V::get(k2[u], e);
-        const float x1 = V::get(k1[u], e + 1), y1 = V::get(k2[u], e + 1);
-        V::set_pair(o1, e >> 1, x0 * cs0.x - y0 * cs0.y, x1 * cs1.x - y1 * cs1.y);
-        V::set_pair(o2, e >> 1, x0 * cs0.y + y0 * cs0.x, x1 * cs1.y + y1 * cs1.x);
-      }
-      *reinterpret_cast<uint4*>(kbase + dst_off[u] + chunk[u] * 16) = o1;
-      *reinterpret_cast<uint4*>(kbase + dst_off[u] + half_bytes + chunk[u] * 16) = o2;
-      *reinterpret_cast<uint4*>(vbase + dst_off[u] + chunk[u] * 16) = v1[u];
-      *reinterpret_cast<uint4*>(vbase + dst_off[u] + half_bytes + chunk[u] * 16) = v2[u];
-    }
+    for (int u = 0; u < kItemsPerThread; ++u)
+      if (dst_off[u] >= 0)
+        rotate_store<T>(s_cs, chunk[u], k1[u], k2[u], v1[u], v2[u], kbase + dst_off[u],
+                        vbase + dst_off[u], half_bytes);
     __syncthreads();  // writes of this pass land before the next pass reads
   }
   pdl_launch_dependents();
@@ -137,16 +206,38 @@ __global__ void __launch_bounds__(kShiftThreads) kv_shift_kernel(const ShiftArgs
 // order inside one CTA per (layer, head).
 constexpr int kMaxSegments = 8;
 
-cudaError_t launch_kv_shift(const ShiftArgs& a0, cudaStream_t s, bool pdl) {
-  const int half_chunks = a0.row_bytes / 32;
-  const int rows_per_pass = kItemsPerThread * kShiftThreads / half_chunks;
+cudaError_t launch_kv_shift(const ShiftArgs& a0, cudaStream_t s, int num_sms, bool pdl) {
+  static int resident[64][2] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const int bf = a0.elem_bytes == 2;
+  int per_sm = dev < 64 ? resident[dev][bf] : 0;
+  if (per_sm == 0) {
+    e = bf ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+                 &per_sm, kv_shift_flat_kernel<__nv_bfloat16>, kShiftThreads, 0)
+           : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kv_shift_flat_kernel<float>,
+                                                            kShiftThreads, 0);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) per_sm = 1;
+    if (dev < 64) resident[dev][bf] = per_sm;
+  }
   auto launch = [&](const ShiftArgs& a) {
-    const int passes = (a.count + rows_per_pass - 1) / rows_per_pass;
-    const dim3 grid(a.overlap ? 1 : (unsigned)passes, (unsigned)(a.L * a.Hkv));
-    if (a.elem_bytes == 2)
-      return launch_ex(kv_shift_kernel<__nv_bfloat16>, grid, dim3(kShiftThreads), 0, s, 1, pdl,
-                       a);
-    return launch_ex(kv_shift_kernel<float>, grid, dim3(kShiftThreads), 0, s, 1, pdl, a);
+    if (a.overlap) {
+      const dim3 grid(1, (unsigned)(a.L * a.Hkv));
+      return bf ? launch_ex(kv_shift_kernel<__nv_bfloat16>, grid, dim3(kShiftThreads), 0, s, 1,
+                            pdl, a)
+                : launch_ex(kv_shift_kernel<float>, grid, dim3(kShiftThreads), 0, s, 1, pdl, a);
+    }
+    const long long items = (long long)a.count * (a.row_bytes / 32) * a.L * a.Hkv;
+    const long long want = (items + (long long)kShiftThreads * kItemsPerThread - 1) /
+                           ((long long)kShiftThreads * kItemsPerThread);
+    const unsigned grid = (unsigned)std::max<long long>(
+        1, std::min<long long>(want, (long long)num_sms * per_sm));
+    return bf ? launch_ex(kv_shift_flat_kernel<__nv_bfloat16>, dim3(grid), dim3(kShiftThreads), 0,
+                          s, 1, pdl, a)
+              : launch_ex(kv_shift_flat_kernel<float>, dim3(grid), dim3(kShiftThreads), 0, s, 1,
+                          pdl, a);
   };
   ShiftArgs a = a0;
   const int d = a0.dst > a0.src ? a0.dst - a0.src : a0.src - a0.dst;
@@ -167,7 +258,7 @@ cudaError_t launch_kv_shift(const ShiftArgs& a0, cudaStream_t s, bool pdl) {
     a.src = a0.src + off;
     a.dst = a0.dst + off;
     a.count = std::min(d, a0.count - off);
-    const cudaError_t e = launch(a);
+    e = launch(a);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;

@@ -130,7 +130,7 @@ struct ShiftArgs {
   float2 cs[128];  // cos / sin of shift * theta_i, i < D/2 (host, double precision)
 };
 
-cudaError_t launch_kv_shift(const ShiftArgs& a, cudaStream_t s, bool pdl);
+cudaError_t launch_kv_shift(const ShiftArgs& a, cudaStream_t s, int num_sms, bool pdl);
 
 // ------------------------------------------------------------ retrieval
 constexpr int kRetrievalMaxBlocks = 1024;

@@ -69,6 +69,14 @@ __device__ __forceinline__ bool cand_better(const Cand& a, const Cand& b) {
   return a.dot >= 0 ? gt : !gt;  // negative cosines: the smaller ratio is the larger cosine
 }
 
+// atomicAdd with release (publishes this thread's earlier writes) and
+// acquire (sees what earlier arrivals published) at GPU scope.
+__device__ __forceinline__ unsigned atomic_add_acq_rel(unsigned* p, unsigned v) {
+  unsigned old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+
 __device__ __forceinline__ float dot8_bf16(const uint4& x, const uint4& y, float acc) {
   const uint32_t* xa = &x.x;
   const uint32_t* ya = &y.x;
@@ -127,12 +135,12 @@ __global__ void __launch_bounds__(kKeyThreads) retrieval_key_kernel(const KeyArg
     for (int w = 0; w < kKeyRowThreads / 32; ++w) z += s_part[r * (kKeyRowThreads / 32) + w];
     a.z[row] = z;
   }
-  __threadfence();
+  // one release/acquire atomic per CTA publishes this CTA's rows (ordered
+  // before it by the barrier) and, in the last CTA, makes every row visible
   __syncthreads();
-  if (threadIdx.x == 0) s_last = (atomicAdd(a.ticket, 1u) == gridDim.x - 1);
+  if (threadIdx.x == 0) s_last = atomic_add_acq_rel(a.ticket, 1u) == gridDim.x - 1;
   __syncthreads();
   if (!s_last) return;
-  __threadfence();
   __shared__ float s_max[kKeyThreads / 32];
   const float z = threadIdx.x < PF_KEY_DIM ? __ldcg(&a.z[threadIdx.x]) : 0.f;
   float m = fabsf(z);
@@ -211,14 +219,6 @@ __device__ __forceinline__ void cp_async16(uint32_t saddr, const void* g) {
 
 __device__ __forceinline__ void cp_async_wait_all() {
   asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
-}
-
-// atomicAdd with release (publishes this thread's earlier writes) and
-// acquire (sees what earlier arrivals published) at GPU scope.
-__device__ __forceinline__ unsigned atomic_add_acq_rel(unsigned* p, unsigned v) {
-  unsigned old;
-  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
-  return old;
 }
 
 // Score up to kScanRound listed keys: all their bytes are copied to the

@@ -183,6 +183,14 @@ __device__ __forceinline__ void bulk_commit_group() {
 __device__ __forceinline__ void bulk_wait_read_all() {
   asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
+// 16-byte asynchronous global -> shared copy (L2 only), and the wait for
+// all of this thread's outstanding copies.
+__device__ __forceinline__ void cp_async16(uint32_t saddr, const void* g) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(saddr), "l"(g) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
 // Shared::cta address -> the same offset in the shared memory of CTA `rank`.
 __device__ __forceinline__ uint32_t mapa_cluster(uint32_t smem_addr, uint32_t rank) {
   uint32_t r;

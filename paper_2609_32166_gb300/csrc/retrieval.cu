@@ -213,14 +213,6 @@ __device__ __forceinline__ int filter_group(const RetrievalArgs& a, long long j0
   return __shfl_sync(0xffffffffu, incl, 31);
 }
 
-__device__ __forceinline__ void cp_async16(uint32_t saddr, const void* g) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(saddr), "l"(g) : "memory");
-}
-
-__device__ __forceinline__ void cp_async_wait_all() {
-  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
-}
-
 // Score up to kScanRound listed keys: all their bytes are copied to the
 // warp's stage with asynchronous 16-byte copies (coalesced, all in flight
 // at once), then lane i scores key i from shared memory (chunks visited in

@@ -255,6 +255,28 @@ def cpu_sample_text(w, nl):
 
 
 # ---------------------------------------------------------------------------
+# multi-rank aggregation (replicas: one process per GPU, no data exchange)
+# ---------------------------------------------------------------------------
+def max_over_ranks(x: float, world: int, device: str = "cpu") -> float:
+    """The largest x over all ranks (the slowest replica's time); x itself
+    when there is one rank.  `device` is where the reduction tensor lives
+    (cuda for nccl, cpu for gloo)."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: float, slowest_seconds: float, world: int) -> float:
+    """Units all ranks processed (every replica runs the same work) per
+    second of the slowest rank."""
+    return world * float(units_per_rank) / float(slowest_seconds)
+
+
+# ---------------------------------------------------------------------------
 # reference arm: the oracle as it stands, on the host cores
 # ---------------------------------------------------------------------------
 def run_reference(args):
@@ -454,18 +476,14 @@ def main():
         dist.barrier()
     clk = clocks.stop()
     assert len(per_step) == K
-    t_total_ms = float(np.sum(per_step))
-    if world > 1:
-        tt = torch.tensor([t_total_ms], device="cuda")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        t_total_ms = float(tt.item())
+    t_total_ms = max_over_ranks(float(np.sum(per_step)), world, "cuda")
     res = vs.results()
     assert res["err"] == 0, f"device error flag {res['err']}"
     assert int(np.sum(res["accept_len"] + 1)) == accepted_steps[-1]
 
     ms_step = t_total_ms / K
     accepted = float(np.mean(accepted_steps))
-    value = world * float(np.sum(accepted_steps)) / (t_total_ms / 1e3)
+    value = whole_job_rate(float(np.sum(accepted_steps)), t_total_ms / 1e3, world)
     attn_b, lm_b, commit_b = step_bytes(w, batch, res["accept_len"])
     attn_b_layer = attn_b
     step_b = attn_b * w.layers + lm_b + commit_b
@@ -715,8 +733,9 @@ def run_e2e(vs, w, batch, K, stream, flush, world, tok_table, planned):
             got = int((outs["accept_len"] + 1).sum())
             assert got == planned[k % len(planned)]
             tok += got
-    t = float(np.sum(times))
-    return {"value": world * tok / (t * 1e-3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+    t = max_over_ranks(float(np.sum(times)), world, "cuda")
+    return {"value": whole_job_rate(tok, t * 1e-3, world), "unit": "tokens/s",
+            "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": n, "ms_per_step": t / n}
 
 

@@ -485,3 +485,36 @@ def check_retrieval_zero_keys(top1):
 
 RETRIEVAL_CHECKS = [check_retrieval_golden, check_retrieval_float_bruteforce,
                     check_retrieval_ties_and_ranges, check_retrieval_zero_keys]
+
+
+# ----------------------------------------------------------------------------
+# prompt-prefix carryover
+# ----------------------------------------------------------------------------
+def check_prefix_special_cases(lcp):
+    assert lcp([], []) == 0
+    assert lcp([5, 6, 7], []) == 0
+    assert lcp([5, 6, 7], [5, 6, 7]) == 3              # identical prompts
+    assert lcp([5, 6, 7], [5, 6, 7, 8, 9]) == 3        # the old prompt is a prefix
+    assert lcp([5, 6, 7, 8, 9], [5, 6]) == 2           # the new prompt is a prefix
+    assert lcp([1, 2, 3], [9, 2, 3]) == 0              # differs at the first token
+    assert lcp([1, 2, 3, 4], [1, 2, 3, 5]) == 3        # differs at the last token
+    assert lcp([-1, 0, 2**31 - 1], [-1, 0, 2**31 - 1]) == 3   # negative / extreme keys
+
+
+def check_prefix_planted(lcp, seed=14):
+    """A mismatch planted at position k of otherwise equal random prompts is
+    found at k, in either argument order, whatever follows it."""
+    rng = np.random.default_rng(seed)
+    for _ in range(200):
+        n = int(rng.integers(1, 300))
+        a = rng.integers(0, 50, size=n)
+        b = a.copy()
+        k = int(rng.integers(0, n))
+        b[k] = a[k] + 1 + int(rng.integers(0, 5))
+        b[k + 1:] = rng.integers(0, 50, size=n - k - 1)   # anything may follow
+        tail = rng.integers(0, 50, size=int(rng.integers(0, 20)))
+        b = np.concatenate([b, tail])
+        assert lcp(a, b) == k and lcp(b, a) == k
+
+
+PREFIX_CHECKS = [check_prefix_special_cases, check_prefix_planted]

@@ -341,3 +341,39 @@ def test_project_key_mutants_caught():
     for mut in (round_half_up, no_normalise):
         with pytest.raises(AssertionError):
             C.check_project_key(mut)
+
+
+# ----------------------------------------------------------------------------
+# prompt-prefix carryover
+# ----------------------------------------------------------------------------
+from oracle import prefix as PX
+
+
+@pytest.mark.parametrize("check", C.PREFIX_CHECKS, ids=lambda f: f.__name__)
+def test_prefix_pins(check):
+    check(PX.common_prefix)
+
+
+def test_prefix_carry_over():
+    assert PX.carry_over([3, 4, 5, 6], [3, 4, 9, 6, 7]) == (2, 2, 3)
+
+
+def _lcp_off_by_one(a, b):
+    return min(PX.common_prefix(a, b) + 1, min(len(a), len(b)))
+
+
+def _lcp_shorter_only(a, b):
+    # forgets that a prompt ending early ends the common prefix
+    p = PX.common_prefix(a, b)
+    return max(p, min(len(a), len(b))) if p == 0 else p
+
+
+def _lcp_last_mismatch(a, b):
+    n = min(len(a), len(b))
+    diff = [i for i in range(n) if int(a[i]) != int(b[i])]
+    return diff[-1] if diff else n
+
+
+@pytest.mark.parametrize("mut", [_lcp_off_by_one, _lcp_shorter_only, _lcp_last_mismatch])
+def test_prefix_mutants_caught(mut):
+    assert _fails_some(C.PREFIX_CHECKS, mut) > 0

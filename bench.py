@@ -685,6 +685,34 @@ def measure_next_rows(stream, flush, hbm_peak, reps=4):
                       "scan_algorithmic_bytes": scan_bytes,
                       "scan_gbs": scan_bytes / (ms_s * 1e-3) / 1e9}
     assert int(err.item()) == 0
+    # --- pf_prefix_match: consecutive action-step prompts of 3.9K keys that
+    # share a 2.1K-key system prompt and history, then differ (new screenshot)
+    rng = np.random.default_rng(3)
+    shared = rng.integers(0, 151936, size=2100)
+    pairs = []
+    for r in range(reps):
+        a = np.concatenate([shared, rng.integers(1 << 30, (1 << 30) + (1 << 20), size=1800)])
+        b = np.concatenate([shared, rng.integers(1 << 30, (1 << 30) + (1 << 20), size=1800)])
+        pairs.append((torch.from_numpy(a.astype(np.int32)).cuda(),
+                      torch.from_numpy(b.astype(np.int32)).cuda()))
+    lcp = torch.zeros(2 * reps, dtype=torch.int32, device="cuda")
+    pds = []
+    for r, (a, b) in enumerate(pairs):
+        d = pb.pf_prefix_desc()
+        d.prev, d.n_prev, d.next, d.n_next = a.data_ptr(), a.numel(), b.data_ptr(), b.numel()
+        d.lcp, d.cache_len = lcp.data_ptr() + 8 * r, lcp.data_ptr() + 8 * r + 4
+        pds.append(d)
+
+    def matches(i):
+        for d in pds:
+            pb.pf_prefix_match(d, sp)
+
+    ms_p = _time_events(stream, flush, matches, 30) / reps
+    assert int(lcp[0].item()) >= 2100
+    out["prefix_match"] = {
+        "workload": "two 3900-key prompts sharing a 2100-key prefix",
+        "us": ms_p * 1e3, "bytes": 8 * 2101,
+        "timing": f"{reps} calls on {reps} prompt pairs per event pair, L2 flushed between pairs"}
     out["retrieval"] = {
         "workload": f"{M} entries (int8 256-d keys, Zipf(1.2) tokens), H={H} bf16 query state",
         "lookup": "pf_retrieval_key + pf_retrieve",

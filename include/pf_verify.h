@@ -364,6 +364,30 @@ PF_API pf_status pf_retrieval_key(const pf_key_desc* d, void* workspace, size_t 
 PF_API pf_status pf_retrieve(const pf_retrieval_desc* d, void* workspace, size_t workspace_bytes,
                              void* stream);
 
+/*
+ * pf_prefix_match -- prompt-prefix KV carryover (Section 3.4 "Prompt-prefix
+ * KV-state carryover"): p = the length of the longest identical prefix of
+ * the prompt whose K/V is cached (prev) and the new prompt (next).  Cached
+ * rows 0 .. p-1 stay valid; computation resumes at position p.  Prompts are
+ * int32 token keys: text tokens are their ids, image tokens an identifier of
+ * the image content at that position, so that "identical" covers content.
+ * Outputs (device): lcp[0] = p and, if cache_len is not NULL, cache_len[0]
+ * = p (the cache's new length; rows >= p are stale).  n_prev and n_next are
+ * in [0, 2^30]; prev / next may be NULL only when their length is 0.
+ * 16-byte aligned arrays are read with vector loads.  One launch, no
+ * workspace, no host synchronisation.
+ */
+typedef struct pf_prefix_desc {
+  const int32_t* prev;         /* device [n_prev] keys of the cached prompt  */
+  int32_t n_prev;
+  const int32_t* next;         /* device [n_next] keys of the new prompt     */
+  int32_t n_next;
+  int32_t* lcp;                /* out device [1]                             */
+  int32_t* cache_len;          /* optional out device [1]                    */
+} pf_prefix_desc;
+
+PF_API pf_status pf_prefix_match(const pf_prefix_desc* d, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -105,6 +105,11 @@ class pf_retrieval_desc(C.Structure):
                 ("similarity", C.c_void_p), ("error_flag", C.c_void_p)]
 
 
+class pf_prefix_desc(C.Structure):
+    _fields_ = [("prev", C.c_void_p), ("n_prev", C.c_int32), ("next", C.c_void_p),
+                ("n_next", C.c_int32), ("lcp", C.c_void_p), ("cache_len", C.c_void_p)]
+
+
 _lib = None
 
 
@@ -144,6 +149,8 @@ def lib() -> C.CDLL:
     L.pf_retrieve.restype = C.c_int
     L.pf_retrieve.argtypes = [C.POINTER(pf_retrieval_desc), C.c_void_p, C.c_size_t,
                               C.c_void_p]
+    L.pf_prefix_match.restype = C.c_int
+    L.pf_prefix_match.argtypes = [C.POINTER(pf_prefix_desc), C.c_void_p]
     _lib = L
     return L
 
@@ -219,3 +226,7 @@ def pf_retrieve(desc: pf_retrieval_desc, workspace: int, workspace_bytes: int,
                 stream: int = 0) -> None:
     _check(lib().pf_retrieve(C.byref(desc), C.c_void_p(workspace),
                              C.c_size_t(workspace_bytes), C.c_void_p(stream)))
+
+
+def pf_prefix_match(desc: pf_prefix_desc, stream: int = 0) -> None:
+    _check(lib().pf_prefix_match(C.byref(desc), C.c_void_p(stream)))

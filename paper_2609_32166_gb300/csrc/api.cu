@@ -604,4 +604,25 @@ pf_status pf_retrieve(const pf_retrieval_desc* d, void* workspace, size_t worksp
   return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
 }
 
+pf_status pf_prefix_match(const pf_prefix_desc* d, void* stream) {
+  static const char* who = "pf_prefix_match";
+  if (!d) return fail(PF_ERR_NULL, "%s: desc is NULL", who);
+  if (!d->lcp) return fail(PF_ERR_NULL, "%s: lcp is NULL", who);
+  if (d->n_prev < 0 || d->n_next < 0 || d->n_prev > (1 << 30) || d->n_next > (1 << 30))
+    return fail(PF_ERR_SHAPE, "%s: prompt lengths must be in [0, 2^30]", who);
+  if ((d->n_prev > 0 && !d->prev) || (d->n_next > 0 && !d->next))
+    return fail(PF_ERR_NULL, "%s: a prompt with keys has a NULL array", who);
+  pf::PrefixArgs a = {};
+  a.prev = d->prev;
+  a.next = d->next;
+  a.n_prev = d->n_prev;
+  a.n_next = d->n_next;
+  a.vec = aligned16(d->prev) && aligned16(d->next);
+  a.lcp = d->lcp;
+  a.cache_len = d->cache_len;
+  if (num_sms() <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
+  cudaError_t e = pf::launch_prefix_match(a, static_cast<cudaStream_t>(stream), pdl_enabled());
+  return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
+}
+
 }  // extern "C"

@@ -170,6 +170,18 @@ struct RetrievalArgs {
 cudaError_t launch_retrieval_key(const KeyArgs& a, cudaStream_t s, bool pdl);
 cudaError_t launch_retrieve(const RetrievalArgs& a, cudaStream_t s, int num_sms, bool pdl);
 
+// ------------------------------------------------------------ prefix carryover
+struct PrefixArgs {
+  const int32_t* prev;
+  const int32_t* next;
+  int n_prev, n_next;
+  int vec;  // both arrays 16-byte aligned
+  int32_t* lcp;
+  int32_t* cache_len;
+};
+
+cudaError_t launch_prefix_match(const PrefixArgs& a, cudaStream_t s, bool pdl);
+
 // Record the message pf_last_error() returns on this thread; returns s.
 pf_status set_error(pf_status s, const char* fmt, ...);
 

@@ -22,7 +22,8 @@ def test_exports_every_declared_symbol():
     assert set(names) >= {"pf_tree_prepare", "pf_verify_attention", "pf_lmhead_accept",
                           "pf_lmhead_accept_workspace_size", "pf_kv_commit", "pf_last_error",
                           "pf_version", "pf_kv_shift", "pf_retrieval_key", "pf_retrieve",
-                          "pf_retrieval_workspace_size", "pf_lmhead_accept_noalloc"}
+                          "pf_retrieval_workspace_size", "pf_lmhead_accept_noalloc",
+                          "pf_prefix_match"}
     L = pb.lib()
     for n in names:
         assert hasattr(L, n), n
@@ -46,6 +47,7 @@ int main(void) {
          offsetof(pf_shift_desc, cache_layer_stride), sizeof(pf_key_desc),
          offsetof(pf_key_desc, key_out), sizeof(pf_retrieval_desc),
          offsetof(pf_retrieval_desc, similarity));
+  printf("%zu %zu\n", sizeof(pf_prefix_desc), offsetof(pf_prefix_desc, cache_len));
   return 0;
 }
 '''
@@ -62,7 +64,8 @@ int main(void) {
             C.sizeof(pb.pf_shift_desc), pb.pf_shift_desc.cache.offset,
             pb.pf_shift_desc.cache_layer_stride.offset, C.sizeof(pb.pf_key_desc),
             pb.pf_key_desc.key_out.offset, C.sizeof(pb.pf_retrieval_desc),
-            pb.pf_retrieval_desc.similarity.offset]
+            pb.pf_retrieval_desc.similarity.offset,
+            C.sizeof(pb.pf_prefix_desc), pb.pf_prefix_desc.cache_len.offset]
     assert got == want
 
 
@@ -280,3 +283,18 @@ def test_retrieval_rejects_bad_arguments():
         with pytest.raises(pb.PfError) as e:
             call()
         assert e.value.status == status, pb.pf_last_error()
+
+
+def test_prefix_match_rejects_bad_arguments():
+    def desc(**kw):
+        d = pb.pf_prefix_desc()
+        d.prev, d.n_prev, d.next, d.n_next, d.lcp = 0x10000, 10, 0x10000, 12, 0x20000
+        for k, v in kw.items():
+            setattr(d, k, v)
+        return d
+    for kw, status in ((dict(lcp=None), pb.PF_ERR_NULL), (dict(n_prev=-1), pb.PF_ERR_SHAPE),
+                       (dict(n_next=(1 << 30) + 1), pb.PF_ERR_SHAPE),
+                       (dict(prev=None), pb.PF_ERR_NULL), (dict(next=None), pb.PF_ERR_NULL)):
+        with pytest.raises(pb.PfError) as e:
+            pb.pf_prefix_match(desc(**kw), 0)
+        assert e.value.status == status

@@ -350,3 +350,77 @@ def test_retrieve_saturated_keys_need_wide_products():
     assert _check_top1(mem, q, 3) == 50
     assert _check_top1(mem, q, 3, lo=0, hi=50) == 30
     assert _check_top1(mem, q, 3, lo=31, hi=50) == 40
+
+
+# ---------------------------------------------------------------------------
+# pf_prefix_match
+# ---------------------------------------------------------------------------
+from oracle import prefix as OPX
+
+
+def _prefix(prev, nxt, offset=0, with_len=True):
+    """Run pf_prefix_match on device copies; `offset` elements of padding in
+    front of each array make the pointers not 16-byte aligned."""
+    pad = np.zeros(offset, dtype=np.int32)
+    dp = torch.from_numpy(np.concatenate([pad, np.asarray(prev, np.int32)])).cuda()
+    dn = torch.from_numpy(np.concatenate([pad, np.asarray(nxt, np.int32)])).cuda()
+    out = torch.full((2,), -5, dtype=torch.int32, device="cuda")
+    d = pb.pf_prefix_desc()
+    d.prev = dp.data_ptr() + 4 * offset if len(prev) else None
+    d.next = dn.data_ptr() + 4 * offset if len(nxt) else None
+    d.n_prev, d.n_next = len(prev), len(nxt)
+    d.lcp = out.data_ptr()
+    d.cache_len = out.data_ptr() + 4 if with_len else None
+    pb.pf_prefix_match(d, _stream())
+    torch.cuda.synchronize()
+    got = out.cpu().numpy()
+    if not with_len:
+        assert got[1] == -5
+    else:
+        assert got[1] == got[0]
+    return int(got[0])
+
+
+@pytest.mark.parametrize("offset", [0, 1, 3])
+def test_prefix_match_planted(offset):
+    rng = np.random.default_rng(20 + offset)
+    n = 40000
+    a = rng.integers(0, 151936, size=n).astype(np.int32)
+    for k in (0, 1, 3, 4, 4095, 4096, 4097, 8191, 12345, n - 1):
+        b = a.copy()
+        b[k] ^= 1 + int(rng.integers(0, 1000))
+        b[k + 1:] = rng.integers(0, 151936, size=n - k - 1)
+        want = OPX.common_prefix(a, b)
+        assert want == k
+        assert _prefix(a, b, offset) == want
+        # other order, unequal lengths (the cut may remove the mismatch)
+        assert _prefix(b[: n - 7], a, offset) == OPX.common_prefix(b[: n - 7], a)
+
+
+def test_prefix_match_edges():
+    rng = np.random.default_rng(7)
+    a = rng.integers(-5, 5, size=9000).astype(np.int32)
+    assert _prefix(a, a) == 9000                              # identical prompts
+    assert _prefix(a, np.concatenate([a, a[:77]])) == 9000    # old prompt is a prefix
+    assert _prefix(a[:4100], a) == 4100
+    assert _prefix(a[:1], a[:1], offset=1) == 1
+    assert _prefix([], a) == 0
+    assert _prefix(a, []) == 0
+    assert _prefix([], []) == 0
+    assert _prefix(a, a, with_len=False) == 9000
+
+
+def test_prefix_match_action_step_prompts():
+    """Two consecutive action-step prompts of about 3.9K keys: shared system
+    prompt and history, then a new screenshot (content keys) and question."""
+    rng = np.random.default_rng(3)
+    system = rng.integers(0, 151936, size=1200)
+    hist = rng.integers(0, 151936, size=900)
+    img_prev = (1 << 30) + rng.integers(0, 1 << 20, size=1300)   # content keys of a screenshot
+    img_next = (1 << 30) + rng.integers(0, 1 << 20, size=1300)
+    tail = rng.integers(0, 151936, size=500)
+    prev = np.concatenate([system, hist, img_prev, tail]).astype(np.int32)
+    nxt = np.concatenate([system, hist, img_next, tail]).astype(np.int32)
+    want = OPX.common_prefix(prev, nxt)
+    assert 2100 <= want < 2110
+    assert _prefix(prev, nxt) == want

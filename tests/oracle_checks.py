@@ -518,3 +518,59 @@ def check_prefix_planted(lcp, seed=14):
 
 
 PREFIX_CHECKS = [check_prefix_special_cases, check_prefix_planted]
+
+
+# ----------------------------------------------------------------------------
+# proposal-length controller (eq. 1)
+# ----------------------------------------------------------------------------
+def check_expected_accepted_closed_forms(expected):
+    for p1 in (0.0, 0.3, 1.0):
+        assert expected(p1, 0.5, 0) == 0.0                       # no proposal, nothing accepted
+        assert abs(expected(p1, 0.0, 7) - p1) < 1e-12            # never continues
+        assert abs(expected(p1, 1.0, 7) - 7 * p1) < 1e-12        # always continues
+    for pc in (0.2, 0.9):                                        # geometric series
+        for ell in (1, 5, 64):
+            assert abs(expected(0.7, pc, ell) - 0.7 * (1 - pc ** ell) / (1 - pc)) < 1e-12
+
+
+def check_select_length_cases(select):
+    L = 8
+    # free verification, certain acceptance: the longest proposal
+    assert select([1.0] * (L + 1), [1.0] * (L + 1), [1.0] * (L + 1), L)[0] == L
+    # latency proportional to tokens produced: every length ties -> shortest
+    assert select([1.0 + l for l in range(L + 1)], [1.0] * (L + 1), [1.0] * (L + 1), L)[0] == 0
+    # nothing is ever accepted: greedy (l = 0) is cheapest
+    assert select([1.0 + 0.1 * l for l in range(L + 1)], [0.0] * (L + 1), [0.5] * (L + 1), L)[0] == 0
+    # hand-worked: T = (1, 1.2, 1.6), p1 = 0.5, pc = 0.5 -> objectives 1, 0.8, 0.91..
+    best, obj = select([1.0, 1.2, 1.6], [0.5] * 3, [0.5] * 3, 2)
+    assert best == 1 and abs(obj - 0.8) < 1e-12
+
+
+def check_latency_fit_exact(model_cls):
+    """Noise-free log-quadratic data are fitted exactly."""
+    c = (5.5, 0.004, -8e-6)
+    m = model_cls()
+    for ell in (0, 1, 4, 16, 64, 127, 3, 32):
+        m.update(ell, math.exp(c[0] + c[1] * ell + c[2] * ell * ell))
+    for ell in (0, 10, 100):
+        want = math.exp(c[0] + c[1] * ell + c[2] * ell * ell)
+        assert abs(m.predict(ell) / want - 1.0) < 1e-6
+
+
+def check_acceptance_consistency(model_cls, seed=15):
+    """Bernoulli acceptance at fixed rates: the online estimates approach
+    the rates (first token 0.8, continuation 0.6) at the trained (l, s)."""
+    rng = np.random.default_rng(seed)
+    m = model_cls(16, 0.05)
+    for _ in range(6000):
+        a = 0
+        if rng.random() < 0.8:
+            a = 1
+            while a < 16 and rng.random() < 0.6:
+                a += 1
+        m.update(16, 0.9, a)
+    p1, pc = m.predict(16, 0.9)
+    assert abs(p1 - 0.8) < 0.05 and abs(pc - 0.6) < 0.05
+
+
+CONTROLLER_CHECKS = [check_select_length_cases]

@@ -377,3 +377,55 @@ def _lcp_last_mismatch(a, b):
 @pytest.mark.parametrize("mut", [_lcp_off_by_one, _lcp_shorter_only, _lcp_last_mismatch])
 def test_prefix_mutants_caught(mut):
     assert _fails_some(C.PREFIX_CHECKS, mut) > 0
+
+
+# ----------------------------------------------------------------------------
+# proposal-length controller (eq. 1)
+# ----------------------------------------------------------------------------
+from oracle import controller as CT
+
+
+def test_controller_pins():
+    C.check_expected_accepted_closed_forms(CT.expected_accepted)
+    C.check_select_length_cases(CT.select_length)
+    C.check_latency_fit_exact(CT.LatencyModel)
+    C.check_acceptance_consistency(CT.AcceptanceModel)
+
+
+def test_controller_mutants_caught():
+    def no_plus_one(t, p1, pc, L):
+        best, bo = 0, None
+        for ell in range(L + 1):
+            o = t[ell] / max(CT.expected_accepted(p1[ell], pc[ell], ell), 1e-300)
+            if bo is None or o < bo:
+                best, bo = ell, o
+        return best, bo
+
+    def ties_longest(t, p1, pc, L):
+        best, bo = 0, None
+        for ell in range(L + 1):
+            o = t[ell] / (CT.expected_accepted(p1[ell], pc[ell], ell) + 1.0)
+            if bo is None or o <= bo:
+                best, bo = ell, o
+        return best, bo
+
+    for mut in (no_plus_one, ties_longest):
+        assert _fails_some(C.CONTROLLER_CHECKS, mut) > 0
+
+    def off_by_one_sum(p1, pc, ell):
+        return sum(p1 * pc ** k for k in range(1, ell + 1))
+    with pytest.raises(AssertionError):
+        C.check_expected_accepted_closed_forms(off_by_one_sum)
+
+    class LinearLatency(CT.LatencyModel):   # fits T, not log T
+        def update(self, ell, t):
+            super().update(ell, math.exp(t / 100.0))
+    with pytest.raises(AssertionError):
+        C.check_latency_fit_exact(LinearLatency)
+
+    class NoContinuation(CT.AcceptanceModel):   # continuation trials dropped
+        def update(self, ell, s, accepted):
+            x = self._x(ell, s)
+            self._step(self.w1, x, 1.0 if accepted >= 1 else 0.0, self.lr)
+    with pytest.raises(AssertionError):
+        C.check_acceptance_consistency(NoContinuation)

@@ -50,6 +50,8 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-next-rows", action="store_true",
                    help="skip the key re-rotation and retrieval measurements")
+    p.add_argument("--ell-sweep", action="store_true",
+                   help="verify-step latency vs proposal length on the workload's chain shape")
     p.add_argument("--cpu-worker", default=None, help=argparse.SUPPRESS)
     return p.parse_args()
 
@@ -326,6 +328,9 @@ def main():
         return
     if args.impl == "reference":
         run_reference(args)
+        return
+    if args.ell_sweep:
+        run_ell_sweep(args)
         return
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -720,6 +725,98 @@ def measure_next_rows(stream, flush, hbm_peak, reps=4):
                   "L2 flushed between pairs",
         "queries": res}
     return out
+
+
+ELL_POINTS = (0, 1, 2, 3, 4, 6, 8, 12, 16, 24, 32, 48, 64, 96, 127)
+
+
+def run_ell_sweep(args):
+    """Verify-step latency T(l) for chain proposals of l drafts (N = l + 1
+    nodes) on the workload's model shape and prefix: L attention launches,
+    the LM head with acceptance, the commit; CUDA-graph steps with events
+    at every step boundary, L2 flushed between steps (outside the events),
+    accepted length drawn per step as in the main benchmark.  Prints one
+    JSON line with the curve and a log-quadratic least-squares fit
+    log T = c0 + c1 l + c2 l^2 (the latency model of eq. 1's controller)."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_32166_gb300 import inputs as I
+    from paper_2609_32166_gb300.step import VerifyStep
+    base = I.WORKLOADS[args.workload]
+    weight = I.lm_weight(base, args.seed)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.Stream()
+    K = max(10, args.steps)
+    G = max(d for d in range(1, min(K, 50) + 1) if K % d == 0)
+    points = []
+    for ell in ELL_POINTS:
+        w = I.scaled(base, nodes=ell + 1, max_depth=ell, tree="chain", accept="chain", batch=1,
+                     layout="contiguous")
+        batch = I.make_batch(w, args.seed)
+        vs = VerifyStep(w, batch, np.zeros(batch.total_nodes, np.int32), weight=weight)
+        vs.lmhead()
+        torch.cuda.synchronize()
+        greedy = vs.argmax.cpu().numpy()
+        ends = I.step_forced_ends(batch, G)
+        toks = torch.from_numpy(np.stack([I.plant_tokens(batch, greedy, e, salt=g)
+                                          for g, e in enumerate(ends)])).cuda()
+        with torch.cuda.stream(stream):
+            for k in range(max(args.warmup, 3)):
+                flush.zero_()
+                vs.tokens.copy_(toks[k % G])
+                vs.step(stream.cuda_stream)
+        stream.synchronize()
+        ev = [(torch.cuda.Event(enable_timing=True, external=True),
+               torch.cuda.Event(enable_timing=True, external=True)) for _ in range(G)]
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr, stream=stream):
+            st = torch.cuda.current_stream()
+            for g in range(G):
+                flush.zero_()
+                vs.tokens.copy_(toks[g])
+                ev[g][0].record(st)
+                vs.step(st.cuda_stream)
+                ev[g][1].record(st)
+        times = []
+        with torch.cuda.stream(stream):
+            gr.replay()   # untimed: uploads the graph
+            stream.synchronize()
+            for r in range(K // G):
+                gr.replay()
+                stream.synchronize()
+                times.extend(a.elapsed_time(b) for a, b in ev)
+        res = vs.results()
+        assert res["err"] == 0
+        del vs, gr
+        torch.cuda.empty_cache()
+        points.append({"ell": ell, "nodes": ell + 1, "us_step": float(np.mean(times)) * 1e3})
+    ell = np.array([p["ell"] for p in points], dtype=np.float64)
+    logt = np.log(np.array([p["us_step"] for p in points]))
+    A = np.stack([np.ones_like(ell), ell, ell * ell], axis=1)
+    coef, *_ = np.linalg.lstsq(A, logt, rcond=None)
+    # eq. 1 driven by the measured curve: the library's controller fits its
+    # latency model to the points; for a per-token acceptance rate q (p1 =
+    # pc = q) the chosen length and the resulting tokens per second
+    from paper_2609_32166_gb300 import binding as pb
+    l_max = ELL_POINTS[-1]
+    ctl = pb.pf_controller_init(l_max, 0.05, 0.0)
+    for p in points:
+        pb.pf_controller_observe(ctl, p["ell"], 0.0, -1, p["us_step"])
+    u = np.arange(l_max + 1) / l_max
+    t_hat = np.exp(ctl.c[0] + ctl.c[1] * u + ctl.c[2] * u * u)
+    choices = []
+    for q in (0.3, 0.6, 0.8, 0.9, 0.95, 0.99):
+        best, obj = pb.pf_length_select(t_hat, np.full(l_max + 1, q), np.full(l_max + 1, q))
+        choices.append({"per_token_acceptance": q, "chosen_length": best,
+                        "us_per_token": obj, "tokens_per_s": 1e6 / obj})
+    print(json.dumps({"mode": "ell_sweep", "workload": base.name, "unit": "us per verify step",
+                      "steps_per_point": K, "points": points,
+                      "log_quadratic_fit": [float(c) for c in coef],
+                      "controller": {"l_max": l_max, "latency_model": list(ctl.c),
+                                     "choices": choices},
+                      "timing": "CUDA graphs of %d steps, events around every step; L2 "
+                                "flushed before every step, outside the events" % G}))
 
 
 def run_e2e(vs, w, batch, K, stream, flush, world, tok_table, planned):

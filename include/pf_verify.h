@@ -388,6 +388,54 @@ typedef struct pf_prefix_desc {
 
 PF_API pf_status pf_prefix_match(const pf_prefix_desc* d, void* stream);
 
+/*
+ * Proposal-length controller (Section 3.2 "Runtime-adaptive
+ * proposal-length controller", eq. 1).  Host code: no GPU, no allocation.
+ *
+ *   L* = argmin_{0 <= l <= l_max}  T(l) / (A(l, s) + 1),
+ *   A(l, s) = sum_{k=1..l} p1 * pc^(k-1)
+ *
+ * p1 (first proposal token accepted) and pc (token k accepted given token
+ * k-1 was) come from two online logistic regressions on x = (1, l/l_max,
+ * s); one observation (l, s, a accepted tokens) is one first-token trial
+ * (success iff a >= 1) and, if a >= 1, the continuation trials k = 2 ..
+ * min(a+1, l) (success iff k <= a), each a gradient step
+ * w += lr (y - sigmoid(w.x)) x.  T(l) = exp(c0 + c1 u + c2 u^2), u =
+ * l / l_max, is fitted to observed iteration latencies by recursive least
+ * squares from a zero prior of variance 1e8.  Ties go to the shorter length.  Exploration: with
+ * the caller's uniform draw u < epsilon the choice moves to an adjacent
+ * length (up unless at l_max, or down when u_dir >= 0.5 and above 0).
+ */
+typedef struct pf_length_controller {
+  int32_t l_max;
+  int32_t n_latency;   /* latency observations so far                      */
+  double lr;           /* logistic-regression step size                    */
+  double epsilon;      /* exploration rate                                 */
+  double w_first[3];
+  double w_cont[3];
+  double c[3];         /* log-latency coefficients                         */
+  double P[9];         /* recursive-least-squares covariance, row-major    */
+} pf_length_controller;
+
+#define PF_CTL_MAX_LEN 4096
+
+/* l_max in [1, PF_CTL_MAX_LEN], lr > 0, epsilon in [0, 1]. */
+PF_API pf_status pf_controller_init(pf_length_controller* c, int32_t l_max, double lr,
+                                    double epsilon);
+/* One decoding iteration's outcome: ell in [0, l_max], similarity s,
+ * accepted in [0, ell] (or < 0: no acceptance observation), latency_us > 0
+ * (or <= 0: no latency observation). */
+PF_API pf_status pf_controller_observe(pf_length_controller* c, int32_t ell, double similarity,
+                                       int32_t accepted, double latency_us);
+/* The next length for similarity s; u, u_dir are the caller's uniform
+ * draws in [0, 1) for exploration.  objective_out may be NULL. */
+PF_API pf_status pf_controller_choose(const pf_length_controller* c, double similarity, double u,
+                                      double u_dir, int32_t* ell_out, double* objective_out);
+/* Eq. 1 over explicit estimates t_hat[l], p_first[l], p_cont[l], l = 0..l_max. */
+PF_API pf_status pf_length_select(const double* t_hat, const double* p_first,
+                                  const double* p_cont, int32_t l_max, int32_t* ell_out,
+                                  double* objective_out);
+
 #ifdef __cplusplus
 }
 #endif

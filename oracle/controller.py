@@ -15,9 +15,9 @@ Estimators (the paper names their form, not their details; readings):
     gives one first-token trial (success iff a >= 1) and, when a >= 1, the
     continuation trials k = 2 .. min(a + 1, l) (success iff k <= a); each
     trial is one gradient step w += lr (y - sigmoid(w.x)) x.
-  * latency: log T(l) = c0 + c1 l + c2 l^2 fitted by recursive least
-    squares from a zero prior of variance 1e8 per coefficient (least
-    squares up to a relative bias of about 1e-8).
+  * latency: log T(l) = c0 + c1 u + c2 u^2 with u = l / l_max, fitted by
+    recursive least squares from a zero prior of variance 1e8 per
+    coefficient (least squares up to a relative bias of about 1e-8).
   * ties in the objective go to the shortest length; "occasionally explores
     an adjacent length": with the caller's uniform draw u < epsilon the
     choice moves to L* + 1 (or L* - 1 at l_max), the direction given by a
@@ -79,15 +79,21 @@ class AcceptanceModel:
 
 
 class LatencyModel:
-    """Recursive least squares for log T = c . (1, l, l^2)."""
+    """Recursive least squares for log T = c . (1, l/l_scale, (l/l_scale)^2)
+    (the scaled length keeps the normal equations well conditioned)."""
 
-    def __init__(self, prior_var=1e8):
+    def __init__(self, l_scale=128, prior_var=1e8):
+        self.l_scale = l_scale
         self.c = [0.0, 0.0, 0.0]
         self.P = [[prior_var if i == j else 0.0 for j in range(3)] for i in range(3)]
         self.n = 0
 
+    def _x(self, ell):
+        u = ell / self.l_scale
+        return [1.0, u, u * u]
+
     def update(self, ell, t):
-        x = [1.0, float(ell), float(ell) * ell]
+        x = self._x(ell)
         y = math.log(t)
         Px = [sum(self.P[i][j] * x[j] for j in range(3)) for i in range(3)]
         denom = 1.0 + sum(x[i] * Px[i] for i in range(3))
@@ -98,10 +104,12 @@ class LatencyModel:
         self.n += 1
 
     def predict(self, ell):
-        return math.exp(self.c[0] + self.c[1] * ell + self.c[2] * ell * ell)
+        x = self._x(ell)
+        return math.exp(self.c[0] * x[0] + self.c[1] * x[1] + self.c[2] * x[2])
 
 
 def choose(lat, acc, s, l_max, u=1.0, u_dir=0.0, epsilon=0.0):
+    """lat: a LatencyModel with l_scale = l_max."""
     """The controller's choice for similarity s from the two estimators."""
     t = [lat.predict(ell) for ell in range(l_max + 1)]
     pr = [acc.predict(ell, s) for ell in range(l_max + 1)]

@@ -22,6 +22,7 @@ LIB = os.path.join(PKG, "libpfverify.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "--expt-relaxed-constexpr",
                  "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
+                 "-Xcompiler", "-ffp-contract=off",
                  "-I", INCLUDE, "-I", CSRC]
 
 

@@ -110,6 +110,12 @@ class pf_prefix_desc(C.Structure):
                 ("n_next", C.c_int32), ("lcp", C.c_void_p), ("cache_len", C.c_void_p)]
 
 
+class pf_length_controller(C.Structure):
+    _fields_ = [("l_max", C.c_int32), ("n_latency", C.c_int32), ("lr", C.c_double),
+                ("epsilon", C.c_double), ("w_first", C.c_double * 3), ("w_cont", C.c_double * 3),
+                ("c", C.c_double * 3), ("P", C.c_double * 9)]
+
+
 _lib = None
 
 
@@ -149,6 +155,19 @@ def lib() -> C.CDLL:
     L.pf_retrieve.restype = C.c_int
     L.pf_retrieve.argtypes = [C.POINTER(pf_retrieval_desc), C.c_void_p, C.c_size_t,
                               C.c_void_p]
+    L.pf_controller_init.restype = C.c_int
+    L.pf_controller_init.argtypes = [C.POINTER(pf_length_controller), C.c_int32, C.c_double,
+                                     C.c_double]
+    L.pf_controller_observe.restype = C.c_int
+    L.pf_controller_observe.argtypes = [C.POINTER(pf_length_controller), C.c_int32, C.c_double,
+                                        C.c_int32, C.c_double]
+    L.pf_controller_choose.restype = C.c_int
+    L.pf_controller_choose.argtypes = [C.POINTER(pf_length_controller), C.c_double, C.c_double,
+                                       C.c_double, C.POINTER(C.c_int32),
+                                       C.POINTER(C.c_double)]
+    L.pf_length_select.restype = C.c_int
+    L.pf_length_select.argtypes = [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32,
+                                   C.POINTER(C.c_int32), C.POINTER(C.c_double)]
     L.pf_prefix_match.restype = C.c_int
     L.pf_prefix_match.argtypes = [C.POINTER(pf_prefix_desc), C.c_void_p]
     _lib = L
@@ -230,3 +249,34 @@ def pf_retrieve(desc: pf_retrieval_desc, workspace: int, workspace_bytes: int,
 
 def pf_prefix_match(desc: pf_prefix_desc, stream: int = 0) -> None:
     _check(lib().pf_prefix_match(C.byref(desc), C.c_void_p(stream)))
+
+
+def pf_controller_init(l_max: int, lr: float, epsilon: float) -> pf_length_controller:
+    c = pf_length_controller()
+    _check(lib().pf_controller_init(C.byref(c), l_max, lr, epsilon))
+    return c
+
+
+def pf_controller_observe(c: pf_length_controller, ell: int, similarity: float, accepted: int,
+                          latency_us: float) -> None:
+    _check(lib().pf_controller_observe(C.byref(c), ell, similarity, accepted, latency_us))
+
+
+def pf_controller_choose(c: pf_length_controller, similarity: float, u: float = 1.0,
+                         u_dir: float = 0.0) -> tuple:
+    ell, obj = C.c_int32(), C.c_double()
+    _check(lib().pf_controller_choose(C.byref(c), similarity, u, u_dir, C.byref(ell),
+                                      C.byref(obj)))
+    return int(ell.value), float(obj.value)
+
+
+def pf_length_select(t_hat, p_first, p_cont) -> tuple:
+    """Eq. 1 over explicit float64 arrays of length l_max + 1 (host)."""
+    t = np.ascontiguousarray(t_hat, dtype=np.float64)
+    p1 = np.ascontiguousarray(p_first, dtype=np.float64)
+    pc = np.ascontiguousarray(p_cont, dtype=np.float64)
+    assert t.shape == p1.shape == pc.shape and t.ndim == 1
+    ell, obj = C.c_int32(), C.c_double()
+    _check(lib().pf_length_select(t.ctypes.data, p1.ctypes.data, pc.ctypes.data,
+                                  int(t.shape[0]) - 1, C.byref(ell), C.byref(obj)))
+    return int(ell.value), float(obj.value)

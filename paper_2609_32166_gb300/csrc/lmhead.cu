@@ -13,6 +13,8 @@
 // Every CTA then folds its per-node best into the workspace with a 64-bit
 // atomicMax; the last CTA to finish (a ticket counter, no spinning) decodes
 // the argmax of every node and walks each proposal tree.
+#include <cstdlib>
+
 #include "pf_internal.h"
 #include "pf_ptx.cuh"
 
@@ -24,7 +26,7 @@ constexpr int kBM = 128;           // vocabulary rows per tile (UMMA M)
 constexpr int kBK = 64;            // hidden elements per stage (128 bytes of bf16)
 constexpr int kABytes = kBM * kBK * 2;
 constexpr int kTcThreads = 192;    // warp 0 TMA, warp 1 MMA, warps 2..5 epilogue
-constexpr int kMaxStages = 8;
+constexpr int kMaxStages = 12;
 
 // Greedy descent of every proposal tree of the batch.  Runs in the last CTA
 // after all per-node maxima are final.  One warp per sequence.
@@ -318,17 +320,22 @@ __global__ void __launch_bounds__(256) lmhead_f32_kernel(const LmArgs a) {
 
 }  // namespace
 
-int lmhead_bf16_stages(int npad) {
-  const int stage = kABytes + npad * 128;
-  int ns = (200 * 1024) / stage;
-  if (ns > kMaxStages) ns = kMaxStages;
-  if (ns < 2) ns = 2;
-  return ns;
-}
-
 int lmhead_bf16_smem_bytes(int npad, int stages) {
   return 1024 + stages * (kABytes + npad * 128) + (2 * kMaxStages + 4) * 8 + 8 +
          PF_MAX_LM_ROWS * 8 + PF_MAX_LM_ROWS * 4 + 16;
+}
+
+// Ring depth: as many stages as about 200 KB of shared memory holds (at
+// most kMaxStages, at least 2); PF_LM_STAGES overrides it within what the
+// 227 KB per-CTA limit allows.
+int lmhead_bf16_stages(int npad) {
+  const int stage = kABytes + npad * 128;
+  int ns = (200 * 1024) / stage;
+  if (const char* e = getenv("PF_LM_STAGES")) ns = atoi(e);
+  if (ns > kMaxStages) ns = kMaxStages;
+  while (ns > 2 && lmhead_bf16_smem_bytes(npad, ns) > 232448) --ns;
+  if (ns < 2) ns = 2;
+  return ns;
 }
 
 cudaError_t launch_lmhead_bf16(const LmArgs& a, const CUtensorMap& w_map,

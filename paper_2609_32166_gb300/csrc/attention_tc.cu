@@ -254,17 +254,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         for (int c = 0; c < 64; ++c)
           if (!((vis >> c) & 1ull)) sv[c] = -INFINITY;
       }
-      // row maximum of the raw scores (scale > 0 commutes with max), as a
-      // tree so that the dependent chain is 6 deep rather than 64
-      float mxs[8];
+      // row maximum of the raw scores (scale > 0 commutes with max): a tree
+      // of three-input maxima, 64 -> 22 -> 8 -> 3 -> 1 (32 instructions)
+      float m22[22];
 #pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        float m2 = fmaxf(fmaxf(sv[k], sv[k + 8]), fmaxf(sv[k + 16], sv[k + 24]));
-        float m3 = fmaxf(fmaxf(sv[k + 32], sv[k + 40]), fmaxf(sv[k + 48], sv[k + 56]));
-        mxs[k] = fmaxf(m2, m3);
-      }
-      const float mx = fmaxf(fmaxf(fmaxf(mxs[0], mxs[1]), fmaxf(mxs[2], mxs[3])),
-                             fmaxf(fmaxf(mxs[4], mxs[5]), fmaxf(mxs[6], mxs[7]))) *
+      for (int k = 0; k < 21; ++k) m22[k] = fmax3(sv[3 * k], sv[3 * k + 1], sv[3 * k + 2]);
+      m22[21] = sv[63];
+      float m8[8];
+#pragma unroll
+      for (int k = 0; k < 7; ++k) m8[k] = fmax3(m22[3 * k], m22[3 * k + 1], m22[3 * k + 2]);
+      m8[7] = m22[21];
+      const float mx = fmax3(fmax3(m8[0], m8[1], m8[2]), fmax3(m8[3], m8[4], m8[5]),
+                             fmaxf(m8[6], m8[7])) *
                        a.scale_log2;
       const float m_new = fmaxf(m_ref, mx);
       const bool resc = m_ref != -INFINITY && m_new > m_ref + kRescaleLog2;
@@ -289,18 +290,25 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           m_ref = m_new;
         }
       }
-      // p = 2^(s * scale_log2 - m): one FFMA and one MUFU per score
+      // p = 2^(s * scale_log2 - m): one paired FMA per two scores, one MUFU
+      // per score; the row sum in four paired accumulators
       const float neg_mu = m_ref == -INFINITY ? 0.f : -m_ref;
-      float rs[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      const unsigned long long sc2 = f32x2_pack(a.scale_log2, a.scale_log2);
+      const unsigned long long mu2 = f32x2_pack(neg_mu, neg_mu);
+      unsigned long long rs2[4] = {0ull, 0ull, 0ull, 0ull};
       uint32_t pk[32];
 #pragma unroll
       for (int c = 0; c < 32; ++c) {
-        const float p0 = ex2_approx(fmaf(sv[2 * c], a.scale_log2, neg_mu));
-        const float p1 = ex2_approx(fmaf(sv[2 * c + 1], a.scale_log2, neg_mu));
-        rs[c & 7] += p0 + p1;
+        float x0, x1;
+        f32x2_unpack(ffma2(f32x2_pack(sv[2 * c], sv[2 * c + 1]), sc2, mu2), x0, x1);
+        const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+        const unsigned long long p2 = f32x2_pack(p0, p1);
+        rs2[c & 3] = fadd2(rs2[c & 3], p2);
         pk[c] = pack_bf16(p0, p1);
       }
-      l += ((rs[0] + rs[1]) + (rs[2] + rs[3])) + ((rs[4] + rs[5]) + (rs[6] + rs[7]));
+      float r0, r1;
+      f32x2_unpack(fadd2(fadd2(rs2[0], rs2[1]), fadd2(rs2[2], rs2[3])), r0, r1);
+      l += r0 + r1;
       // P buffer sb was last read by PV_{i-2}.
       if (i >= 2) mbar_wait(smem_u32(&pv_done[sb]), ((i - 2) >> 1) & 1, a.err);
       uint8_t* prow = sP + sb * S::kPBytes + r * 128;

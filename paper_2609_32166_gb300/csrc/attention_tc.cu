@@ -181,36 +181,60 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       const uint32_t id_o = umma_idesc_bf16_bmn(128, D);
       bool ok = mbar_wait(smem_u32(q_full), 0, a.err);
       const uint32_t q0 = smem_u32(sQ);
-      for (int i = 0; i <= my_tiles && ok; ++i) {
-        if (i < my_tiles) {
-          const int st = i % kTcStages, sb = i & 1;
-          ok = mbar_wait(smem_u32(&kv_full[st]), (i / kTcStages) & 1, a.err) &&
-               mbar_wait(smem_u32(&s_empty[sb]), ((i >> 1) & 1) ^ 1, a.err);
-          if (!ok) break;
-          tc_fence_after();
-          const uint32_t k0 = smem_u32(sKV + st * S::kStageBytes);
+      // Event-driven issue: S_n as soon as its K/V tile has landed and the
+      // softmax has read S_{n-2} out of the same TMEM buffer; PV_j as soon
+      // as P_j is in shared memory.  S_{n+1} thus never waits behind P_{n-1}
+      // and is computed while the softmax still works on S_{n-1}, S_n.
+      int ns = 0, np = 0;
+      unsigned idle = 0;
+      unsigned long long t0 = 0;
+      while (ok && np < my_tiles) {
+        bool progressed = false;
+        if (ns < my_tiles) {
+          const int st = ns % kTcStages, sb = ns & 1;
+          if (mbar_test_wait(smem_u32(&kv_full[st]), (ns / kTcStages) & 1) &&
+              mbar_test_wait(smem_u32(&s_empty[sb]), ((ns >> 1) & 1) ^ 1)) {
+            tc_fence_after();
+            const uint32_t k0 = smem_u32(sKV + st * S::kStageBytes);
 #pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk) {
-            const uint32_t qa = q0 + (kk >> 2) * (128 * 128) + (kk & 3) * 32;
-            const uint32_t kb = k0 + (kk >> 2) * (kBN * 128) + (kk & 3) * 32;
-            umma_bf16(tmem + sb * kBN, umma_desc_sw128(qa), umma_desc_sw128(kb), id_s, kk > 0);
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t qa = q0 + (kk >> 2) * (128 * 128) + (kk & 3) * 32;
+              const uint32_t kb = k0 + (kk >> 2) * (kBN * 128) + (kk & 3) * 32;
+              umma_bf16(tmem + sb * kBN, umma_desc_sw128(qa), umma_desc_sw128(kb), id_s, kk > 0);
+            }
+            umma_commit(smem_u32(&s_full[sb]));
+            ++ns;
+            progressed = true;
           }
-          umma_commit(smem_u32(&s_full[sb]));
         }
-        if (i >= 1) {
-          const int j = i - 1, pb = j & 1, stj = j % kTcStages;
-          ok = mbar_wait(smem_u32(&p_full[pb]), (j >> 1) & 1, a.err);
-          if (!ok) break;
-          tc_fence_after();
-          const uint32_t p0 = smem_u32(sP + pb * S::kPBytes);
-          const uint32_t v0 = smem_u32(sKV + stj * S::kStageBytes + S::kTileBytes);
+        if (np < ns) {
+          const int pb = np & 1, stj = np % kTcStages;
+          if (mbar_test_wait(smem_u32(&p_full[pb]), (np >> 1) & 1)) {
+            tc_fence_after();
+            const uint32_t p0 = smem_u32(sP + pb * S::kPBytes);
+            const uint32_t v0 = smem_u32(sKV + stj * S::kStageBytes + S::kTileBytes);
 #pragma unroll
-          for (int kt = 0; kt < kBN / 16; ++kt)
-            umma_bf16(tmem + 2 * kBN, umma_desc_sw128(p0 + kt * 32),
-                      umma_desc_sw128_lbo(v0 + kt * 16 * 128, kBN * 128, 1024), id_o,
-                      (j > 0 || kt > 0) ? 1u : 0u);
-          umma_commit(smem_u32(&pv_done[pb]));
-          umma_commit(smem_u32(&kv_empty[stj]));
+            for (int kt = 0; kt < kBN / 16; ++kt)
+              umma_bf16(tmem + 2 * kBN, umma_desc_sw128(p0 + kt * 32),
+                        umma_desc_sw128_lbo(v0 + kt * 16 * 128, kBN * 128, 1024), id_o,
+                        (np > 0 || kt > 0) ? 1u : 0u);
+            umma_commit(smem_u32(&pv_done[pb]));
+            umma_commit(smem_u32(&kv_empty[stj]));
+            ++np;
+            progressed = true;
+          }
+        }
+        // bounded like mbar_wait: give up (and flag) after kWaitLimitNs
+        // without progress
+        if (progressed) {
+          idle = 0;
+        } else if ((++idle & 63u) == 0u) {
+          const unsigned long long now = globaltimer();
+          if (t0 == 0 || idle == 64u) t0 = now;
+          if (now - t0 > kWaitLimitNs) {
+            flag_error(a.err, PF_DEVERR_TIMEOUT);
+            ok = false;
+          }
         }
       }
     }

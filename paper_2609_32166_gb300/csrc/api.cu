@@ -133,12 +133,12 @@ int max_cluster_for(int kernel, int D, int want) {
   return w;
 }
 
-int tc_max_active_clusters(int cluster) {
-  static int cache[64][17];
+int tc_max_active_clusters(int cluster, int bm) {
+  static int cache[64][2][17];
   int dev = 0;
   cudaGetDevice(&dev);
-  int& c = cache[dev & 63][cluster];
-  if (c == 0) c = std::max(1, pf::attention_tc_max_active_clusters(cluster)) + 1;
+  int& c = cache[dev & 63][bm > 128 ? 1 : 0][cluster];
+  if (c == 0) c = std::max(1, pf::attention_tc_max_active_clusters(cluster, bm)) + 1;
   return c - 1;
 }
 
@@ -152,8 +152,14 @@ bool use_tc_attention(const pf::AttnArgs& a) {
 void choose_attention_shape(pf::AttnArgs& a, int max_prefix_len, int sms) {
   const int max_tiles = (max_prefix_len + 63) / 64 + (a.max_nodes + 63) / 64;
   if (use_tc_attention(a)) {
-    a.bm = 128;
-    a.nb = 128 / a.G;
+    // Two 128-row blocks per CTA (each K/V tile serves 256 rows, two
+    // softmax warpgroups) when that covers all of a KV head's rows; beyond
+    // 256 rows the tensor pipe of one SM, not the tile reads, bounds a CTA,
+    // and 128-row CTAs spread the work over more SMs.
+    const int head_rows = a.G * a.max_nodes;
+    a.bm = head_rows > 128 && head_rows <= 256 ? 256 : 128;
+    if (const char* e = getenv("PF_ATTN_BM")) a.bm = atoi(e) > 128 ? 256 : 128;
+    a.nb = a.bm / a.G;
     a.rb_count = (a.max_nodes + a.nb - 1) / a.nb;
     // One CTA per SM (shared memory), clusters must be co-resident: take the
     // widest even split whose clusters all fit on the GPU at once, so the
@@ -162,7 +168,7 @@ void choose_attention_shape(pf::AttnArgs& a, int max_prefix_len, int sms) {
     int splits = std::min(16, max_tiles);
     if (splits > 1) splits &= ~1;
     for (; splits > 1; splits -= 2)
-      if (tc_max_active_clusters(splits) >= groups) break;
+      if (tc_max_active_clusters(splits, a.bm) >= groups) break;
     if (const char* e = getenv("PF_ATTN_SPLITS")) splits = std::max(1, std::min(16, atoi(e)));
     a.splits = std::max(1, splits);
     return;

@@ -1,22 +1,27 @@
 // Tree-masked GQA attention on the 5th-generation tensor cores (tcgen05).
 // Same contract and work split as the mma.sync kernel in attention.cu (one
-// CTA = 128 query rows of one KV head x a slice of the 64-token KV tiles,
-// clusters merge the slices); the arithmetic moves to UMMA with TMEM
+// CTA = a block of query rows of one KV head x a slice of the 64-token KV
+// tiles, clusters merge the slices); the arithmetic moves to UMMA with TMEM
 // accumulators:
 //
 //   warp 0     TMA producer: Q once, then K/V tiles into a 3-stage ring
-//   warp 1     TMEM owner and MMA issuer (one thread):
-//                S_i  = Q K_i^T      M=128, N=64, K=D   -> TMEM S[i % 2]
-//                O   += P_i V_i      M=128, N=D,  K=64  -> TMEM O
-//              issued in the order S_0 S_1 PV_0 S_2 PV_1 ... so the tensor
-//              core computes S_{i+1} while the softmax warps work on S_i
-//   warps 2-5  one query row per thread (its TMEM lane): read S_i, mask
-//              (prefix length / ancestor bits), online softmax in the exp2
-//              domain, write P_i as bf16 into shared memory (K-major,
-//              128-byte swizzle); the running maximum is only moved (and O
-//              rescaled in TMEM) when it grows by more than 2^8, so the
-//              common case never touches O; at the end they read O back
-//              and publish (m, l, O) for the cluster merge.
+//   warp 1     TMEM owner and MMA issuer (one thread), per row block w:
+//                S_w,i = Q_w K_i^T    M=128, N=64, K=D   -> TMEM S_w[i % 2]
+//                O_w  += P_w,i V_i    M=128, N=D,  K=64  -> TMEM O_w
+//              issued as their inputs become ready, so the tensor core
+//              computes S_{i+1} while the softmax warps work on S_i
+//   softmax    one warpgroup per 128-row block, one query row per thread
+//              (its TMEM lane): read S, mask (prefix length / ancestor
+//              bits), online softmax in the exp2 domain, write P as bf16
+//              into shared memory (K-major, 128-byte swizzle); the running
+//              maximum is only moved (and O rescaled in TMEM) when it grows
+//              by more than 2^8, so the common case never touches O; at the
+//              end they read O back and publish (m, l, O) for the merge.
+//
+// kWG = 1 (128 rows, 192 threads) serves problems of at most 128 rows per
+// KV head; kWG = 2 (256 rows, 320 threads: two softmax warpgroups, 512
+// TMEM columns) larger ones: each K/V tile then serves twice the rows and
+// two warps share every scheduler during the softmax.
 //
 // V is the B operand of PV in its natural token-major layout (an MN-major
 // UMMA operand), so no transpose is needed anywhere.
@@ -31,42 +36,57 @@ namespace pf {
 namespace {
 
 constexpr int kTcStages = 3;
-constexpr int kTcThreads = 192;
 constexpr float kRescaleLog2 = 8.f;   // move the reference max when it grows by > 2^8
-constexpr uint32_t kTmemCols = 256;   // S[0] 0..63, S[1] 64..127, O 128..128+D-1
 
-template <int D>
+template <int WG>
+struct TcShape {
+  static constexpr int kThreads = 64 + 128 * WG;      // producer, MMA, softmax warpgroups
+  static constexpr uint32_t kTmemCols = 256 * WG;     // per block: S[0] 0..63, S[1] 64..127, O
+};
+
+template <int D, int WG>
 struct TcSmem {
   static constexpr int kHalves = D / 64;
+  static constexpr int kRows = 128 * WG;
   static constexpr int kTileBytes = kBN * D * 2;         // one K or V tile
   static constexpr int kStageBytes = 2 * kTileBytes;     // K + V
-  static constexpr int kQBytes = 128 * D * 2;
-  static constexpr int kPBytes = 128 * kBN * 2;          // one P tile (bf16)
+  static constexpr int kQBytes = kRows * D * 2;
+  static constexpr int kPBytes = 128 * kBN * 2;          // one P tile (bf16) of one block
   static constexpr int kQOff = kTcStages * kStageBytes;
   static constexpr int kPOff = kQOff + kQBytes;
+  static constexpr int kPEnd = kPOff + 2 * WG * kPBytes;
   // Merge inbox: one slot per (split, row) a CTA may receive, at most
-  // splits * ceil(rows / splits) <= 128 + 15 slots.  A slot holds the
+  // splits * ceil(rows / splits) <= rows + 15 slots.  A slot holds the
   // normalised partial O / l in fp16 (D halves) followed by its log2-sum-exp
   // (one float) in the 16-byte pad; the same format is staged locally.
-  static constexpr int kInboxSlots = 144;
+  // kWG = 1: the inbox has its own space (peers may send while this CTA is
+  // still working) and rows are staged in the idle K/V ring.  kWG = 2: no
+  // room; the inbox takes the K/V ring and rows are staged over Q and P,
+  // and peers send only after every CTA of the cluster has left its loop.
+  static constexpr int kInboxSlots = kRows + 16;
   static constexpr int kInboxPitch = D + 8;              // halves
-  static constexpr int kInboxOff = kPOff + 2 * kPBytes;
-  static constexpr int kLseOff = kInboxOff + kInboxSlots * kInboxPitch * 2;
-  static constexpr int kBarOff = kLseOff + kInboxSlots * 4;
-  // kv_full[3] kv_empty[3] q_full s_full[2] s_empty[2] p_full[2] pv_done[2] inbox
-  static constexpr int kNumBars = 2 * kTcStages + 10;
+  static constexpr int kRowBytes = kInboxPitch * 2;
+  static constexpr int kStageOff = WG == 1 ? 0 : kQOff;
+  static constexpr int kInboxOff = WG == 1 ? kPEnd : 0;
+  static constexpr int kBarOff = WG == 1 ? kInboxOff + kInboxSlots * kRowBytes : kPEnd;
+  static_assert(kRows * kRowBytes <= (WG == 1 ? kQOff : kPEnd - kQOff), "staged rows fit");
+  static_assert(WG == 1 || kInboxSlots * kRowBytes <= kQOff, "inbox fits in the ring");
+  // kv_full[3] kv_empty[3] q_full, per block s_full[2] s_empty[2] p_full[2] pv_done[2], inbox
+  static constexpr int kNumBars = 2 * kTcStages + 1 + 8 * WG + 1;
   static constexpr int kTotal = kBarOff + kNumBars * 8 + 16;
   static_assert(kTotal + 1024 <= 232448, "shared memory budget");
 };
 
-template <int D>
-__global__ void __launch_bounds__(kTcThreads, 1)
+template <int D, int WG>
+__global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
                    const __grid_constant__ CUtensorMap tm_tk,
                    const __grid_constant__ CUtensorMap tm_tv,
                    const __grid_constant__ CUtensorMap tm_ck,
                    const __grid_constant__ CUtensorMap tm_cv, const AttnArgs a) {
-  using S = TcSmem<D>;
+  using S = TcSmem<D, WG>;
+  constexpr int kThreads = TcShape<WG>::kThreads;
+  constexpr uint32_t kTmemCols = TcShape<WG>::kTmemCols;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   uint8_t* sKV = smem;
@@ -77,11 +97,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   uint64_t* kv_full = bars;
   uint64_t* kv_empty = bars + kTcStages;
   uint64_t* q_full = bars + 2 * kTcStages;
-  uint64_t* s_full = q_full + 1;
-  uint64_t* s_empty = s_full + 2;
-  uint64_t* p_full = s_empty + 2;
-  uint64_t* pv_done = p_full + 2;
-  uint64_t* inbox_full = pv_done + 2;
+  // per row block w: s_full[2] s_empty[2] p_full[2] pv_done[2] at blk + 8 w
+  uint64_t* blk = q_full + 1;
+  uint64_t* inbox_full = blk + 8 * WG;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + S::kNumBars);
 
   cg::cluster_group cluster = cg::this_cluster();
@@ -112,6 +130,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const int nfirst = rb * a.nb;
   if (nfirst >= nn) return;  // uniform over the cluster (same b, g, rb)
   const int rows = min(a.nb, nn - nfirst) * a.G;
+  const int nblk = WG == 1 ? 1 : (rows > 128 ? 2 : 1);  // row blocks with work
   const int n_ptiles = (P + kBN - 1) / kBN;
   const int ntiles = n_ptiles + (nn + kBN - 1) / kBN;
   const int t_begin = (int)((long long)ntiles * split / nsplit);
@@ -121,15 +140,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   if (tid == 0) {
     for (int i = 0; i < kTcStages; ++i) {
       mbar_init(smem_u32(&kv_full[i]), 1);
-      mbar_init(smem_u32(&kv_empty[i]), 1);
+      mbar_init(smem_u32(&kv_empty[i]), (uint32_t)nblk);  // one PV per active block
     }
     mbar_init(smem_u32(q_full), 1);
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(smem_u32(&s_full[i]), 1);
-      mbar_init(smem_u32(&s_empty[i]), 128);
-      mbar_init(smem_u32(&p_full[i]), 128);
-      mbar_init(smem_u32(&pv_done[i]), 1);
-    }
+    for (int w = 0; w < WG; ++w)
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(smem_u32(&blk[8 * w + i]), 1);          // s_full
+        mbar_init(smem_u32(&blk[8 * w + 2 + i]), 128);    // s_empty
+        mbar_init(smem_u32(&blk[8 * w + 4 + i]), 128);    // p_full
+        mbar_init(smem_u32(&blk[8 * w + 6 + i]), 1);      // pv_done
+      }
     mbar_init(smem_u32(inbox_full), 1);
     fence_mbar_init();
     for (int i = 0; i < first; ++i)
@@ -142,7 +162,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     mbar_arrive_expect_tx(smem_u32(q_full), S::kHalves * a.G * a.nb * 128);
 #pragma unroll
     for (int h = 0; h < S::kHalves; ++h)
-      tma_load_3d(smem_u32(sQ + h * 128 * 128), &tm_q, h * 64, g * a.G, node0 + nfirst,
+      tma_load_3d(smem_u32(sQ + h * S::kRows * 128), &tm_q, h * 64, g * a.G, node0 + nfirst,
                   smem_u32(q_full));
     for (int i = 0; i < first; ++i)
       if (t_begin + i >= n_ptiles)
@@ -157,15 +177,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  // Peers may signal this CTA's inbox barrier only after it is initialised:
-  // arrive now, wait just before sending partials.  (A single split is
-  // launched without a cluster and uses no cluster feature at all.)
-  if (nsplit > 1) cluster_arrive_release();
+  // kWG = 1: peers may signal this CTA's inbox barrier once it is
+  // initialised: arrive now, wait just before sending partials.  (A single
+  // split is launched without a cluster and uses no cluster feature.)
+  if (WG == 1 && nsplit > 1) cluster_arrive_release();
   pdl_launch_dependents();
 
   float m_ref = -INFINITY, l = 0.f;   // softmax threads: running max (log2) and sum of their row
+  const int wg = warp >= 2 ? (warp - 2) >> 2 : 0;   // softmax: this thread's row block
   if (warp == 0) {
-    // ---------------- producer: refill the ring as PV releases stages
+    // ---------------- producer: refill the ring as the PVs release stages
     if (lane == 0) {
       for (int i = kTcStages; i < my_tiles; ++i) {
         const int st = i % kTcStages;
@@ -181,56 +202,67 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       const uint32_t id_o = umma_idesc_bf16_bmn(128, D);
       bool ok = mbar_wait(smem_u32(q_full), 0, a.err);
       const uint32_t q0 = smem_u32(sQ);
-      // Event-driven issue: S_n as soon as its K/V tile has landed and the
-      // softmax has read S_{n-2} out of the same TMEM buffer; PV_j as soon
-      // as P_j is in shared memory.  S_{n+1} thus never waits behind P_{n-1}
-      // and is computed while the softmax still works on S_{n-1}, S_n.
-      int ns = 0, np = 0;
+      // Event-driven issue, per row block w: S_n as soon as its K/V tile
+      // has landed and the softmax has read S_{n-2} out of the same TMEM
+      // buffer; PV_j as soon as P_j is in shared memory.  S_{n+1} thus
+      // never waits behind P_{n-1}.
+      int ns[WG], np[WG];
+#pragma unroll
+      for (int w = 0; w < WG; ++w) ns[w] = np[w] = 0;
       unsigned idle = 0;
       unsigned long long t0 = 0;
-      while (ok && np < my_tiles) {
-        bool progressed = false;
-        if (ns < my_tiles) {
-          const int st = ns % kTcStages, sb = ns & 1;
-          if (mbar_test_wait(smem_u32(&kv_full[st]), (ns / kTcStages) & 1) &&
-              mbar_test_wait(smem_u32(&s_empty[sb]), ((ns >> 1) & 1) ^ 1)) {
-            tc_fence_after();
-            const uint32_t k0 = smem_u32(sKV + st * S::kStageBytes);
+      while (ok) {
+        bool progressed = false, done = true;
 #pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t qa = q0 + (kk >> 2) * (128 * 128) + (kk & 3) * 32;
-              const uint32_t kb = k0 + (kk >> 2) * (kBN * 128) + (kk & 3) * 32;
-              umma_bf16(tmem + sb * kBN, umma_desc_sw128(qa), umma_desc_sw128(kb), id_s, kk > 0);
+        for (int w = 0; w < WG; ++w) {
+          if (w >= nblk) continue;
+          uint64_t* bw = blk + 8 * w;
+          const uint32_t tw = tmem + (uint32_t)(w * 256);
+          if (ns[w] < my_tiles) {
+            const int n = ns[w], st = n % kTcStages, sb = n & 1;
+            if (mbar_test_wait(smem_u32(&kv_full[st]), (n / kTcStages) & 1) &&
+                mbar_test_wait(smem_u32(&bw[2 + sb]), ((n >> 1) & 1) ^ 1)) {
+              tc_fence_after();
+              const uint32_t k0 = smem_u32(sKV + st * S::kStageBytes);
+#pragma unroll
+              for (int kk = 0; kk < D / 16; ++kk) {
+                const uint32_t qa =
+                    q0 + (kk >> 2) * (S::kRows * 128) + w * (128 * 128) + (kk & 3) * 32;
+                const uint32_t kb = k0 + (kk >> 2) * (kBN * 128) + (kk & 3) * 32;
+                umma_bf16(tw + sb * kBN, umma_desc_sw128(qa), umma_desc_sw128(kb), id_s, kk > 0);
+              }
+              umma_commit(smem_u32(&bw[sb]));
+              ++ns[w];
+              progressed = true;
             }
-            umma_commit(smem_u32(&s_full[sb]));
-            ++ns;
-            progressed = true;
           }
-        }
-        if (np < ns) {
-          const int pb = np & 1, stj = np % kTcStages;
-          if (mbar_test_wait(smem_u32(&p_full[pb]), (np >> 1) & 1)) {
-            tc_fence_after();
-            const uint32_t p0 = smem_u32(sP + pb * S::kPBytes);
-            const uint32_t v0 = smem_u32(sKV + stj * S::kStageBytes + S::kTileBytes);
+          if (np[w] < ns[w]) {
+            const int j = np[w], pb = j & 1, stj = j % kTcStages;
+            if (mbar_test_wait(smem_u32(&bw[4 + pb]), (j >> 1) & 1)) {
+              tc_fence_after();
+              const uint32_t p0 = smem_u32(sP + (2 * w + pb) * S::kPBytes);
+              const uint32_t v0 = smem_u32(sKV + stj * S::kStageBytes + S::kTileBytes);
 #pragma unroll
-            for (int kt = 0; kt < kBN / 16; ++kt)
-              umma_bf16(tmem + 2 * kBN, umma_desc_sw128(p0 + kt * 32),
-                        umma_desc_sw128_lbo(v0 + kt * 16 * 128, kBN * 128, 1024), id_o,
-                        (np > 0 || kt > 0) ? 1u : 0u);
-            umma_commit(smem_u32(&pv_done[pb]));
-            umma_commit(smem_u32(&kv_empty[stj]));
-            ++np;
-            progressed = true;
+              for (int kt = 0; kt < kBN / 16; ++kt)
+                umma_bf16(tw + 2 * kBN, umma_desc_sw128(p0 + kt * 32),
+                          umma_desc_sw128_lbo(v0 + kt * 16 * 128, kBN * 128, 1024), id_o,
+                          (j > 0 || kt > 0) ? 1u : 0u);
+              umma_commit(smem_u32(&bw[6 + pb]));
+              umma_commit(smem_u32(&kv_empty[stj]));
+              ++np[w];
+              progressed = true;
+            }
           }
+          if (np[w] < my_tiles) done = false;
         }
+        if (done) break;
         // bounded like mbar_wait: give up (and flag) after kWaitLimitNs
         // without progress
         if (progressed) {
           idle = 0;
         } else if ((++idle & 63u) == 0u) {
           const unsigned long long now = globaltimer();
-          if (t0 == 0 || idle == 64u) t0 = now;
+          if (idle == 64u) t0 = now;
           if (now - t0 > kWaitLimitNs) {
             flag_error(a.err, PF_DEVERR_TIMEOUT);
             ok = false;
@@ -238,10 +270,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
       }
     }
-  } else {
-    // ---------------- softmax / correction / epilogue: one row per thread
+  } else if (wg < nblk) {
+    // ---------------- softmax / correction: one row per thread
+    uint64_t* bw = blk + 8 * wg;
+    const uint32_t tw = tmem + (uint32_t)(wg * 256);
     const int quad = warp & 3;
-    const int r = quad * 32 + lane;
+    const int rl = quad * 32 + lane;       // row within the block (its TMEM lane)
+    const int r = wg * 128 + rl;           // row within the CTA
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
     uint64_t mk0 = 0, mk1 = 0;
     if (r < rows) {
@@ -253,15 +288,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     for (int i = 0; i < my_tiles && ok; ++i) {
       const int sb = i & 1;
       const int st = i % kTcStages;
-      ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&s_full[sb]), (i >> 1) & 1, a.err));
+      ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&bw[sb]), (i >> 1) & 1, a.err));
       if (!ok) break;  // warp-uniform
       tc_fence_after();
       uint32_t lo[32], hi[32];
-      tmem_ld_32(tmem + lane_base + sb * kBN, lo);
-      tmem_ld_32(tmem + lane_base + sb * kBN + 32, hi);
+      tmem_ld_32(tw + lane_base + sb * kBN, lo);
+      tmem_ld_32(tw + lane_base + sb * kBN + 32, hi);
       tmem_ld_wait();
       tc_fence_before();
-      mbar_arrive(smem_u32(&s_empty[sb]));
+      mbar_arrive(smem_u32(&bw[2 + sb]));
 
       const int t = t_begin + i;
       const bool is_prefix = t < n_ptiles;
@@ -296,17 +331,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       if (m_ref == -INFINITY) m_ref = m_new;
       if (__any_sync(0xffffffffu, resc)) {
         // O must hold exactly the tiles before i: wait for PV_{i-1}.
-        if (i >= 1) mbar_wait(smem_u32(&pv_done[(i - 1) & 1]), ((i - 1) >> 1) & 1, a.err);
+        if (i >= 1) mbar_wait(smem_u32(&bw[6 + ((i - 1) & 1)]), ((i - 1) >> 1) & 1, a.err);
         tc_fence_after();
         const float alpha = resc ? ex2_approx(m_ref - m_new) : 1.f;
 #pragma unroll
         for (int c0 = 0; c0 < D; c0 += 32) {
           uint32_t ov[32];
-          tmem_ld_32(tmem + lane_base + 2 * kBN + c0, ov);
+          tmem_ld_32(tw + lane_base + 2 * kBN + c0, ov);
           tmem_ld_wait();
 #pragma unroll
           for (int c = 0; c < 32; ++c) ov[c] = __float_as_uint(__uint_as_float(ov[c]) * alpha);
-          tmem_st_32(tmem + lane_base + 2 * kBN + c0, ov);
+          tmem_st_32(tw + lane_base + 2 * kBN + c0, ov);
         }
         tmem_st_wait();
         if (resc) {
@@ -334,18 +369,19 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       f32x2_unpack(fadd2(fadd2(rs2[0], rs2[1]), fadd2(rs2[2], rs2[3])), r0, r1);
       l += r0 + r1;
       // P buffer sb was last read by PV_{i-2}.
-      if (i >= 2) mbar_wait(smem_u32(&pv_done[sb]), ((i - 2) >> 1) & 1, a.err);
-      uint8_t* prow = sP + sb * S::kPBytes + r * 128;
+      if (i >= 2) mbar_wait(smem_u32(&bw[6 + sb]), ((i - 2) >> 1) & 1, a.err);
+      uint8_t* prow = sP + (2 * wg + sb) * S::kPBytes + rl * 128;
 #pragma unroll
       for (int c = 0; c < 8; ++c)
-        *reinterpret_cast<uint4*>(prow + ((c ^ (r & 7)) << 4)) =
+        *reinterpret_cast<uint4*>(prow + ((c ^ (rl & 7)) << 4)) =
             make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
       if (valid < kBN) {
         // Cache rows past the prefix end may hold anything (even NaN bit
         // patterns): zero their V so masked columns contribute exactly 0.
+        // (With two blocks both write the same zeros before their PV.)
         uint8_t* sv = sKV + st * S::kStageBytes + S::kTileBytes;
         const int per_half = (kBN - valid) * 8;
-        for (int c = r; c < per_half * S::kHalves; c += 128) {
+        for (int c = rl; c < per_half * S::kHalves; c += 128) {
           const int h = c / per_half, rem = c % per_half;
           *reinterpret_cast<uint4*>(sv + h * kBN * 128 + (valid + rem / 8) * 128 + (rem % 8) * 16) =
               make_uint4(0, 0, 0, 0);
@@ -353,33 +389,36 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       }
       fence_proxy_async_smem();
       tc_fence_before();
-      mbar_arrive(smem_u32(&p_full[sb]));
+      mbar_arrive(smem_u32(&bw[4 + sb]));
     }
-    // O of this row is complete once the last PV has landed
+    // O of this row is complete once the block's last PV has landed
     if (my_tiles > 0)
-      mbar_wait(smem_u32(&pv_done[(my_tiles - 1) & 1]), ((my_tiles - 1) >> 1) & 1, a.err);
+      mbar_wait(smem_u32(&bw[6 + ((my_tiles - 1) & 1)]), ((my_tiles - 1) >> 1) & 1, a.err);
   }
   __syncwarp();  // the producer and MMA lanes rejoin their warps before the barriers
 
+  // ---- epilogue: each softmax thread reads its row of O / l from TMEM
+  const bool has_row = warp >= 2 && wg < nblk;
+  const int quad = warp & 3;
+  const int r = wg * 128 + quad * 32 + lane;
+  const uint32_t o_addr = tmem + (uint32_t)(wg * 256) + ((uint32_t)(quad * 32) << 16) + 2 * kBN;
+  const float inv_l = (my_tiles > 0 && l > 0.f) ? 1.f / l : 0.f;
+
   // ---- split-KV merge.  Each row's partial result, normalised (O / l,
   // fp16) with its log2-sum-exp lse = m + log2(l) in the row's pad, is
-  // staged in this CTA's (now idle) KV ring, row r at slot r, so the rows
-  // each peer merges are contiguous.  One bulk copy per peer moves them into
-  // the peer's inbox and completes on the peer's inbox barrier, which
-  // expects one block from every CTA of the cluster; the peer then merges
-  // from its own shared memory:
+  // staged in this CTA's shared memory, row r at slot r, so the rows each
+  // peer merges are contiguous.  One bulk copy per peer moves them into the
+  // peer's inbox and completes on the peer's inbox barrier, which expects
+  // one block from every CTA of the cluster; the peer then merges from its
+  // own shared memory:
   //   out = sum_s 2^(lse_s - M) (O/l)_s / sum_s 2^(lse_s - M),  M = max_s lse_s
   if (nsplit == 1) {
     // ---- single split: O / l is the output
-    if (warp >= 2) {
-      const int quad = warp & 3;
-      const int r = quad * 32 + lane;
-      const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
-      const float inv_l = (my_tiles > 0 && l > 0.f) ? 1.f / l : 0.f;
+    if (has_row) {
       uint32_t ov[D];
 #pragma unroll
       for (int c0 = 0; c0 < D; c0 += 32)
-        tmem_ld_32(tmem + lane_base + 2 * kBN + c0, *reinterpret_cast<uint32_t(*)[32]>(&ov[c0]));
+        tmem_ld_32(o_addr + c0, *reinterpret_cast<uint32_t(*)[32]>(&ov[c0]));
       tmem_ld_wait();
       if (r < rows) {
         const int node = node0 + nfirst + r / a.G;
@@ -406,19 +445,21 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   }
   const int per = (rows + nsplit - 1) / nsplit;
   const int cnt_mine = max(0, min(per, rows - split * per));
-  constexpr int kRowBytes = S::kInboxPitch * 2;
-  __half* stage_rows = reinterpret_cast<__half*>(sKV);
+  __half* stage_rows = reinterpret_cast<__half*>(smem + S::kStageOff);
+  if (WG == 2) {
+    // The rows are staged over Q and P: every block's last PV must have
+    // completed (each softmax warpgroup waited for its own) -- and the ring
+    // is idle, so peers may now fill the inbox it holds.
+    __syncthreads();
+    cluster_arrive_release();
+  }
   if (tid == 0)
-    mbar_arrive_expect_tx(smem_u32(inbox_full), (uint32_t)(nsplit * cnt_mine * kRowBytes));
-  if (warp >= 2) {
-    const int quad = warp & 3;
-    const int r = quad * 32 + lane;
-    const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
-    const float inv_l = (my_tiles > 0 && l > 0.f) ? 1.f / l : 0.f;
+    mbar_arrive_expect_tx(smem_u32(inbox_full), (uint32_t)(nsplit * cnt_mine * S::kRowBytes));
+  if (has_row) {
     uint32_t ov[D];  // the whole O row: all TMEM loads in flight behind one wait
 #pragma unroll
     for (int c0 = 0; c0 < D; c0 += 32)
-      tmem_ld_32(tmem + lane_base + 2 * kBN + c0, *reinterpret_cast<uint32_t(*)[32]>(&ov[c0]));
+      tmem_ld_32(o_addr + c0, *reinterpret_cast<uint32_t(*)[32]>(&ov[c0]));
     tmem_ld_wait();
     if (r < rows) {
       __half* dst = stage_rows + r * S::kInboxPitch;
@@ -437,14 +478,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   fence_proxy_async_smem();  // staged rows are read by the bulk-copy engine
   tc_fence_before();
   __syncthreads();
-  cluster_wait_acquire();    // every peer's inbox barrier is initialised
+  cluster_wait_acquire();    // every peer's inbox is ready to be filled
   if (tid < nsplit) {
     const int q = tid;
     const int cnt = min(per, rows - q * per);
     if (cnt > 0) {
       const uint32_t src = smem_u32(stage_rows + q * per * S::kInboxPitch);
       const uint32_t dst = mapa_cluster(smem_u32(sInbox + split * per * S::kInboxPitch), q);
-      bulk_copy_s2cluster(dst, src, (uint32_t)(cnt * kRowBytes),
+      bulk_copy_s2cluster(dst, src, (uint32_t)(cnt * S::kRowBytes),
                           mapa_cluster(smem_u32(inbox_full), q));
       bulk_commit_group();
     }
@@ -454,27 +495,34 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tmem_dealloc(tmem, kTmemCols);
   }
   if (cnt_mine > 0) mbar_wait(smem_u32(inbox_full), 0, a.err);
-  inbox_merge<D, kTcThreads, S::kInboxPitch>(a, sInbox, rows, split, per, nsplit, node0 + nfirst,
-                                             g, tid);
+  inbox_merge<D, kThreads, S::kInboxPitch>(a, sInbox, rows, split, per, nsplit, node0 + nfirst,
+                                           g, tid);
   // this CTA's staged rows must stay readable until its copies have left
   if (tid < nsplit) bulk_wait_read_all();
 }
 
 }  // namespace
 
-int attention_tc_smem_bytes() { return TcSmem<128>::kTotal + 1024; }
+template <int WG>
+static int tc_smem_bytes() {
+  return TcSmem<128, WG>::kTotal + 1024;
+}
 
-int attention_tc_max_active_clusters(int cluster) {
-  const int smem = TcSmem<128>::kTotal + 1024;
+int attention_tc_smem_bytes() { return tc_smem_bytes<1>(); }
+
+template <int WG>
+static int tc_max_active_clusters_impl(int cluster) {
+  const int smem = tc_smem_bytes<WG>();
   static int limit[64] = {};
-  if (ensure_smem_limit((const void*)attn_tc_kernel<128>, smem, limit) != cudaSuccess) return 0;
-  if (cluster > 8 && cudaFuncSetAttribute(attn_tc_kernel<128>,
+  if (ensure_smem_limit((const void*)attn_tc_kernel<128, WG>, smem, limit) != cudaSuccess)
+    return 0;
+  if (cluster > 8 && cudaFuncSetAttribute(attn_tc_kernel<128, WG>,
                                           cudaFuncAttributeNonPortableClusterSizeAllowed,
                                           1) != cudaSuccess)
     return 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(cluster);
-  cfg.blockDim = dim3(kTcThreads);
+  cfg.blockDim = dim3(TcShape<WG>::kThreads);
   cfg.dynamicSmemBytes = smem;
   cudaLaunchAttribute attr;
   attr.id = cudaLaunchAttributeClusterDimension;
@@ -484,30 +532,40 @@ int attention_tc_max_active_clusters(int cluster) {
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<128>, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<128, WG>, &cfg) != cudaSuccess) {
     cudaGetLastError();
     return 0;
   }
   return n;
 }
 
-cudaError_t launch_attention_tc(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl) {
-  const int smem = TcSmem<128>::kTotal + 1024;
+int attention_tc_max_active_clusters(int cluster, int rows_per_cta) {
+  return rows_per_cta > 128 ? tc_max_active_clusters_impl<2>(cluster)
+                            : tc_max_active_clusters_impl<1>(cluster);
+}
+
+template <int WG>
+static cudaError_t launch_tc(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl) {
+  const int smem = tc_smem_bytes<WG>();
   static int limit[64] = {};
   static bool nonportable[64] = {};
-  cudaError_t e = ensure_smem_limit((const void*)attn_tc_kernel<128>, smem, limit);
+  cudaError_t e = ensure_smem_limit((const void*)attn_tc_kernel<128, WG>, smem, limit);
   if (e != cudaSuccess) return e;
   int dev = 0;
   cudaGetDevice(&dev);
   if (a.splits > 8 && dev >= 0 && dev < 64 && !nonportable[dev]) {
-    e = cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeNonPortableClusterSizeAllowed,
-                             1);
+    e = cudaFuncSetAttribute(attn_tc_kernel<128, WG>,
+                             cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
     nonportable[dev] = true;
   }
   const dim3 grid(a.B * a.Hkv * a.rb_count * a.splits);
-  return launch_ex(attn_tc_kernel<128>, grid, dim3(kTcThreads), smem, s, a.splits, pdl, m.q, m.tk,
-                   m.tv, m.ck, m.cv, a);
+  return launch_ex(attn_tc_kernel<128, WG>, grid, dim3(TcShape<WG>::kThreads), smem, s, a.splits,
+                   pdl, m.q, m.tk, m.tv, m.ck, m.cv, a);
+}
+
+cudaError_t launch_attention_tc(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl) {
+  return a.bm > 128 ? launch_tc<2>(a, m, s, pdl) : launch_tc<1>(a, m, s, pdl);
 }
 
 }  // namespace pf

@@ -52,10 +52,11 @@ int attention_bf16_smem_bytes(int D, int bm);
 // Whether a cluster of `cluster` CTAs of the bf16 attention kernel can be
 // resident at once on this device.
 bool attention_cluster_fits(int D, int bm, int cluster);
-// tcgen05 variant (bf16, D = 128, 128 query rows per CTA).
+// tcgen05 variant (bf16, D = 128, a.bm = 128 or 256 query rows per CTA).
 cudaError_t launch_attention_tc(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl);
 // How many clusters of `cluster` CTAs of the tcgen05 kernel fit at once.
-int attention_tc_max_active_clusters(int cluster);
+// rows_per_cta: 128 (one softmax warpgroup) or 256 (two).
+int attention_tc_max_active_clusters(int cluster, int rows_per_cta);
 int attention_tc_smem_bytes();
 
 // ------------------------------------------------------------ LM head

@@ -66,6 +66,10 @@ EDGE = {
     # 256 LM-head rows (2 x 128 nodes), paged
     "256-rows-paged": I.scaled(W["7b-bf16-batch8-paged"], layers=1, batch=2, prefix=(33, 300),
                                nodes=128, vocab=1000, hidden=192),
+    # 192 rows of one KV head (two 128-row blocks in one CTA), one KV tile
+    # (no split): the direct epilogue of the two-block kernel
+    "two-blocks-one-tile": I.scaled(W["7b-bf16-tree64"], layers=1, hq=32, hkv=2, prefix=(0, 0),
+                                    nodes=12, max_depth=5, vocab=300, hidden=64),
     # fp32 paged tree
     "f32-paged-tree": I.scaled(W["7b-bf16-batch8-paged"], dtype="f32", layers=2, batch=3,
                                hq=8, hkv=2, d=32, prefix=(5, 90), nodes=12, vocab=300,
@@ -92,6 +96,19 @@ def test_mma_sync_kernel(name, monkeypatch):
     correct at D = 128, where the tcgen05 kernel is the default."""
     monkeypatch.setenv("PF_ATTN_IMPL", "mma")
     c = Case(SMALL[name], seed=6)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for s in range(c.w.batch):
+        c.check_attention(0, s)
+
+
+@pytest.mark.parametrize("name", ["7b-tree64-small", "7b-32k-tree128-small"])
+def test_two_block_kernel_on_many_rows(name, monkeypatch):
+    """Two 128-row blocks per CTA (PF_ATTN_BM=256) where a KV head has more
+    than 256 rows, so several two-block CTAs share a head."""
+    monkeypatch.setenv("PF_ATTN_BM", "256")
+    c = Case(SMALL[name], seed=8)
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0

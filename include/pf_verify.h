@@ -389,6 +389,18 @@ typedef struct pf_prefix_desc {
 PF_API pf_status pf_prefix_match(const pf_prefix_desc* d, void* stream);
 
 /*
+ * pf_selftest_wait -- exercises the failure path shared by every kernel's
+ * waits (no counterpart in the paper).  One GPU thread waits on an
+ * mbarrier with the library's bounded wait, limited to limit_ns (1e3 ..
+ * 5e9).  signal = 0: nothing arrives, so the wait runs out, ORs
+ * PF_DEVERR_TIMEOUT into *error_flag and the kernel returns normally (the
+ * context stays usable); signal = 1: the barrier completes at once.
+ * waited_ok (device int32) receives 1 if the wait completed, else 0.
+ */
+PF_API pf_status pf_selftest_wait(int32_t* error_flag, int64_t limit_ns, int32_t signal,
+                                  int32_t* waited_ok, void* stream);
+
+/*
  * Proposal-length controller (Section 3.2 "Runtime-adaptive
  * proposal-length controller", eq. 1).  Host code: no GPU, no allocation.
  *

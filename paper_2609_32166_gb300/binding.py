@@ -168,6 +168,8 @@ def lib() -> C.CDLL:
     L.pf_length_select.restype = C.c_int
     L.pf_length_select.argtypes = [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32,
                                    C.POINTER(C.c_int32), C.POINTER(C.c_double)]
+    L.pf_selftest_wait.restype = C.c_int
+    L.pf_selftest_wait.argtypes = [C.c_void_p, C.c_int64, C.c_int32, C.c_void_p, C.c_void_p]
     L.pf_prefix_match.restype = C.c_int
     L.pf_prefix_match.argtypes = [C.POINTER(pf_prefix_desc), C.c_void_p]
     _lib = L
@@ -280,3 +282,9 @@ def pf_length_select(t_hat, p_first, p_cont) -> tuple:
     _check(lib().pf_length_select(t.ctypes.data, p1.ctypes.data, pc.ctypes.data,
                                   int(t.shape[0]) - 1, C.byref(ell), C.byref(obj)))
     return int(ell.value), float(obj.value)
+
+
+def pf_selftest_wait(error_flag: int, limit_ns: int, signal: bool, waited_ok: int,
+                     stream: int = 0) -> None:
+    _check(lib().pf_selftest_wait(C.c_void_p(error_flag), int(limit_ns), 1 if signal else 0,
+                                  C.c_void_p(waited_ok), C.c_void_p(stream)))

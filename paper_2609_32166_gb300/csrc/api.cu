@@ -610,6 +610,18 @@ pf_status pf_retrieve(const pf_retrieval_desc* d, void* workspace, size_t worksp
   return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
 }
 
+pf_status pf_selftest_wait(int32_t* error_flag, int64_t limit_ns, int32_t signal,
+                           int32_t* waited_ok, void* stream) {
+  static const char* who = "pf_selftest_wait";
+  if (!error_flag || !waited_ok) return fail(PF_ERR_NULL, "%s: a required pointer is NULL", who);
+  if (limit_ns < 1000 || limit_ns > 5000000000LL)
+    return fail(PF_ERR_SHAPE, "%s: limit_ns must be in [1e3, 5e9]", who);
+  if (num_sms() <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
+  cudaError_t e = pf::launch_selftest_wait(error_flag, (unsigned long long)limit_ns, signal ? 1 : 0,
+                                           waited_ok, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
+}
+
 pf_status pf_prefix_match(const pf_prefix_desc* d, void* stream) {
   static const char* who = "pf_prefix_match";
   if (!d) return fail(PF_ERR_NULL, "%s: desc is NULL", who);

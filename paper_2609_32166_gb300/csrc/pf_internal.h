@@ -183,6 +183,9 @@ struct PrefixArgs {
 
 cudaError_t launch_prefix_match(const PrefixArgs& a, cudaStream_t s, bool pdl);
 
+cudaError_t launch_selftest_wait(int32_t* err, unsigned long long limit_ns, int signal,
+                                 int32_t* waited_ok, cudaStream_t s);
+
 // Record the message pf_last_error() returns on this thread; returns s.
 pf_status set_error(pf_status s, const char* fmt, ...);
 

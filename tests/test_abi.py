@@ -23,7 +23,8 @@ def test_exports_every_declared_symbol():
                           "pf_lmhead_accept_workspace_size", "pf_kv_commit", "pf_last_error",
                           "pf_version", "pf_kv_shift", "pf_retrieval_key", "pf_retrieve",
                           "pf_retrieval_workspace_size", "pf_lmhead_accept_noalloc",
-                          "pf_prefix_match"}
+                          "pf_prefix_match", "pf_selftest_wait", "pf_controller_init",
+                          "pf_controller_observe", "pf_controller_choose", "pf_length_select"}
     L = pb.lib()
     for n in names:
         assert hasattr(L, n), n

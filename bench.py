@@ -820,17 +820,20 @@ def run_ell_sweep(args):
 
 
 def run_e2e(vs, w, batch, K, stream, flush, world, tok_table, planned):
-    """Same metric through host buffers: every step copies its inputs from
-    pinned host memory, runs the step and reads the accepted tokens back."""
+    """Same metric through host buffers: every step copies its inputs (the
+    queries, proposal K/V of every layer, hidden states, tokens, tree and
+    lengths: one packed arena) from pinned host memory, runs the step and
+    reads its outputs (accepted lengths, tokens, new lengths: one arena)
+    back."""
     import torch
-    names = ["q", "tree_k", "tree_v", "hidden", "tokens", "parent", "mask", "cu_nodes",
-             "prefix_len"]
-    host = {n: getattr(vs, n).detach().cpu().pin_memory() for n in names}
-    host_tokens = [t.cpu().pin_memory() for t in tok_table]
-    outs = {n: torch.empty_like(getattr(vs, n), device="cpu").pin_memory()
-            for n in ("accept_len", "out_tokens", "new_len")}
-    h2d = sum(t.numel() * t.element_size() for t in host.values())
-    d2h = sum(t.numel() * t.element_size() for t in outs.values())
+    host_in = vs.in_arena.detach().cpu().pin_memory()
+    host_out = torch.empty(vs.out_arena.numel(), dtype=torch.uint8).pin_memory()
+    tok_off = vs.tokens.data_ptr() - vs.in_arena.data_ptr()
+    tok_bytes = vs.tokens.numel() * vs.tokens.element_size()
+    host_tokens = [t.cpu().contiguous().view(torch.uint8) for t in tok_table]
+    acc_off = vs.accept_len.data_ptr() - vs.out_arena.data_ptr()
+    h2d = host_in.numel()
+    d2h = host_out.numel()
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g, stream=stream):
         vs.step(torch.cuda.current_stream().cuda_stream)
@@ -845,23 +848,22 @@ def run_e2e(vs, w, batch, K, stream, flush, world, tok_table, planned):
     with torch.cuda.stream(stream):
         for k in range(n):
             flush.zero_()
-            host["tokens"] = host_tokens[k % len(host_tokens)]
+            host_in[tok_off:tok_off + tok_bytes].copy_(host_tokens[k % len(host_tokens)])
             e0.record(stream)
-            for name, t in host.items():
-                getattr(vs, name).copy_(t, non_blocking=True)
+            vs.in_arena.copy_(host_in, non_blocking=True)
             g.replay()
-            for name, t in outs.items():
-                t.copy_(getattr(vs, name), non_blocking=True)
+            host_out.copy_(vs.out_arena, non_blocking=True)
             e1.record(stream)
             stream.synchronize()
             times.append(e0.elapsed_time(e1))
-            got = int((outs["accept_len"] + 1).sum())
+            acc = host_out[acc_off:acc_off + 4 * w.batch].view(torch.int32)
+            got = int((acc + 1).sum())
             assert got == planned[k % len(planned)]
             tok += got
     t = max_over_ranks(float(np.sum(times)), world, "cuda")
     return {"value": whole_job_rate(tok, t * 1e-3, world), "unit": "tokens/s",
-            "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h, "steps": n, "ms_per_step": t / n}
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n, "ms_per_step": t / n,
+            "copies_per_step": {"h2d": 1, "d2h": 1}}
 
 
 if __name__ == "__main__":

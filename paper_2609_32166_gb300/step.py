@@ -110,7 +110,31 @@ class VerifyStep:
         self.err = torch.zeros((1,), **i32)
         self.ws_bytes = pb.pf_lmhead_accept_workspace_size()
         self.workspace = torch.zeros((self.ws_bytes,), dtype=torch.uint8, device=device)
+        # A step's inputs and outputs each live in one contiguous arena (the
+        # tensors above become views of it), so that a host round trip is
+        # one copy each way.
+        self.in_arena = self._arena(("q", "tree_k", "tree_v", "hidden", "tokens", "parent",
+                                     "mask", "cu_nodes", "prefix_len"), device)
+        self.out_arena = self._arena(("accept_len", "out_tokens", "new_len"), device)
         self._build_descs()
+
+    def _arena(self, names, device) -> torch.Tensor:
+        """Move the named tensors into one 256-byte-aligned byte arena and
+        replace each by a view of it; returns the arena."""
+        layout, total = [], 0
+        for n in names:
+            t = getattr(self, n)
+            total = (total + 255) // 256 * 256
+            nbytes = t.numel() * t.element_size()
+            layout.append((n, total, nbytes))
+            total += nbytes
+        arena = torch.empty(total, dtype=torch.uint8, device=device)
+        for n, off, nbytes in layout:
+            t = getattr(self, n)
+            v = arena[off:off + nbytes].view(t.dtype).view(t.shape)
+            v.copy_(t)
+            setattr(self, n, v)
+        return arena
 
     # ------------------------------------------------------------------ descs
     def _view(self, l: int) -> pb.pf_kv_view:

@@ -5,6 +5,7 @@
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -45,13 +46,13 @@ bool pdl_enabled() {
 }
 
 int num_sms() {
-  static int cache[64] = {};
+  static pf::DeviceMemo cache;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 0;
-  if (dev >= 0 && dev < 64 && cache[dev]) return cache[dev];
+  if (const int n = cache.get(dev)) return n;
   int n = 0;
-  cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-  if (dev >= 0 && dev < 64) cache[dev] = n;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  cache.set(dev, n);
   return n;
 }
 
@@ -116,16 +117,18 @@ pf_status check_cache_view(const pf_kv_view& c, int need_rows, const char* who) 
 // is used only if the device can schedule it.
 // kernel index 0..2: mma.sync BM 32/64/128; 3: tcgen05
 int max_cluster_for(int kernel, int D, int want) {
-  static int cache[64][4][2][17];
+  static std::atomic<int> cache[64][4][2][17];
   int dev = 0;
   cudaGetDevice(&dev);
   const int di = D == 64 ? 0 : 1;
   int w = want;
   while (w > 8) {
-    int& c = cache[dev & 63][kernel][di][w];
+    std::atomic<int>& slot = cache[dev & 63][kernel][di][w];
+    int c = slot.load(std::memory_order_acquire);
     if (c == 0) {
       const bool fits = pf::attention_cluster_fits(D, 32 << kernel, w);
       c = fits ? 1 : -1;
+      slot.store(c, std::memory_order_release);
     }
     if (c > 0) break;
     w -= kernel == 3 ? 2 : 1;
@@ -134,11 +137,15 @@ int max_cluster_for(int kernel, int D, int want) {
 }
 
 int tc_max_active_clusters(int cluster, int bm) {
-  static int cache[64][2][17];
+  static std::atomic<int> cache[64][2][17];
   int dev = 0;
   cudaGetDevice(&dev);
-  int& c = cache[dev & 63][bm > 128 ? 1 : 0][cluster];
-  if (c == 0) c = std::max(1, pf::attention_tc_max_active_clusters(cluster, bm)) + 1;
+  std::atomic<int>& slot = cache[dev & 63][bm > 128 ? 1 : 0][cluster];
+  int c = slot.load(std::memory_order_acquire);
+  if (c == 0) {
+    c = std::max(1, pf::attention_tc_max_active_clusters(cluster, bm)) + 1;
+    slot.store(c, std::memory_order_release);
+  }
   return c - 1;
 }
 

@@ -434,17 +434,13 @@ __global__ void __launch_bounds__(256) attn_f32_kernel(const AttnArgs a) {
 template <int D, int BM>
 cudaError_t launch_bf16_t(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl) {
   const int smem = AttnSmem<D, BM>::kTotal + 1024;
-  static int limit[64] = {};
-  static bool nonportable[64] = {};
+  static DeviceMemo limit;
+  static DeviceMemo nonportable;
   cudaError_t e = ensure_smem_limit((const void*)attn_bf16_kernel<D, BM>, smem, limit);
   if (e != cudaSuccess) return e;
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (a.splits > 8 && dev >= 0 && dev < 64 && !nonportable[dev]) {
-    e = cudaFuncSetAttribute(attn_bf16_kernel<D, BM>,
-                             cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (a.splits > 8) {
+    e = ensure_nonportable_cluster((const void*)attn_bf16_kernel<D, BM>, nonportable);
     if (e != cudaSuccess) return e;
-    nonportable[dev] = true;
   }
   const dim3 grid(a.B * a.Hkv * a.rb_count * a.splits);
   return launch_ex(attn_bf16_kernel<D, BM>, grid, dim3(AttnSmem<D, BM>::kThreads), smem, s,
@@ -473,7 +469,7 @@ int attention_bf16_smem_bytes(int D, int bm) {
 template <int D, int BM>
 bool cluster_fits_t(int cluster) {
   const int smem = AttnSmem<D, BM>::kTotal + 1024;
-  static int limit[64] = {};
+  static DeviceMemo limit;
   if (ensure_smem_limit((const void*)attn_bf16_kernel<D, BM>, smem, limit) != cudaSuccess)
     return false;
   if (cluster > 8 && cudaFuncSetAttribute(attn_bf16_kernel<D, BM>,
@@ -514,7 +510,7 @@ cudaError_t launch_attention_bf16(const AttnArgs& a, const AttnMaps& m, cudaStre
 }
 
 cudaError_t launch_attention_f32(const AttnArgs& a, cudaStream_t s, bool pdl) {
-  static int limit[64] = {};
+  static DeviceMemo limit;
   const int smem = (kF32Tile * (a.D + 1) + kF32Tile * a.D + kF32Rows * a.D) * 4;
   cudaError_t e = ensure_smem_limit((const void*)attn_f32_kernel, smem, limit);
   if (e != cudaSuccess) return e;

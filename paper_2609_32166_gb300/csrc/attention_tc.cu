@@ -513,7 +513,7 @@ int attention_tc_smem_bytes() { return tc_smem_bytes<1>(); }
 template <int WG>
 static int tc_max_active_clusters_impl(int cluster) {
   const int smem = tc_smem_bytes<WG>();
-  static int limit[64] = {};
+  static DeviceMemo limit;
   if (ensure_smem_limit((const void*)attn_tc_kernel<128, WG>, smem, limit) != cudaSuccess)
     return 0;
   if (cluster > 8 && cudaFuncSetAttribute(attn_tc_kernel<128, WG>,
@@ -547,17 +547,13 @@ int attention_tc_max_active_clusters(int cluster, int rows_per_cta) {
 template <int WG>
 static cudaError_t launch_tc(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl) {
   const int smem = tc_smem_bytes<WG>();
-  static int limit[64] = {};
-  static bool nonportable[64] = {};
+  static DeviceMemo limit;
+  static DeviceMemo nonportable;
   cudaError_t e = ensure_smem_limit((const void*)attn_tc_kernel<128, WG>, smem, limit);
   if (e != cudaSuccess) return e;
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (a.splits > 8 && dev >= 0 && dev < 64 && !nonportable[dev]) {
-    e = cudaFuncSetAttribute(attn_tc_kernel<128, WG>,
-                             cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (a.splits > 8) {
+    e = ensure_nonportable_cluster((const void*)attn_tc_kernel<128, WG>, nonportable);
     if (e != cudaSuccess) return e;
-    nonportable[dev] = true;
   }
   const dim3 grid(a.B * a.Hkv * a.rb_count * a.splits);
   return launch_ex(attn_tc_kernel<128, WG>, grid, dim3(TcShape<WG>::kThreads), smem, s, a.splits,

@@ -207,12 +207,12 @@ __global__ void __launch_bounds__(kShiftThreads) kv_shift_kernel(const ShiftArgs
 constexpr int kMaxSegments = 8;
 
 cudaError_t launch_kv_shift(const ShiftArgs& a0, cudaStream_t s, int num_sms, bool pdl) {
-  static int resident[64][2] = {};
+  static DeviceMemo resident[2];  // resident CTAs per SM, fp32 / bf16 kernel
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   const int bf = a0.elem_bytes == 2;
-  int per_sm = dev < 64 ? resident[dev][bf] : 0;
+  int per_sm = resident[bf].get(dev);
   if (per_sm == 0) {
     e = bf ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(
                  &per_sm, kv_shift_flat_kernel<__nv_bfloat16>, kShiftThreads, 0)
@@ -220,7 +220,7 @@ cudaError_t launch_kv_shift(const ShiftArgs& a0, cudaStream_t s, int num_sms, bo
                                                             kShiftThreads, 0);
     if (e != cudaSuccess) return e;
     if (per_sm < 1) per_sm = 1;
-    if (dev < 64) resident[dev][bf] = per_sm;
+    resident[bf].set(dev, per_sm);
   }
   auto launch = [&](const ShiftArgs& a) {
     if (a.overlap) {

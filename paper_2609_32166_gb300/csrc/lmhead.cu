@@ -340,7 +340,7 @@ int lmhead_bf16_stages(int npad) {
 
 cudaError_t launch_lmhead_bf16(const LmArgs& a, const CUtensorMap& w_map,
                                const CUtensorMap& h_map, cudaStream_t s, int num_sms, bool pdl) {
-  static int limit[64] = {};
+  static DeviceMemo limit;
   const int smem = lmhead_bf16_smem_bytes(a.npad, a.stages);
   cudaError_t e = ensure_smem_limit((const void*)lmhead_tc_kernel, smem, limit);
   if (e != cudaSuccess) return e;

@@ -6,6 +6,7 @@
 #include <stdint.h>
 
 #include <algorithm>
+#include <atomic>
 #include <utility>
 
 #include "pf_verify.h"
@@ -191,13 +192,36 @@ pf_status set_error(pf_status s, const char* fmt, ...);
 
 // Raise a kernel's dynamic shared-memory limit once per device (never while
 // a stream is being captured after the first call on that device).
-inline cudaError_t ensure_smem_limit(const void* func, int bytes, int* per_device) {
+// Per-device memo of one int (0: not yet known), safe to read and fill
+// from several host threads at once (a racing fill stores the same value).
+struct DeviceMemo {
+  std::atomic<int> v[64];
+  int get(int dev) const {
+    return dev >= 0 && dev < 64 ? v[dev].load(std::memory_order_acquire) : 0;
+  }
+  void set(int dev, int x) {
+    if (dev >= 0 && dev < 64) v[dev].store(x, std::memory_order_release);
+  }
+};
+
+inline cudaError_t ensure_smem_limit(const void* func, int bytes, DeviceMemo& per_device) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  if (dev >= 0 && dev < 64 && per_device[dev] >= bytes) return cudaSuccess;
+  if (per_device.get(dev) >= bytes) return cudaSuccess;
   e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-  if (e == cudaSuccess && dev >= 0 && dev < 64) per_device[dev] = bytes;
+  if (e == cudaSuccess) per_device.set(dev, bytes);
+  return e;
+}
+
+// Allow cluster sizes above 8 for a kernel, once per device.
+inline cudaError_t ensure_nonportable_cluster(const void* func, DeviceMemo& per_device) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (per_device.get(dev)) return cudaSuccess;
+  e = cudaFuncSetAttribute(func, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e == cudaSuccess) per_device.set(dev, 1);
   return e;
 }
 

@@ -338,7 +338,7 @@ cudaError_t launch_retrieval_key(const KeyArgs& a, cudaStream_t s, bool pdl) {
 }
 
 cudaError_t launch_retrieve(const RetrievalArgs& a, cudaStream_t s, int num_sms, bool pdl) {
-  static int smem_set[64] = {};
+  static DeviceMemo smem_set;
   cudaError_t e = ensure_smem_limit(reinterpret_cast<const void*>(retrieve_kernel), kScanSmem,
                                     smem_set);
   if (e != cudaSuccess) return e;

@@ -161,14 +161,14 @@ __global__ void __launch_bounds__(BM * 2, 1)
     if (valid < kBN) {
       // Rows past the prefix end may hold anything (even NaN bit patterns):
       // zero their V so masked-out columns contribute exactly 0.
-      uint8_t* sv = stage + S::kTileBytes;
-      const int per_half = (kBN - valid) * 8;
-      for (int c = tid; c < per_half * S::kHalves; c += kThreads) {
-        const int h = c / per_half;
-        const int rem = c % per_half;
-        *reinterpret_cast<uint4*>(sv + h * kBN * 128 + (valid + rem / 8) * 128 + (rem % 8) * 16) =
-            make_uint4(0, 0, 0, 0);
-      }
+      // (each 64-column half holds its rows at 128-byte pitch: the rows
+      // from `valid` on are one contiguous run per half)
+      uint4* sv = reinterpret_cast<uint4*>(stage + S::kTileBytes);
+      const int per_half = (kBN - valid) * 8;   // 16-byte chunks past the end
+#pragma unroll
+      for (int h = 0; h < S::kHalves; ++h)
+        for (int c = tid; c < per_half; c += kThreads)
+          sv[h * kBN * 8 + valid * 8 + c] = make_uint4(0, 0, 0, 0);
       fence_proxy_async_smem();
       __syncthreads();
     }

@@ -132,9 +132,23 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
   const int rows = min(a.nb, nn - nfirst) * a.G;
   const int nblk = WG == 1 ? 1 : (rows > 128 ? 2 : 1);  // row blocks with work
   const int n_ptiles = (P + kBN - 1) / kBN;
-  const int ntiles = n_ptiles + (nn + kBN - 1) / kBN;
+  const int n_qtiles = (nn + kBN - 1) / kBN;
+  const int ntiles = n_ptiles + n_qtiles;
+  // Split s takes tiles [t_begin, t_end) of the order (proposal tiles,
+  // prefix tiles): the proposal's K/V can only be loaded once the preceding
+  // kernel has finished, so those tiles go to the first split, which holds
+  // the fewest tiles (ntiles * s / nsplit rounds down).  Within a split the
+  // prefix tiles come first (their loads start before that wait).
   const int t_begin = (int)((long long)ntiles * split / nsplit);
-  const int my_tiles = (int)((long long)ntiles * (split + 1) / nsplit) - t_begin;
+  const int t_end = (int)((long long)ntiles * (split + 1) / nsplit);
+  const int my_tiles = t_end - t_begin;
+  const int pre_lo = max(t_begin, n_qtiles);        // first prefix tile of the split
+  const int my_ptiles = max(0, t_end - pre_lo);
+  // cache tile index (prefix tiles 0..n_ptiles-1, then proposal tiles) of
+  // the split's i-th tile
+  auto tile_at = [&](int i) {
+    return i < my_ptiles ? pre_lo - n_qtiles + i : n_ptiles + t_begin + (i - my_ptiles);
+  };
   const int first = min(kTcStages, my_tiles);
 
   if (tid == 0) {
@@ -153,9 +167,9 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
     mbar_init(smem_u32(inbox_full), 1);
     fence_mbar_init();
     for (int i = 0; i < first; ++i)
-      if (t_begin + i < n_ptiles)
+      if (i < my_ptiles)
         issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
-                         smem_u32(&kv_full[i]), t_begin + i, n_ptiles, b, g, node0, P);
+                         smem_u32(&kv_full[i]), tile_at(i), n_ptiles, b, g, node0, P);
   }
   if (early) pdl_wait();
   if (tid == 0) {
@@ -165,9 +179,9 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
       tma_load_3d(smem_u32(sQ + h * S::kRows * 128), &tm_q, h * 64, g * a.G, node0 + nfirst,
                   smem_u32(q_full));
     for (int i = 0; i < first; ++i)
-      if (t_begin + i >= n_ptiles)
+      if (i >= my_ptiles)
         issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
-                         smem_u32(&kv_full[i]), t_begin + i, n_ptiles, b, g, node0, P);
+                         smem_u32(&kv_full[i]), tile_at(i), n_ptiles, b, g, node0, P);
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), kTmemCols);
@@ -192,7 +206,7 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
         const int st = i % kTcStages;
         if (!mbar_wait(smem_u32(&kv_empty[st]), ((i / kTcStages) & 1) ^ 1, a.err)) break;
         issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + st * S::kStageBytes,
-                         smem_u32(&kv_full[st]), t_begin + i, n_ptiles, b, g, node0, P);
+                         smem_u32(&kv_full[st]), tile_at(i), n_ptiles, b, g, node0, P);
       }
     }
   } else if (warp == 1) {
@@ -298,7 +312,7 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
       tc_fence_before();
       mbar_arrive(smem_u32(&bw[2 + sb]));
 
-      const int t = t_begin + i;
+      const int t = tile_at(i);
       const bool is_prefix = t < n_ptiles;
       const int valid = is_prefix ? min(kBN, P - t * kBN) : kBN;
       float sv[64];
@@ -379,13 +393,14 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
         // Cache rows past the prefix end may hold anything (even NaN bit
         // patterns): zero their V so masked columns contribute exactly 0.
         // (With two blocks both write the same zeros before their PV.)
-        uint8_t* sv = sKV + st * S::kStageBytes + S::kTileBytes;
-        const int per_half = (kBN - valid) * 8;
-        for (int c = rl; c < per_half * S::kHalves; c += 128) {
-          const int h = c / per_half, rem = c % per_half;
-          *reinterpret_cast<uint4*>(sv + h * kBN * 128 + (valid + rem / 8) * 128 + (rem % 8) * 16) =
-              make_uint4(0, 0, 0, 0);
-        }
+        // Each 64-column half of the V tile holds its rows at 128-byte
+        // pitch, so the rows from `valid` on are one contiguous run per half.
+        uint4* sv = reinterpret_cast<uint4*>(sKV + st * S::kStageBytes + S::kTileBytes);
+        const int per_half = (kBN - valid) * 8;   // 16-byte chunks past the end
+#pragma unroll
+        for (int h = 0; h < S::kHalves; ++h)
+          for (int c = rl; c < per_half; c += 128)
+            sv[h * kBN * 8 + valid * 8 + c] = make_uint4(0, 0, 0, 0);
       }
       fence_proxy_async_smem();
       tc_fence_before();

@@ -147,6 +147,8 @@ typedef struct pf_attn_desc {
   void* out;                   /* device [T][Hq][D]                          */
   int32_t* error_flag;         /* optional device int32                      */
   int32_t flags;               /* PF_ATTN_* bits, 0 = none                   */
+  void* workspace;             /* optional device scratch (see below)        */
+  size_t workspace_bytes;      /* its size                                   */
 } pf_attn_desc;
 
 /* PF_ATTN_EARLY_PREFETCH: the prefix cache, page_table, cu_nodes, prefix_len
@@ -158,6 +160,19 @@ typedef struct pf_attn_desc {
  * read only after it finishes.  Leave it clear when the preceding kernel may
  * write any of those inputs. */
 #define PF_ATTN_EARLY_PREFETCH 1
+
+/* Workspace (optional; batches of B > 1 sequences, bf16, head_dim 128):
+ * with workspace != NULL and at least pf_verify_attention_workspace_size(d)
+ * bytes (16-byte aligned), a batch's KV tiles are dealt out to one CTA per
+ * SM in proportion to each sequence's length (prefix plus proposal tiles),
+ * so long and short prefixes finish together; sequences spread over several
+ * CTAs are merged by a second kernel in the same stream (the call then
+ * launches two kernels).  Without it every (sequence, KV head) gets the
+ * same number of CTAs.  The contents need no initialisation and are
+ * scratch between calls; one workspace serves calls in stream order but
+ * not concurrent calls.  A workspace that is too small is an error
+ * (PF_ERR_WORKSPACE); for shapes that do not use it, it is ignored. */
+PF_API size_t pf_verify_attention_workspace_size(const pf_attn_desc* d);
 
 PF_API pf_status pf_verify_attention(const pf_attn_desc* d, void* stream);
 

@@ -57,7 +57,8 @@ class pf_attn_desc(C.Structure):
                 ("max_prefix_len", C.c_int32), ("cu_nodes", C.c_void_p),
                 ("prefix_len", C.c_void_p), ("q", C.c_void_p), ("tree_k", C.c_void_p),
                 ("tree_v", C.c_void_p), ("mask", C.c_void_p), ("cache", pf_kv_view),
-                ("out", C.c_void_p), ("error_flag", C.c_void_p), ("flags", C.c_int32)]
+                ("out", C.c_void_p), ("error_flag", C.c_void_p), ("flags", C.c_int32),
+                ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t)]
 
 
 class pf_lm_desc(C.Structure):
@@ -138,6 +139,8 @@ def lib() -> C.CDLL:
     L.pf_tree_prepare.argtypes = [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p]
     L.pf_verify_attention.restype = C.c_int
     L.pf_verify_attention.argtypes = [C.POINTER(pf_attn_desc), C.c_void_p]
+    L.pf_verify_attention_workspace_size.restype = C.c_size_t
+    L.pf_verify_attention_workspace_size.argtypes = [C.POINTER(pf_attn_desc)]
     L.pf_lmhead_accept_workspace_size.restype = C.c_size_t
     L.pf_lmhead_accept_workspace_size.argtypes = [C.POINTER(pf_lm_desc)]
     L.pf_lmhead_accept.restype = C.c_int
@@ -203,6 +206,10 @@ def pf_tree_prepare(parent) -> tuple:
     mask = np.zeros((max(n, 1), PF_MASK_WORDS), dtype=np.uint64)
     _check(lib().pf_tree_prepare(p.ctypes.data, n, depth.ctypes.data, mask.ctypes.data))
     return depth[:n], mask[:n]
+
+
+def pf_verify_attention_workspace_size(desc: pf_attn_desc) -> int:
+    return int(lib().pf_verify_attention_workspace_size(C.byref(desc)))
 
 
 def pf_verify_attention(desc: pf_attn_desc, stream: int = 0) -> None:

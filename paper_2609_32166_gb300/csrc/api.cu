@@ -208,6 +208,15 @@ void choose_attention_shape(pf::AttnArgs& a, int max_prefix_len, int sms) {
   a.splits = splits;
 }
 
+// Balanced batch mode (tcgen05 path, B > 1): one CTA per SM, provided the
+// plan can give every (sequence, KV head, row block) group at least one.
+int balanced_items(const pf::AttnArgs& a, int sms) {
+  if (a.B < 2 || !use_tc_attention(a)) return 0;
+  const int groups = a.B * a.Hkv * a.rb_count;
+  if (groups > sms || groups > pf::kPlanMaxGroups) return 0;
+  return sms;
+}
+
 }  // namespace
 
 namespace pf {
@@ -254,6 +263,26 @@ pf_status pf_tree_prepare(const int32_t* parent, int32_t n_nodes, int32_t* depth
     mj[j >> 6] |= 1ull << (j & 63);
   }
   return PF_OK;
+}
+
+size_t pf_verify_attention_workspace_size(const pf_attn_desc* d) {
+  if (!d || d->dtype != PF_BF16 || d->batch < 2 || d->n_kv_heads < 1 || d->n_q_heads < 1 ||
+      d->n_q_heads % d->n_kv_heads != 0 || d->max_nodes < 1 || d->max_nodes > PF_MAX_NODES ||
+      d->max_prefix_len < 0)
+    return 0;
+  const int sms = num_sms();
+  if (sms <= 0) return 0;
+  pf::AttnArgs a = {};
+  a.B = d->batch;
+  a.Hq = d->n_q_heads;
+  a.Hkv = d->n_kv_heads;
+  a.D = d->head_dim;
+  a.G = a.Hq / a.Hkv;
+  a.max_nodes = d->max_nodes;
+  if (!use_tc_attention(a) || a.G > 128) return 0;
+  choose_attention_shape(a, d->max_prefix_len, sms);
+  const int items = balanced_items(a, sms);
+  return items > 0 ? pf::attention_balanced_ws_bytes(items, a.bm, a.D) : 0;
 }
 
 pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
@@ -355,8 +384,22 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
     if ((st = make_map(&m.ck, 4, d->cache.k, dims, str, box, "cache.k")) != PF_OK) return st;
     if ((st = make_map(&m.cv, 4, d->cache.v, dims, str, box, "cache.v")) != PF_OK) return st;
   }
+  if (d->workspace) {
+    const int items = balanced_items(a, sms);
+    if (items > 0) {
+      const size_t need = pf::attention_balanced_ws_bytes(items, a.bm, a.D);
+      if (d->workspace_bytes < need)
+        return fail(PF_ERR_WORKSPACE, "%s: workspace needs %zu bytes", who, need);
+      if (!aligned16(d->workspace))
+        return fail(PF_ERR_ALIGN, "%s: workspace must be 16-byte aligned", who);
+      a.splits = 1;
+      a.items = items;
+      a.ws = d->workspace;
+    }
+  }
   cudaError_t e = use_tc_attention(a) ? pf::launch_attention_tc(a, m, s, pdl_enabled())
                                       : pf::launch_attention_bf16(a, m, s, sms, pdl_enabled());
+  if (e == cudaSuccess && a.items > 0) e = pf::launch_attention_combine(a, s, pdl_enabled());
   return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
 }
 

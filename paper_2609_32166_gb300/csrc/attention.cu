@@ -99,10 +99,15 @@ __global__ void __launch_bounds__(BM * 2, 1)
     for (int i = 0; i < kStages; ++i) mbar_init(smem_u32(&bars[i]), 1);
     mbar_init(qbar, 1);
     fence_mbar_init();
-    for (int i = 0; i < first; ++i)
-      if (t_begin + i < n_ptiles)
+    int4 pg[kStages];  // every first tile's page entries in one round trip
+#pragma unroll
+    for (int i = 0; i < kStages; ++i)
+      pg[i] = i < first ? kv_tile_pages(a, t_begin + i, n_ptiles, b, P) : make_int4(-1, -1, -1, -1);
+#pragma unroll
+    for (int i = 0; i < kStages; ++i)
+      if (i < first && t_begin + i < n_ptiles)
         issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
-                             smem_u32(&bars[i]), t_begin + i, n_ptiles, b, g, node0, P);
+                         smem_u32(&bars[i]), t_begin + i, n_ptiles, b, g, node0, P, pg[i]);
   }
   if (early) pdl_wait();
   if (tid == 0) {
@@ -111,9 +116,10 @@ __global__ void __launch_bounds__(BM * 2, 1)
     for (int h = 0; h < S::kHalves; ++h)
       tma_load_3d(smem_u32(sQ + h * BM * 128), &tm_q, h * 64, g * a.G, node0 + nfirst, qbar);
     for (int i = 0; i < first; ++i)
-      if (t_begin + i >= n_ptiles)
+      if (t_begin + i >= n_ptiles)  // proposal tiles: no page entries
         issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
-                             smem_u32(&bars[i]), t_begin + i, n_ptiles, b, g, node0, P);
+                         smem_u32(&bars[i]), t_begin + i, n_ptiles, b, g, node0, P,
+                         make_int4(-1, -1, -1, -1));
   }
   __syncthreads();
   pdl_launch_dependents();
@@ -256,10 +262,13 @@ __global__ void __launch_bounds__(BM * 2, 1)
       }
     }
     if (i + kStages < my_tiles) {
+      // the refill's page entries are in flight while the warps finish
+      const int4 pg = tid == 0 ? kv_tile_pages(a, t + kStages, n_ptiles, b, P)
+                               : make_int4(-1, -1, -1, -1);
       __syncthreads();  // every warp is done with this stage before it is refilled
       if (tid == 0)
         issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, stage, smem_u32(&bars[st]),
-                             t + kStages, n_ptiles, b, g, node0, P);
+                         t + kStages, n_ptiles, b, g, node0, P, pg);
     }
   }
 

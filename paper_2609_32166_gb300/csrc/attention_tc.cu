@@ -73,7 +73,9 @@ struct TcSmem {
   static_assert(WG == 1 || kInboxSlots * kRowBytes <= kQOff, "inbox fits in the ring");
   // kv_full[3] kv_empty[3] q_full, per block s_full[2] s_empty[2] p_full[2] pv_done[2], inbox
   static constexpr int kNumBars = 2 * kTcStages + 1 + 8 * WG + 1;
-  static constexpr int kTotal = kBarOff + kNumBars * 8 + 16;
+  // then the TMEM address (4 bytes, padded to 16) and the balanced batch
+  // mode's plan entry (16 bytes)
+  static constexpr int kTotal = kBarOff + kNumBars * 8 + 32;
   static_assert(kTotal + 1024 <= 232448, "shared memory budget");
 };
 
@@ -105,11 +107,6 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
   cg::cluster_group cluster = cg::this_cluster();
   const int nsplit = a.splits;
   const int split = (int)cluster.block_rank();
-  int cid = blockIdx.x / nsplit;
-  const int rb = cid % a.rb_count;
-  cid /= a.rb_count;
-  const int g = cid % a.Hkv;
-  const int b = cid / a.Hkv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
   // With PF_ATTN_EARLY_PREFETCH the tree structure, prefix lengths and the
@@ -118,6 +115,40 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
   // dependent launch); q and the proposal K/V only after.
   const bool early = (a.flags & PF_ATTN_EARLY_PREFETCH) != 0;
   if (!early) pdl_wait();
+
+  // This CTA's group (sequence, KV head, row block) and its part of the
+  // group's tiles: split `split` of the cluster, or (balanced batch mode,
+  // one CTA per cluster) the item the plan gives it.
+  int group = blockIdx.x / nsplit, part = split, nparts = nsplit;
+  if (a.items > 0) {
+    // warp 0 derives the plan; the first n_groups CTAs also record group
+    // blockIdx.x's (first item, items) for the combine kernel
+    int4* plan_slot = reinterpret_cast<int4*>(smem + S::kBarOff + S::kNumBars * 8 + 16);
+    if (warp == 0) {
+      const int n_groups = a.B * a.Hkv * a.rb_count;
+      const int gq = (int)blockIdx.x < n_groups ? (int)blockIdx.x : -1;
+      PlanItem ge;
+      const PlanItem it = balanced_plan(a, (int)blockIdx.x, gq, &ge);
+      if (lane == 0) {
+        *plan_slot = make_int4(it.group, it.j, it.k, 0);
+        if (gq >= 0) {
+          // the group's first node and rows, for the combine kernel
+          const int bq = gq / (a.rb_count * a.Hkv), nfq = (gq % a.rb_count) * a.nb;
+          const int n0 = a.cu_nodes[bq], nnq = a.cu_nodes[bq + 1] - n0;
+          plan_table(a)[gq] = make_int4(ge.first, ge.k, n0 + nfq, max(0, min(a.nb, nnq - nfq)) * a.G);
+        }
+      }
+    }
+    __syncthreads();
+    const int4 pi = *plan_slot;
+    if (pi.x < 0) return;  // uniform over the CTA: no work for this item
+    group = pi.x;
+    part = pi.y;
+    nparts = pi.z;
+  }
+  const int rb = group % a.rb_count;
+  const int g = (group / a.rb_count) % a.Hkv;
+  const int b = group / (a.rb_count * a.Hkv);
 
   const int node0 = a.cu_nodes[b];
   const int nn = a.cu_nodes[b + 1] - node0;
@@ -139,8 +170,8 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
   // kernel has finished, so those tiles go to the first split, which holds
   // the fewest tiles (ntiles * s / nsplit rounds down).  Within a split the
   // prefix tiles come first (their loads start before that wait).
-  const int t_begin = (int)((long long)ntiles * split / nsplit);
-  const int t_end = (int)((long long)ntiles * (split + 1) / nsplit);
+  const int t_begin = (int)((long long)ntiles * part / nparts);
+  const int t_end = (int)((long long)ntiles * (part + 1) / nparts);
   const int my_tiles = t_end - t_begin;
   const int pre_lo = max(t_begin, n_qtiles);        // first prefix tile of the split
   const int my_ptiles = max(0, t_end - pre_lo);
@@ -166,10 +197,15 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
       }
     mbar_init(smem_u32(inbox_full), 1);
     fence_mbar_init();
-    for (int i = 0; i < first; ++i)
-      if (i < my_ptiles)
+    int4 pg[kTcStages];  // every first tile's page entries in one round trip
+#pragma unroll
+    for (int i = 0; i < kTcStages; ++i)
+      pg[i] = i < first ? kv_tile_pages(a, tile_at(i), n_ptiles, b, P) : make_int4(-1, -1, -1, -1);
+#pragma unroll
+    for (int i = 0; i < kTcStages; ++i)
+      if (i < first && i < my_ptiles)
         issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
-                         smem_u32(&kv_full[i]), tile_at(i), n_ptiles, b, g, node0, P);
+                         smem_u32(&kv_full[i]), tile_at(i), n_ptiles, b, g, node0, P, pg[i]);
   }
   if (early) pdl_wait();
   if (tid == 0) {
@@ -179,9 +215,10 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
       tma_load_3d(smem_u32(sQ + h * S::kRows * 128), &tm_q, h * 64, g * a.G, node0 + nfirst,
                   smem_u32(q_full));
     for (int i = 0; i < first; ++i)
-      if (i >= my_ptiles)
+      if (i >= my_ptiles)  // proposal tiles: no page entries
         issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
-                         smem_u32(&kv_full[i]), tile_at(i), n_ptiles, b, g, node0, P);
+                         smem_u32(&kv_full[i]), tile_at(i), n_ptiles, b, g, node0, P,
+                         make_int4(-1, -1, -1, -1));
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), kTmemCols);
@@ -204,9 +241,11 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
     if (lane == 0) {
       for (int i = kTcStages; i < my_tiles; ++i) {
         const int st = i % kTcStages;
+        const int t = tile_at(i);
+        const int4 pg = kv_tile_pages(a, t, n_ptiles, b, P);  // in flight during the wait
         if (!mbar_wait(smem_u32(&kv_empty[st]), ((i / kTcStages) & 1) ^ 1, a.err)) break;
         issue_kv_tile<D>(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + st * S::kStageBytes,
-                         smem_u32(&kv_full[st]), tile_at(i), n_ptiles, b, g, node0, P);
+                         smem_u32(&kv_full[st]), t, n_ptiles, b, g, node0, P, pg);
       }
     }
   } else if (warp == 1) {
@@ -428,14 +467,28 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
   // own shared memory:
   //   out = sum_s 2^(lse_s - M) (O/l)_s / sum_s 2^(lse_s - M),  M = max_s lse_s
   if (nsplit == 1) {
-    // ---- single split: O / l is the output
+    // ---- single split: O / l is the output -- or, for a group that the
+    // balanced batch mode spread over several CTAs, this item's partial
+    // (same format as a staged row) for the combine kernel
     if (has_row) {
       uint32_t ov[D];
 #pragma unroll
       for (int c0 = 0; c0 < D; c0 += 32)
         tmem_ld_32(o_addr + c0, *reinterpret_cast<uint32_t(*)[32]>(&ov[c0]));
       tmem_ld_wait();
-      if (r < rows) {
+      if (r < rows && nparts > 1) {
+        __half* dst = reinterpret_cast<__half*>(a.ws) + ((size_t)blockIdx.x * a.bm + r) * S::kInboxPitch;
+#pragma unroll
+        for (int c = 0; c < D; c += 8) {
+          uint4 pk;
+          pk.x = pack_half(__uint_as_float(ov[c]) * inv_l, __uint_as_float(ov[c + 1]) * inv_l);
+          pk.y = pack_half(__uint_as_float(ov[c + 2]) * inv_l, __uint_as_float(ov[c + 3]) * inv_l);
+          pk.z = pack_half(__uint_as_float(ov[c + 4]) * inv_l, __uint_as_float(ov[c + 5]) * inv_l);
+          pk.w = pack_half(__uint_as_float(ov[c + 6]) * inv_l, __uint_as_float(ov[c + 7]) * inv_l);
+          *reinterpret_cast<uint4*>(dst + c) = pk;
+        }
+        *reinterpret_cast<float*>(dst + D) = inv_l > 0.f ? m_ref + __log2f(l) : -INFINITY;
+      } else if (r < rows) {
         const int node = node0 + nfirst + r / a.G;
         const int h = g * a.G + r % a.G;
         __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(a.out) + ((size_t)node * a.Hq + h) * D;
@@ -516,7 +569,90 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
   if (tid < nsplit) bulk_wait_read_all();
 }
 
+// Balanced batch mode, second kernel: for every group that the plan spread
+// over k > 1 CTAs, merge the k partials of each row (same rule as the
+// cluster merge: out = sum_j 2^(lse_j - M) (O/l)_j / sum_j 2^(lse_j - M)).
+// One CTA per (group, 16 rows), one thread per (row, 8 columns).  Every CTA
+// waits for the attention kernel before it exits, so kernels that follow in
+// the stream see the attention outputs complete.
+constexpr int kCombineRows = 16;
+
+__global__ void __launch_bounds__(256) attn_combine_kernel(const AttnArgs a) {
+  constexpr int D = 128, C8 = D / 8, kPitch = D + 8, kBatch = 8;
+  const int chunks = (a.bm + kCombineRows - 1) / kCombineRows;
+  const int group = blockIdx.x / chunks, chunk = blockIdx.x % chunks;
+  pdl_wait();
+  pdl_launch_dependents();
+  const int4 e = plan_table(a)[group];  // from the attention kernel
+  const int first = e.x, k = e.y, node_base = e.z, rows = e.w;
+  const int r = chunk * kCombineRows + (int)threadIdx.x / C8;
+  const int c8 = (int)threadIdx.x % C8;
+  if (k <= 1 || r >= rows) return;
+  const __half* base = reinterpret_cast<const __half*>(a.ws) + ((size_t)first * a.bm + r) * kPitch;
+  const size_t item_stride = (size_t)a.bm * kPitch;
+  // partials in batches of 8 (all loads of a batch in flight together),
+  // folded into a running maximum M, weight sum W and weighted sum acc
+  float M = -INFINITY, W = 0.f;
+  float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  for (int j0 = 0; j0 < k; j0 += kBatch) {
+    float ls[kBatch];
+    uint4 v[kBatch];
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      ls[u] = -INFINITY;
+      if (j0 + u < k) {
+        const __half* row = base + (size_t)(j0 + u) * item_stride;
+        ls[u] = *reinterpret_cast<const float*>(row + D);
+        v[u] = *reinterpret_cast<const uint4*>(row + c8 * 8);
+      }
+    }
+    float Mb = M;
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) Mb = fmaxf(Mb, ls[u]);
+    if (Mb == -INFINITY) continue;  // nothing but empty partials so far
+    const float sc = ex2_approx(M - Mb);  // M = -inf -> 0
+    W *= sc;
+#pragma unroll
+    for (int c = 0; c < 8; ++c) acc[c] *= sc;
+    M = Mb;
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      if (ls[u] == -INFINITY) continue;  // absent or empty partial
+      const float w = ex2_approx(ls[u] - M);
+      W += w;
+      const __half2* h2 = reinterpret_cast<const __half2*>(&v[u]);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const float2 f = __half22float2(h2[c]);
+        acc[2 * c] = fmaf(w, f.x, acc[2 * c]);
+        acc[2 * c + 1] = fmaf(w, f.y, acc[2 * c + 1]);
+      }
+    }
+  }
+  const float inv = W > 0.f ? __fdividef(1.f, W) : 0.f;
+  const int g = (group / a.rb_count) % a.Hkv;
+  const int node = node_base + r / a.G;
+  const int h = g * a.G + r % a.G;
+  uint4 pk;
+  pk.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+  pk.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+  pk.z = pack_bf16(acc[4] * inv, acc[5] * inv);
+  pk.w = pack_bf16(acc[6] * inv, acc[7] * inv);
+  *reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.out) +
+                            ((size_t)node * a.Hq + h) * D + c8 * 8) = pk;
+}
+
 }  // namespace
+
+size_t attention_balanced_ws_bytes(int items, int bm, int D) {
+  return (size_t)items * bm * (D + 8) * 2 + kPlanMaxGroups * sizeof(int4);
+}
+
+cudaError_t launch_attention_combine(const AttnArgs& a, cudaStream_t s, bool pdl) {
+  const int chunks = (a.bm + kCombineRows - 1) / kCombineRows;
+  const dim3 grid(a.B * a.Hkv * a.rb_count * chunks);
+  return launch_ex(attn_combine_kernel, grid, dim3(256), 0, s, 1, pdl, a);
+}
 
 template <int WG>
 static int tc_smem_bytes() {
@@ -570,7 +706,7 @@ static cudaError_t launch_tc(const AttnArgs& a, const AttnMaps& m, cudaStream_t 
     e = ensure_nonportable_cluster((const void*)attn_tc_kernel<128, WG>, nonportable);
     if (e != cudaSuccess) return e;
   }
-  const dim3 grid(a.B * a.Hkv * a.rb_count * a.splits);
+  const dim3 grid(a.items > 0 ? a.items : a.B * a.Hkv * a.rb_count * a.splits);
   return launch_ex(attn_tc_kernel<128, WG>, grid, dim3(TcShape<WG>::kThreads), smem, s, a.splits,
                    pdl, m.q, m.tk, m.tv, m.ck, m.cv, a);
 }

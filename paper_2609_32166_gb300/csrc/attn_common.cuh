@@ -17,12 +17,39 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
 }
 
+// Page-table entries of prefix tile t of a paged cache (a 64-token tile is
+// four 16-token pages), loaded together so that their latencies overlap:
+// callers fetch them before they wait for the ring stage the tile goes to.
+// -1 where the tile has no such page (past the prefix end), and for a
+// contiguous cache or a proposal tile.
+static_assert(kBN == 4 * PF_PAGE_SIZE, "a K/V tile spans four pages");
+
+__device__ __forceinline__ int4 kv_tile_pages(const AttnArgs& a, int t, int n_ptiles, int b,
+                                              int P) {
+  int4 pg = make_int4(-1, -1, -1, -1);
+  if (a.layout != PF_KV_CONTIGUOUS && t < n_ptiles) {
+    const int tok0 = t * kBN;
+    const int npages = min(4, (P - tok0 + PF_PAGE_SIZE - 1) / PF_PAGE_SIZE);  // >= 1
+    const int32_t* pt = a.page_table + (size_t)b * a.pages_per_seq + tok0 / PF_PAGE_SIZE;
+    pg.x = pt[0];
+    if (npages > 1) pg.y = pt[1];
+    if (npages > 2) pg.z = pt[2];
+    if (npages > 3) pg.w = pt[3];
+  }
+  return pg;
+}
+
+// TMA loads of one 64-token K/V tile into a ring stage (K then V, each two
+// 64-column halves): from the prefix cache (contiguous: one 3-D box per
+// half; paged: one 4-D box per 16-token page that holds prefix rows, pages
+// from kv_tile_pages) or, past the prefix, from the proposal's own rows.
+// Arms `bar` with the bytes it will bring.
 template <int D>
 __device__ __forceinline__ void issue_kv_tile(const AttnArgs& a, const CUtensorMap* tm_ck,
                                               const CUtensorMap* tm_cv, const CUtensorMap* tm_tk,
                                               const CUtensorMap* tm_tv, uint8_t* stage,
                                               uint32_t bar, int t, int n_ptiles, int b, int g,
-                                              int node0, int P) {
+                                              int node0, int P, int4 pg) {
   constexpr int kHalves = D / 64;
   constexpr int kTileBytes = kBN * D * 2;
   uint8_t* sk = stage;
@@ -40,14 +67,15 @@ __device__ __forceinline__ void issue_kv_tile(const AttnArgs& a, const CUtensorM
       const int left = P - tok0;
       const int npages = min(kBN / PF_PAGE_SIZE, (left + PF_PAGE_SIZE - 1) / PF_PAGE_SIZE);
       mbar_arrive_expect_tx(bar, 2 * kHalves * npages * PF_PAGE_SIZE * 128);
-      const int32_t* pt = a.page_table + (size_t)b * a.pages_per_seq + tok0 / PF_PAGE_SIZE;
-      for (int p = 0; p < npages; ++p) {
-        const int page = pt[p];
+      const int pages[4] = {pg.x, pg.y, pg.z, pg.w};
+#pragma unroll
+      for (int p = 0; p < 4; ++p) {
+        if (p >= npages) break;
 #pragma unroll
         for (int h = 0; h < kHalves; ++h) {
           const int off = h * kBN * 128 + p * PF_PAGE_SIZE * 128;
-          tma_load_4d(smem_u32(sk + off), tm_ck, h * 64, 0, g, page, bar);
-          tma_load_4d(smem_u32(sv + off), tm_cv, h * 64, 0, g, page, bar);
+          tma_load_4d(smem_u32(sk + off), tm_ck, h * 64, 0, g, pages[p], bar);
+          tma_load_4d(smem_u32(sv + off), tm_cv, h * 64, 0, g, pages[p], bar);
         }
       }
     }
@@ -59,46 +87,6 @@ __device__ __forceinline__ void issue_kv_tile(const AttnArgs& a, const CUtensorM
       tma_load_3d(smem_u32(sk + h * kBN * 128), tm_tk, h * 64, g, node0 + j * kBN, bar);
       tma_load_3d(smem_u32(sv + h * kBN * 128), tm_tv, h * 64, g, node0 + j * kBN, bar);
     }
-  }
-}
-
-// TMA load of one 64-token tile of ONE matrix (K or V): from the prefix
-// cache (contiguous: one 3-D box per 64-column half; paged: one 4-D box per
-// 16-token page, only the pages that hold prefix rows) or, past the prefix,
-// from the proposal's own rows.  Arms `bar` with the bytes it will bring.
-template <int D>
-__device__ __forceinline__ void issue_one_tile(const AttnArgs& a, const CUtensorMap* tm_cache,
-                                               const CUtensorMap* tm_tree, uint8_t* dst,
-                                               uint32_t bar, int t, int n_ptiles, int b, int g,
-                                               int node0, int P) {
-  constexpr int kHalves = D / 64;
-  constexpr int kTileBytes = kBN * D * 2;
-  if (t < n_ptiles) {
-    const int tok0 = t * kBN;
-    if (a.layout == PF_KV_CONTIGUOUS) {
-      mbar_arrive_expect_tx(bar, kTileBytes);
-#pragma unroll
-      for (int h = 0; h < kHalves; ++h)
-        tma_load_3d(smem_u32(dst + h * kBN * 128), tm_cache, h * 64, tok0, b * a.Hkv + g, bar);
-    } else {
-      const int left = P - tok0;
-      const int npages = min(kBN / PF_PAGE_SIZE, (left + PF_PAGE_SIZE - 1) / PF_PAGE_SIZE);
-      mbar_arrive_expect_tx(bar, kHalves * npages * PF_PAGE_SIZE * 128);
-      const int32_t* pt = a.page_table + (size_t)b * a.pages_per_seq + tok0 / PF_PAGE_SIZE;
-      for (int p = 0; p < npages; ++p) {
-        const int page = pt[p];
-#pragma unroll
-        for (int h = 0; h < kHalves; ++h)
-          tma_load_4d(smem_u32(dst + h * kBN * 128 + p * PF_PAGE_SIZE * 128), tm_cache, h * 64, 0,
-                      g, page, bar);
-      }
-    }
-  } else {
-    const int j = t - n_ptiles;
-    mbar_arrive_expect_tx(bar, kTileBytes);
-#pragma unroll
-    for (int h = 0; h < kHalves; ++h)
-      tma_load_3d(smem_u32(dst + h * kBN * 128), tm_tree, h * 64, g, node0 + j * kBN, bar);
   }
 }
 
@@ -182,6 +170,117 @@ __device__ __forceinline__ void cluster_merge(const AttnArgs& a,
     }
   }
   cluster.sync();
+}
+
+// ---- balanced batch mode: the work plan.  Group q = (b * Hkv + g) *
+// rb_count + rb (sequence b, KV head g, row block rb) holds
+//   tiles_q = ceil(P_b / 64) + ceil(nn_b / 64)
+// K/V tiles if its row block has nodes (rb * nb < nn_b), else none.  With
+// the smallest T for which sum_q ceil(tiles_q / T) <= items, group q gets
+// k_q = ceil(tiles_q / T) consecutive items (CTAs), which split its tiles
+// evenly, so no CTA holds more than T tiles while every group is served in
+// one wave.  Warp 0 of every attention CTA derives the plan from cu_nodes
+// and prefix_len (all derive the same one); the combine kernel reads the
+// per-group table the attention kernel leaves in the workspace.
+
+struct PlanItem {
+  int group;  // -1: nothing for this item
+  int j, k;   // the item is the j-th of the group's k (k = 0: the group has no work)
+  int first;  // the group's first item
+};
+
+__device__ __forceinline__ int plan_tiles(const AttnArgs& a, int q) {
+  const int b = q / (a.Hkv * a.rb_count);
+  const int rb = q % a.rb_count;
+  const int node0 = a.cu_nodes[b];
+  const int nn = a.cu_nodes[b + 1] - node0;
+  const int P = a.prefix_len[b];
+  if (node0 < 0 || nn < 1 || nn > a.max_nodes || node0 + nn > a.T || P < 0 || P > a.max_prefix) {
+    flag_error(a.err, PF_DEVERR_BOUNDS);
+    return 0;
+  }
+  if (rb * a.nb >= nn) return 0;
+  return (P + kBN - 1) / kBN + (nn + kBN - 1) / kBN;
+}
+
+// The plan's per-group table in the workspace, after the partials: (first
+// item, items, first node, rows) of every group, written by the attention
+// kernel for the combine kernel.
+__device__ __forceinline__ int4* plan_table(const AttnArgs& a) {
+  return reinterpret_cast<int4*>(reinterpret_cast<uint8_t*>(a.ws) +
+                                 (size_t)a.items * a.bm * (a.D + 8) * 2);
+}
+
+// Warp-collective (all 32 lanes, warp-uniform arguments): the plan entry
+// of item `item`, and in *grp that of group `group` (j = 0) if group >= 0.
+static __device__ __noinline__ PlanItem balanced_plan(const AttnArgs& a, int item, int group,
+                                                      PlanItem* grp) {
+  const int lane = threadIdx.x & 31;
+  const int n_groups = a.B * a.Hkv * a.rb_count;  // <= kPlanMaxGroups and <= items (host)
+  constexpr int kPer = kPlanMaxGroups / 32;
+  const int n_chunks = (n_groups + 31) / 32;
+  int t[kPer];
+  int U = 0, n_active = 0, t_max = 0;
+#pragma unroll
+  for (int s = 0; s < kPer; ++s) {
+    const int q = lane + 32 * s;
+    t[s] = q < n_groups ? plan_tiles(a, q) : 0;
+    U += t[s];
+    n_active += t[s] > 0 ? 1 : 0;
+    t_max = max(t_max, t[s]);
+  }
+  U = __reduce_add_sync(0xffffffffu, U);
+  n_active = __reduce_add_sync(0xffffffffu, n_active);
+  t_max = __reduce_max_sync(0xffffffffu, t_max);
+  PlanItem r = {-1, 0, 0, 0};
+  if (group >= 0) *grp = PlanItem{group, 0, 0, 0};
+  if (U == 0) return r;
+  // T in [lo, hi]: count(T) >= U / T exceeds items below lo, and
+  // count(T) <= U / T + n_active fits at hi (as does count(t_max) = n_active).
+  int hi = t_max;
+  if (a.items > n_active) hi = min(hi, (U + (a.items - n_active) - 1) / (a.items - n_active));
+  int lo = min(hi, max(1, (U + a.items - 1) / a.items));
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    int c = 0;
+#pragma unroll
+    for (int s = 0; s < kPer; ++s)
+      if (s < n_chunks) c += (t[s] + mid - 1) / mid;
+    c = __reduce_add_sync(0xffffffffu, c);
+    if (c <= a.items) hi = mid;
+    else lo = mid + 1;
+  }
+  const int T = lo;
+  int base = 0;
+#pragma unroll
+  for (int s = 0; s < kPer; ++s) {
+    if (s >= n_chunks) break;
+    const int q = lane + 32 * s;
+    const int k = (t[s] + T - 1) / T;
+    int incl = k;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    const int first = base + incl - k;
+    const unsigned mi = __ballot_sync(0xffffffffu, q < n_groups && k > 0 && item >= first &&
+                                                       item < first + k);
+    if (mi) {
+      const int src = __ffs(mi) - 1;
+      r.group = __shfl_sync(0xffffffffu, q, src);
+      r.k = __shfl_sync(0xffffffffu, k, src);
+      r.first = __shfl_sync(0xffffffffu, first, src);
+      r.j = item - r.first;
+    }
+    if (group >= 0 && group / 32 == s) {
+      const int src = group % 32;
+      grp->k = __shfl_sync(0xffffffffu, k, src);
+      grp->first = __shfl_sync(0xffffffffu, first, src);
+    }
+    base += __shfl_sync(0xffffffffu, incl, 31);
+  }
+  return r;
 }
 
 // Local half of the split-KV merge: this CTA (rank `split`) owns rows

@@ -22,6 +22,12 @@ struct AttnArgs {
   int rb_count;    // row blocks per (sequence, KV head)
   int splits;      // CTAs of one cluster, each taking a slice of the KV tiles
   int flags;       // PF_ATTN_* flags
+  // Balanced batch mode (tcgen05 kernel, splits == 1, no cluster): `items`
+  // CTAs share the groups' tiles in proportion to their lengths (see
+  // balanced_plan); a group spread over several CTAs leaves normalised
+  // partials in `ws` ([items][bm][D + 8] halves) for the combine kernel.
+  int items;       // 0 = off
+  void* ws;
   float scale_log2;  // softmax scale * log2(e)
   float scale;
   const int32_t* cu_nodes;
@@ -55,6 +61,14 @@ int attention_bf16_smem_bytes(int D, int bm);
 bool attention_cluster_fits(int D, int bm, int cluster);
 // tcgen05 variant (bf16, D = 128, a.bm = 128 or 256 query rows per CTA).
 cudaError_t launch_attention_tc(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl);
+// Merge of the balanced batch mode's partials (launched after the tcgen05
+// kernel when a.items > 0).
+cudaError_t launch_attention_combine(const AttnArgs& a, cudaStream_t s, bool pdl);
+// Groups (sequence, KV head, row block) the balanced batch mode's plan can
+// hold (8 per lane of a warp).
+constexpr int kPlanMaxGroups = 256;
+// Bytes of a.ws for the balanced batch mode with `items` CTAs of a.bm rows.
+size_t attention_balanced_ws_bytes(int items, int bm, int D);
 // How many clusters of `cluster` CTAs of the tcgen05 kernel fit at once.
 // rows_per_cta: 128 (one softmax warpgroup) or 256 (two).
 int attention_tc_max_active_clusters(int cluster, int rows_per_cta);

@@ -46,11 +46,15 @@ def host_bits(t: torch.Tensor) -> np.ndarray:
 
 class VerifyStep:
     """One workload's device state.  ``layers`` may restrict the layer count
-    (parity tests use a few layers of a full-size workload)."""
+    (parity tests use a few layers of a full-size workload).  ``balanced``
+    gives the attention calls a workspace, with which a batch of several
+    sequences is dealt out to the SMs in proportion to their lengths."""
 
     def __init__(self, w: I.Workload, batch: I.Batch, tokens: np.ndarray, layers: int = None,
-                 device: str = "cuda", weight: np.ndarray = None, hidden: np.ndarray = None):
+                 device: str = "cuda", weight: np.ndarray = None, hidden: np.ndarray = None,
+                 balanced: bool = True):
         self.w, self.batch = w, batch
+        self.balanced = balanced
         self.L = layers if layers is not None else w.layers
         self.device = device
         td = _torch_dtype(w.dtype)
@@ -172,6 +176,14 @@ class VerifyStep:
             # cache tiles while the previous layer is still finishing.
             d.flags = pb.PF_ATTN_EARLY_PREFETCH if l > 0 else 0
             self.attn_descs.append(d)
+        # one attention workspace serves every layer (calls run in stream order)
+        self.attn_ws_bytes = (pb.pf_verify_attention_workspace_size(self.attn_descs[0])
+                              if self.balanced else 0)
+        self.attn_ws = (torch.empty((self.attn_ws_bytes,), dtype=torch.uint8, device=self.device)
+                        if self.attn_ws_bytes else None)
+        for d in self.attn_descs:
+            d.workspace = self.attn_ws.data_ptr() if self.attn_ws is not None else None
+            d.workspace_bytes = self.attn_ws_bytes
         d = pb.pf_lm_desc()
         d.dtype, d.batch, d.hidden, d.vocab = dt, w.batch, w.hidden, w.vocab
         d.total_nodes, d.max_nodes = self.T, self.max_nodes
@@ -221,7 +233,8 @@ class VerifyStep:
         pb.pf_kv_commit(self.commit_desc, s)
 
     def launches_per_step(self) -> int:
-        return self.L + 2
+        # the attention call launches a second (merge) kernel when it has a workspace
+        return self.L * (2 if self.attn_ws is not None else 1) + 2
 
     # ------------------------------------------------------------------ results
     def results(self) -> dict:

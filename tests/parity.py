@@ -32,7 +32,8 @@ def values(x: np.ndarray, dtype: str) -> np.ndarray:
 class Case:
     """A generated workload, the oracle's greedy predictions and a device step."""
 
-    def __init__(self, w: I.Workload, seed: int = 0, layers: int = None, batch: I.Batch = None):
+    def __init__(self, w: I.Workload, seed: int = 0, layers: int = None, batch: I.Batch = None,
+                 balanced: bool = True):
         self.w = w
         self.batch = batch if batch is not None else I.make_batch(w, seed)
         self.L = layers if layers is not None else w.layers
@@ -43,7 +44,7 @@ class Case:
         del lg
         self.tokens = I.plant_tokens(self.batch, self.o_argmax)
         self.vs = VerifyStep(w, self.batch, self.tokens, layers=self.L,
-                             weight=self.weight, hidden=self.hidden)
+                             weight=self.weight, hidden=self.hidden, balanced=balanced)
 
     # --------------------------------------------------------------- attention
     def oracle_attention(self, layer: int, seq: int, nodes=None) -> np.ndarray:

@@ -49,6 +49,7 @@ int main(void) {
          offsetof(pf_key_desc, key_out), sizeof(pf_retrieval_desc),
          offsetof(pf_retrieval_desc, similarity));
   printf("%zu %zu\n", sizeof(pf_prefix_desc), offsetof(pf_prefix_desc, cache_len));
+  printf("%zu %zu\n", offsetof(pf_attn_desc, workspace), offsetof(pf_attn_desc, workspace_bytes));
   return 0;
 }
 '''
@@ -66,7 +67,8 @@ int main(void) {
             pb.pf_shift_desc.cache_layer_stride.offset, C.sizeof(pb.pf_key_desc),
             pb.pf_key_desc.key_out.offset, C.sizeof(pb.pf_retrieval_desc),
             pb.pf_retrieval_desc.similarity.offset,
-            C.sizeof(pb.pf_prefix_desc), pb.pf_prefix_desc.cache_len.offset]
+            C.sizeof(pb.pf_prefix_desc), pb.pf_prefix_desc.cache_len.offset,
+            pb.pf_attn_desc.workspace.offset, pb.pf_attn_desc.workspace_bytes.offset]
     assert got == want
 
 

@@ -116,6 +116,47 @@ def test_two_block_kernel_on_many_rows(name, monkeypatch):
         c.check_attention(0, s)
 
 
+@pytest.mark.parametrize("balanced", [False, True])
+def test_batch_work_split(balanced):
+    """Eight sequences with prefixes from 100 to 700 rows, with an attention
+    workspace (tiles dealt out to the SMs in proportion to each sequence's
+    length, partials merged by a second kernel) and without one (every
+    sequence and KV head gets the same cluster)."""
+    c = Case(SMALL["7b-batch8-paged-small"], seed=11, balanced=balanced)
+    assert (c.vs.attn_ws is not None) == balanced
+    assert c.vs.launches_per_step() == c.L * (2 if balanced else 1) + 2
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for s in range(c.w.batch):
+        c.check_attention(0, s)
+    c.check_lmhead(res)
+    c.check_commit(res)
+
+
+def test_attention_workspace_contract():
+    """The workspace query and the checks on a given workspace."""
+    from paper_2609_32166_gb300 import binding as pb
+    c = Case(SMALL["7b-batch8-paged-small"], seed=12)
+    d = c.vs.attn_descs[0]
+    need = pb.pf_verify_attention_workspace_size(d)
+    assert need > 0 and need == c.vs.attn_ws_bytes
+    d.workspace_bytes = need - 1
+    with pytest.raises(pb.PfError) as e:
+        pb.pf_verify_attention(d, 0)
+    assert e.value.status == pb.PF_ERR_WORKSPACE
+    d.workspace_bytes = need
+    d.workspace = c.vs.attn_ws.data_ptr() + 8
+    with pytest.raises(pb.PfError) as e:
+        pb.pf_verify_attention(d, 0)
+    assert e.value.status == pb.PF_ERR_ALIGN
+    d.workspace = c.vs.attn_ws.data_ptr()
+    # a single sequence needs none (its KV heads and row blocks share clusters)
+    one = Case(SMALL["7b-tree64-small"], seed=12)
+    assert pb.pf_verify_attention_workspace_size(one.vs.attn_descs[0]) == 0
+    assert one.vs.attn_ws is None
+
+
 def test_mixed_tree_sizes():
     """Sequences of 1, 17 and 128 nodes in one batch (variable cu_nodes)."""
     w = I.scaled(W["7b-bf16-batch8-paged"], layers=1, batch=3, prefix=(50, 400), nodes=128,

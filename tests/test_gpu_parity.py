@@ -157,6 +157,24 @@ def test_attention_workspace_contract():
     assert one.vs.attn_ws is None
 
 
+def test_batch_beyond_balanced_groups():
+    """More (sequence, KV head) groups than SMs: no workspace is asked for
+    and every sequence goes through the cluster path."""
+    import torch as _t
+    sms = _t.cuda.get_device_properties(0).multi_processor_count
+    w = I.scaled(W["7b-bf16-batch8-paged"], layers=1, batch=sms // 4 + 2, prefix=(20, 150),
+                 nodes=6, vocab=300, hidden=64)
+    c = Case(w, seed=13)
+    assert c.vs.attn_ws is None
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for s in sorted({0, 1, w.batch // 2, w.batch - 1}):
+        c.check_attention(0, s)
+    c.check_lmhead(res)
+    c.check_commit(res)
+
+
 def test_mixed_tree_sizes():
     """Sequences of 1, 17 and 128 nodes in one batch (variable cu_nodes)."""
     w = I.scaled(W["7b-bf16-batch8-paged"], layers=1, batch=3, prefix=(50, 400), nodes=128,

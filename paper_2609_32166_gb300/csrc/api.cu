@@ -149,11 +149,52 @@ int tc_max_active_clusters(int cluster, int bm) {
   return c - 1;
 }
 
-// The tcgen05 kernel serves bf16 with D = 128 (PF_ATTN_IMPL=mma selects the
+int tc2_max_active_clusters(int cluster) {
+  static std::atomic<int> cache[64][17];
+  int dev = 0;
+  cudaGetDevice(&dev);
+  std::atomic<int>& slot = cache[dev & 63][cluster];
+  int c = slot.load(std::memory_order_acquire);
+  if (c == 0) {
+    c = std::max(1, pf::attention_tc2_max_active_clusters(cluster)) + 1;
+    slot.store(c, std::memory_order_release);
+  }
+  return c - 1;
+}
+
+// The tcgen05 kernels serve bf16 with D = 128 (PF_ATTN_IMPL=mma selects the
 // mma.sync kernel instead).
 bool use_tc_attention(const pf::AttnArgs& a) {
   const char* e = getenv("PF_ATTN_IMPL");
   return a.D == 128 && !(e && strcmp(e, "mma") == 0);
+}
+
+// 128-token tiles (attn_tc2_kernel) for 128-row CTAs outside the balanced
+// batch mode once a CTA holds at least four 64-token tiles: per tile the
+// wider S MMA halves the UMMA instructions per key, while a CTA with one or
+// two tiles gains more from starting on a first, smaller tile (2B chain:
+// 6.70 us per layer with 64-token tiles, 6.95 with 128).  PF_ATTN_IMPL=tc64
+// or tc128 forces either.  `max_tiles` counts 64-token tiles.
+bool use_tc2_attention(const pf::AttnArgs& a, int max_prefix_len) {
+  if (!use_tc_attention(a) || a.bm != 128 || a.items != 0) return false;
+  const char* e = getenv("PF_ATTN_IMPL");
+  if (e && strcmp(e, "tc64") == 0) return false;
+  if (e && strcmp(e, "tc128") == 0) return true;
+  const int max_tiles = (max_prefix_len + 63) / 64 + (a.max_nodes + 63) / 64;
+  return (max_tiles + a.splits - 1) / a.splits >= 4;
+}
+
+// Splits for attn_tc2_kernel: the widest even cluster, at most the tile
+// count, whose clusters all fit on the GPU at once.
+void choose_tc2_splits(pf::AttnArgs& a, int max_prefix_len) {
+  const int max_tiles = (max_prefix_len + 127) / 128 + (a.max_nodes + 127) / 128;
+  const int groups = a.B * a.Hkv * a.rb_count;
+  int splits = std::min(16, max_tiles);
+  if (splits > 1) splits &= ~1;
+  for (; splits > 1; splits -= 2)
+    if (tc2_max_active_clusters(splits) >= groups) break;
+  if (const char* e = getenv("PF_ATTN_SPLITS")) splits = std::max(1, std::min(16, atoi(e)));
+  a.splits = std::max(1, splits);
 }
 
 void choose_attention_shape(pf::AttnArgs& a, int max_prefix_len, int sms) {
@@ -355,35 +396,6 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
     return fail(PF_ERR_SHAPE, "%s: unknown flags 0x%x", who, d->flags);
   a.flags = d->flags;
   choose_attention_shape(a, d->max_prefix_len, sms);
-  pf::AttnMaps m;
-  const cuuint64_t es = 2;
-  {
-    cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)a.Hq, (cuuint64_t)a.T};
-    cuuint64_t str[2] = {D * es, (cuuint64_t)a.Hq * D * es};
-    cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)a.nb};  // nb * G <= bm rows
-    if ((st = make_map(&m.q, 3, d->q, dims, str, box, "q")) != PF_OK) return st;
-  }
-  {
-    cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)a.Hkv, (cuuint64_t)a.T};
-    cuuint64_t str[2] = {D * es, (cuuint64_t)a.Hkv * D * es};
-    cuuint32_t box[3] = {64, 1, 64};
-    if ((st = make_map(&m.tk, 3, d->tree_k, dims, str, box, "tree_k")) != PF_OK) return st;
-    if ((st = make_map(&m.tv, 3, d->tree_v, dims, str, box, "tree_v")) != PF_OK) return st;
-  }
-  if (a.layout == PF_KV_CONTIGUOUS) {
-    cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)a.max_seq, (cuuint64_t)a.B * a.Hkv};
-    cuuint64_t str[2] = {D * es, (cuuint64_t)a.max_seq * D * es};
-    cuuint32_t box[3] = {64, 64, 1};
-    if ((st = make_map(&m.ck, 3, d->cache.k, dims, str, box, "cache.k")) != PF_OK) return st;
-    if ((st = make_map(&m.cv, 3, d->cache.v, dims, str, box, "cache.v")) != PF_OK) return st;
-  } else {
-    cuuint64_t dims[4] = {(cuuint64_t)D, PF_PAGE_SIZE, (cuuint64_t)a.Hkv,
-                          (cuuint64_t)a.num_pages};
-    cuuint64_t str[3] = {D * es, PF_PAGE_SIZE * D * es, (cuuint64_t)a.Hkv * PF_PAGE_SIZE * D * es};
-    cuuint32_t box[4] = {64, PF_PAGE_SIZE, 1, 1};
-    if ((st = make_map(&m.ck, 4, d->cache.k, dims, str, box, "cache.k")) != PF_OK) return st;
-    if ((st = make_map(&m.cv, 4, d->cache.v, dims, str, box, "cache.v")) != PF_OK) return st;
-  }
   if (d->workspace) {
     const int items = balanced_items(a, sms);
     if (items > 0) {
@@ -397,8 +409,41 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
       a.ws = d->workspace;
     }
   }
-  cudaError_t e = use_tc_attention(a) ? pf::launch_attention_tc(a, m, s, pdl_enabled())
-                                      : pf::launch_attention_bf16(a, m, s, sms, pdl_enabled());
+  const bool tc2 = use_tc2_attention(a, d->max_prefix_len);
+  if (tc2) choose_tc2_splits(a, d->max_prefix_len);
+  const cuuint32_t tile_rows = tc2 ? 128 : 64;  // K/V tile height of the chosen kernel
+  pf::AttnMaps m;
+  const cuuint64_t es = 2;
+  {
+    cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)a.Hq, (cuuint64_t)a.T};
+    cuuint64_t str[2] = {D * es, (cuuint64_t)a.Hq * D * es};
+    cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)a.nb};  // nb * G <= bm rows
+    if ((st = make_map(&m.q, 3, d->q, dims, str, box, "q")) != PF_OK) return st;
+  }
+  {
+    cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)a.Hkv, (cuuint64_t)a.T};
+    cuuint64_t str[2] = {D * es, (cuuint64_t)a.Hkv * D * es};
+    cuuint32_t box[3] = {64, 1, tile_rows};
+    if ((st = make_map(&m.tk, 3, d->tree_k, dims, str, box, "tree_k")) != PF_OK) return st;
+    if ((st = make_map(&m.tv, 3, d->tree_v, dims, str, box, "tree_v")) != PF_OK) return st;
+  }
+  if (a.layout == PF_KV_CONTIGUOUS) {
+    cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)a.max_seq, (cuuint64_t)a.B * a.Hkv};
+    cuuint64_t str[2] = {D * es, (cuuint64_t)a.max_seq * D * es};
+    cuuint32_t box[3] = {64, tile_rows, 1};
+    if ((st = make_map(&m.ck, 3, d->cache.k, dims, str, box, "cache.k")) != PF_OK) return st;
+    if ((st = make_map(&m.cv, 3, d->cache.v, dims, str, box, "cache.v")) != PF_OK) return st;
+  } else {
+    cuuint64_t dims[4] = {(cuuint64_t)D, PF_PAGE_SIZE, (cuuint64_t)a.Hkv,
+                          (cuuint64_t)a.num_pages};
+    cuuint64_t str[3] = {D * es, PF_PAGE_SIZE * D * es, (cuuint64_t)a.Hkv * PF_PAGE_SIZE * D * es};
+    cuuint32_t box[4] = {64, PF_PAGE_SIZE, 1, 1};
+    if ((st = make_map(&m.ck, 4, d->cache.k, dims, str, box, "cache.k")) != PF_OK) return st;
+    if ((st = make_map(&m.cv, 4, d->cache.v, dims, str, box, "cache.v")) != PF_OK) return st;
+  }
+  cudaError_t e = tc2 ? pf::launch_attention_tc2(a, m, s, pdl_enabled())
+                 : use_tc_attention(a) ? pf::launch_attention_tc(a, m, s, pdl_enabled())
+                                       : pf::launch_attention_bf16(a, m, s, sms, pdl_enabled());
   if (e == cudaSuccess && a.items > 0) e = pf::launch_attention_combine(a, s, pdl_enabled());
   return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
 }

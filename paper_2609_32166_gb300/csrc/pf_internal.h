@@ -61,6 +61,11 @@ int attention_bf16_smem_bytes(int D, int bm);
 bool attention_cluster_fits(int D, int bm, int cluster);
 // tcgen05 variant (bf16, D = 128, a.bm = 128 or 256 query rows per CTA).
 cudaError_t launch_attention_tc(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl);
+// tcgen05 variant with 128-token K/V tiles and P in tensor memory (bf16,
+// D = 128, a.bm = 128, cluster split-KV only); its tensor maps hold
+// 128-row cache boxes and 128-node proposal boxes.
+cudaError_t launch_attention_tc2(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl);
+int attention_tc2_max_active_clusters(int cluster);
 // Merge of the balanced batch mode's partials (launched after the tcgen05
 // kernel when a.items > 0).
 cudaError_t launch_attention_combine(const AttnArgs& a, cudaStream_t s, bool pdl);

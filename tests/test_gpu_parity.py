@@ -103,6 +103,48 @@ def test_mma_sync_kernel(name, monkeypatch):
         c.check_attention(0, s)
 
 
+@pytest.mark.parametrize("name", ["2b-chain16-small", "7b-tree64-small", "7b-32k-tree128-small"])
+def test_64_token_tile_kernel(name, monkeypatch):
+    """The tcgen05 kernel with 64-token tiles (PF_ATTN_IMPL=tc64), which the
+    balanced batch mode and 256-row CTAs use, on 128-row CTAs too."""
+    monkeypatch.setenv("PF_ATTN_IMPL", "tc64")
+    c = Case(SMALL[name], seed=7)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for l in range(c.L):
+        c.check_attention(l, 0)
+
+
+@pytest.mark.parametrize("name", ["2b-chain16-small", "7b-tree64-small", "7b-32k-tree128-small"])
+def test_128_token_tile_kernel(name, monkeypatch):
+    """The tcgen05 kernel with 128-token tiles and P in tensor memory
+    (PF_ATTN_IMPL=tc128) also where a CTA holds few tiles."""
+    monkeypatch.setenv("PF_ATTN_IMPL", "tc128")
+    c = Case(SMALL[name], seed=9)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for l in range(c.L):
+        c.check_attention(l, 0)
+
+
+EDGE_128 = {k: EDGE[k] for k in ("root-only", "empty-prefix", "65-nodes", "g16-tiny-vocab",
+                                 "two-blocks-one-tile")}
+
+
+@pytest.mark.parametrize("name", sorted(EDGE_128))
+def test_128_token_tile_kernel_edges(name, monkeypatch):
+    monkeypatch.setenv("PF_ATTN_IMPL", "tc128")
+    c = Case(EDGE_128[name], seed=5)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for l in range(c.L):
+        for s in range(c.w.batch):
+            c.check_attention(l, s)
+
+
 @pytest.mark.parametrize("name", ["7b-tree64-small", "7b-32k-tree128-small"])
 def test_two_block_kernel_on_many_rows(name, monkeypatch):
     """Two 128-row blocks per CTA (PF_ATTN_BM=256) where a KV head has more

@@ -31,29 +31,35 @@ namespace pf {
 namespace {
 
 constexpr int kW = 128;              // tokens per K/V tile
-constexpr int kW2Stages = 2;
 constexpr int kW2Threads = 192;      // producer, MMA, one softmax warpgroup
 constexpr uint32_t kW2TmemCols = 512;
 constexpr uint32_t kColO = 256, kColP = 384;
 constexpr float kW2RescaleLog2 = 8.f;
 
+// STAGES = 2: the merge inbox has its own space, so peers may send while
+// this CTA still works.  STAGES = 3: no room; the inbox takes the idle ring
+// from its second stage on, and peers send only after every CTA of the
+// cluster has left its loop.  Partial rows are staged at the ring's start.
+template <int STAGES>
 struct W2Smem {
   static constexpr int D = 128;
   static constexpr int kHalfBytes = kW * 128;             // 128 tokens x 64 columns
   static constexpr int kTileBytes = 2 * kHalfBytes;       // one K or V tile
   static constexpr int kStageBytes = 2 * kTileBytes;      // K + V
-  static constexpr int kQOff = kW2Stages * kStageBytes;
+  static constexpr int kQOff = STAGES * kStageBytes;
   static constexpr int kQHalf = 128 * 128;                // 128 rows x 64 columns
-  static constexpr int kInboxOff = kQOff + 2 * kQHalf;
-  // merge inbox and staging: as in attn_tc_kernel (kWG = 1)
+  static constexpr int kQEnd = kQOff + 2 * kQHalf;
   static constexpr int kInboxSlots = 128 + 16;
   static constexpr int kPitch = D + 8;                    // halves
   static constexpr int kRowBytes = kPitch * 2;
-  static constexpr int kBarOff = kInboxOff + kInboxSlots * kRowBytes;
-  // kv_full[2] kv_empty[2] q_full s_full[2] s_empty[2] p_full[2] pv_done[2] inbox
-  static constexpr int kNumBars = 2 * kW2Stages + 1 + 8 + 1;
+  static constexpr bool kLateInbox = STAGES > 2;
+  static constexpr int kInboxOff = kLateInbox ? kStageBytes : kQEnd;
+  static constexpr int kBarOff = kLateInbox ? kQEnd : kInboxOff + kInboxSlots * kRowBytes;
+  // kv_full[S] kv_empty[S] q_full s_full[2] s_empty[2] p_full[2] pv_done[2] inbox
+  static constexpr int kNumBars = 2 * STAGES + 1 + 8 + 1;
   static constexpr int kTotal = kBarOff + kNumBars * 8 + 16;
-  static_assert(128 * kRowBytes <= kQOff, "staged rows fit in the idle ring");
+  static_assert(128 * kRowBytes <= kStageBytes, "staged rows fit in the ring's first stage");
+  static_assert(!kLateInbox || kInboxOff + kInboxSlots * kRowBytes <= kQOff, "inbox fits in the ring");
   static_assert(kTotal + 1024 <= 232448, "shared memory budget");
 };
 
@@ -88,7 +94,7 @@ __device__ __forceinline__ void w2_issue_tile(const AttnArgs& a, const CUtensorM
                                               const CUtensorMap* tm_tv, uint8_t* stage,
                                               uint32_t bar, int t, int n_ptiles, int b, int g,
                                               int node0, int P, Pages8 pg) {
-  using S = W2Smem;
+  using S = W2Smem<2>;  // the tile layout does not depend on the ring depth
   uint8_t* sk = stage;
   uint8_t* sv = stage + S::kTileBytes;
   if (t < n_ptiles) {
@@ -138,13 +144,15 @@ __device__ __forceinline__ void umma_bf16_tmem_a(uint32_t d_tmem, uint32_t a_tme
       : "memory");
 }
 
+template <int STAGES>
 __global__ void __launch_bounds__(kW2Threads, 1)
     attn_tc2_kernel(const __grid_constant__ CUtensorMap tm_q,
                     const __grid_constant__ CUtensorMap tm_tk,
                     const __grid_constant__ CUtensorMap tm_tv,
                     const __grid_constant__ CUtensorMap tm_ck,
                     const __grid_constant__ CUtensorMap tm_cv, const AttnArgs a) {
-  using S = W2Smem;
+  using S = W2Smem<STAGES>;
+  constexpr int kW2Stages = STAGES;
   constexpr int D = 128;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
@@ -247,8 +255,9 @@ __global__ void __launch_bounds__(kW2Threads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  // peers may signal this CTA's inbox barrier once it is initialised
-  if (nsplit > 1) cluster_arrive_release();
+  // peers may signal this CTA's inbox barrier once it is initialised (and,
+  // with the inbox in the ring, once the ring is idle: after the loop)
+  if (!S::kLateInbox && nsplit > 1) cluster_arrive_release();
   pdl_launch_dependents();
 
   float m_ref = -INFINITY, l = 0.f;   // softmax threads: running max (log2) and sum of their row
@@ -503,6 +512,12 @@ __global__ void __launch_bounds__(kW2Threads, 1)
   const int per = (rows + nsplit - 1) / nsplit;
   const int cnt_mine = max(0, min(per, rows - split * per));
   __half* stage_rows = reinterpret_cast<__half*>(smem);
+  if (S::kLateInbox) {
+    // every PV of this CTA has completed (the softmax threads waited for the
+    // last one): the ring is idle, so peers may now fill the inbox it holds
+    __syncthreads();
+    cluster_arrive_release();
+  }
   if (tid == 0)
     mbar_arrive_expect_tx(smem_u32(inbox_full), (uint32_t)(nsplit * cnt_mine * S::kRowBytes));
   if (has_row) {
@@ -553,13 +568,17 @@ __global__ void __launch_bounds__(kW2Threads, 1)
 
 }  // namespace
 
-static int tc2_smem_bytes() { return W2Smem::kTotal + 1024; }
+template <int STAGES>
+static int tc2_smem_bytes() {
+  return W2Smem<STAGES>::kTotal + 1024;
+}
 
-int attention_tc2_max_active_clusters(int cluster) {
-  const int smem = tc2_smem_bytes();
+template <int STAGES>
+static int tc2_max_active_clusters_impl(int cluster) {
+  const int smem = tc2_smem_bytes<STAGES>();
   static DeviceMemo limit;
-  if (ensure_smem_limit((const void*)attn_tc2_kernel, smem, limit) != cudaSuccess) return 0;
-  if (cluster > 8 && cudaFuncSetAttribute(attn_tc2_kernel,
+  if (ensure_smem_limit((const void*)attn_tc2_kernel<STAGES>, smem, limit) != cudaSuccess) return 0;
+  if (cluster > 8 && cudaFuncSetAttribute(attn_tc2_kernel<STAGES>,
                                           cudaFuncAttributeNonPortableClusterSizeAllowed,
                                           1) != cudaSuccess)
     return 0;
@@ -575,26 +594,43 @@ int attention_tc2_max_active_clusters(int cluster) {
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, attn_tc2_kernel, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, attn_tc2_kernel<STAGES>, &cfg) != cudaSuccess) {
     cudaGetLastError();
     return 0;
   }
   return n;
 }
 
-cudaError_t launch_attention_tc2(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl) {
-  const int smem = tc2_smem_bytes();
+template <int STAGES>
+static cudaError_t launch_tc2(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl) {
+  const int smem = tc2_smem_bytes<STAGES>();
   static DeviceMemo limit;
   static DeviceMemo nonportable;
-  cudaError_t e = ensure_smem_limit((const void*)attn_tc2_kernel, smem, limit);
+  cudaError_t e = ensure_smem_limit((const void*)attn_tc2_kernel<STAGES>, smem, limit);
   if (e != cudaSuccess) return e;
   if (a.splits > 8) {
-    e = ensure_nonportable_cluster((const void*)attn_tc2_kernel, nonportable);
+    e = ensure_nonportable_cluster((const void*)attn_tc2_kernel<STAGES>, nonportable);
     if (e != cudaSuccess) return e;
   }
   const dim3 grid(a.B * a.Hkv * a.rb_count * a.splits);
-  return launch_ex(attn_tc2_kernel, grid, dim3(kW2Threads), smem, s, a.splits, pdl, m.q, m.tk,
-                   m.tv, m.ck, m.cv, a);
+  return launch_ex(attn_tc2_kernel<STAGES>, grid, dim3(kW2Threads), smem, s, a.splits, pdl, m.q,
+                   m.tk, m.tv, m.ck, m.cv, a);
+}
+
+// Ring depth: 3 stages (inbox in the ring, peers send after every CTA of
+// the cluster has left its loop) unless PF_ATTN_W2_STAGES=2.
+static int tc2_stages() {
+  const char* e = getenv("PF_ATTN_W2_STAGES");
+  return e && atoi(e) == 2 ? 2 : 3;
+}
+
+int attention_tc2_max_active_clusters(int cluster) {
+  return tc2_stages() == 2 ? tc2_max_active_clusters_impl<2>(cluster)
+                           : tc2_max_active_clusters_impl<3>(cluster);
+}
+
+cudaError_t launch_attention_tc2(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl) {
+  return tc2_stages() == 2 ? launch_tc2<2>(a, m, s, pdl) : launch_tc2<3>(a, m, s, pdl);
 }
 
 }  // namespace pf

@@ -116,11 +116,14 @@ def test_64_token_tile_kernel(name, monkeypatch):
         c.check_attention(l, 0)
 
 
+@pytest.mark.parametrize("stages", ["2", "3"])
 @pytest.mark.parametrize("name", ["2b-chain16-small", "7b-tree64-small", "7b-32k-tree128-small"])
-def test_128_token_tile_kernel(name, monkeypatch):
+def test_128_token_tile_kernel(name, stages, monkeypatch):
     """The tcgen05 kernel with 128-token tiles and P in tensor memory
-    (PF_ATTN_IMPL=tc128) also where a CTA holds few tiles."""
+    (PF_ATTN_IMPL=tc128) also where a CTA holds few tiles, with both ring
+    depths (3 stages: the merge inbox in the idle ring)."""
     monkeypatch.setenv("PF_ATTN_IMPL", "tc128")
+    monkeypatch.setenv("PF_ATTN_W2_STAGES", stages)
     c = Case(SMALL[name], seed=9)
     c.vs.step()
     res = c.vs.results()

@@ -44,6 +44,9 @@ def parse():
     p.add_argument("--steps", type=int, default=400)
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    p.add_argument("--layers", type=int, default=None,
+                   help="profiling aid: the step over the workload's first N layers only "
+                        "(recorded in the line's config; default: every layer)")
     p.add_argument("--seed", type=int, default=0)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -169,6 +172,8 @@ def cpu_worker(spec: dict) -> dict:
     from paper_2609_32166_gb300 import inputs as I
 
     w = I.WORKLOADS[spec["workload"]]
+    if spec.get("layers"):
+        w = I.scaled(w, layers=spec["layers"])
     batch = I.make_batch(w, spec["seed"])
     f = (lambda x: I.bf16_bits_to_f32(x)) if w.dtype == "bf16" else (lambda x: x)
     hidden = f(I.hidden_states(w, batch))
@@ -340,11 +345,13 @@ def main():
     cpu_base = None
     from paper_2609_32166_gb300 import inputs as I
     w = I.WORKLOADS[args.workload]
+    if args.layers is not None:
+        w = I.scaled(w, layers=max(1, min(args.layers, w.layers)))
     nl_cpu = 1
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         # before any CUDA call in this process
         cpu_base = run_cpu_worker(dict(workload=args.workload, seed=args.seed,
-                                       layers_sample=nl_cpu, budget_s=12.0))
+                                       layers_sample=nl_cpu, budget_s=12.0, layers=w.layers))
 
     import torch
     import torch.distributed as dist

@@ -6,7 +6,8 @@
 // key of 64-token tiles.  The shared memory that the wider tiles need comes
 // from keeping P in tensor memory:
 //
-//   warp 0     TMA producer: Q once, then K/V tiles (64 KB) into a 2-stage ring
+//   warp 0     TMA producer: Q once, then K/V tiles (64 KB) into a ring of
+//              STAGES (3 by default) stages
 //   warp 1     TMEM owner and MMA issuer (one thread):
 //                S_i  = Q K_i^T   M=128, N=128, K=D, A and B in smem -> S[i % 2]
 //                O   += P_i V_i   M=128, N=D,  K=128, A = P in TMEM    -> O

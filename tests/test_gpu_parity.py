@@ -148,6 +148,23 @@ def test_128_token_tile_kernel_edges(name, monkeypatch):
             c.check_attention(l, s)
 
 
+@pytest.mark.parametrize("stages", ["2", "3"])
+def test_128_token_tile_kernel_paged(stages, monkeypatch):
+    """Paged cache (eight 16-token pages per 128-token tile, random page
+    order, ragged last pages), two sequences with 128-node trees, on the
+    128-token kernel (no workspace, so no balanced batch mode)."""
+    monkeypatch.setenv("PF_ATTN_IMPL", "tc128")
+    monkeypatch.setenv("PF_ATTN_W2_STAGES", stages)
+    c = Case(EDGE["256-rows-paged"], seed=10, balanced=False)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for s in range(c.w.batch):
+        c.check_attention(0, s)
+    c.check_lmhead(res)
+    c.check_commit(res)
+
+
 @pytest.mark.parametrize("name", ["7b-tree64-small", "7b-32k-tree128-small"])
 def test_two_block_kernel_on_many_rows(name, monkeypatch):
     """Two 128-row blocks per CTA (PF_ATTN_BM=256) where a KV head has more
@@ -220,8 +237,12 @@ def test_batch_beyond_balanced_groups():
     c.check_commit(res)
 
 
-def test_mixed_tree_sizes():
-    """Sequences of 1, 17 and 128 nodes in one batch (variable cu_nodes)."""
+@pytest.mark.parametrize("impl", ["default", "tc128"])
+def test_mixed_tree_sizes(impl, monkeypatch):
+    """Sequences of 1, 17 and 128 nodes in one batch (variable cu_nodes), on
+    the default path (balanced batch mode) and on the 128-token kernel."""
+    if impl == "tc128":
+        monkeypatch.setenv("PF_ATTN_IMPL", "tc128")
     w = I.scaled(W["7b-bf16-batch8-paged"], layers=1, batch=3, prefix=(50, 400), nodes=128,
                  vocab=640, hidden=128)
     rng = np.random.default_rng(9)
@@ -232,7 +253,7 @@ def test_mixed_tree_sizes():
     per_seq = -(-max_seq // I.PAGE_SIZE)
     pt = rng.permutation(per_seq * 3).astype(np.int32).reshape(3, per_seq)
     b = I.Batch(w, 7, parents, prefix, ends, pt, per_seq * 3, max_seq)
-    c = Case(w, batch=b)
+    c = Case(w, batch=b, balanced=impl == "default")
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0

@@ -79,7 +79,9 @@ struct TcSmem {
   static_assert(kTotal + 1024 <= 232448, "shared memory budget");
 };
 
-template <int D, int WG>
+// BAL: the balanced batch mode's instance (plan, partials to the workspace);
+// the cluster instance carries none of that code.
+template <int D, int WG, bool BAL>
 __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
                    const __grid_constant__ CUtensorMap tm_tk,
@@ -120,7 +122,7 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
   // group's tiles: split `split` of the cluster, or (balanced batch mode,
   // one CTA per cluster) the item the plan gives it.
   int group = blockIdx.x / nsplit, part = split, nparts = nsplit;
-  if (a.items > 0) {
+  if constexpr (BAL) {
     // warp 0 derives the plan; the first n_groups CTAs also record group
     // blockIdx.x's (first item, items) for the combine kernel
     int4* plan_slot = reinterpret_cast<int4*>(smem + S::kBarOff + S::kNumBars * 8 + 16);
@@ -476,7 +478,7 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
       for (int c0 = 0; c0 < D; c0 += 32)
         tmem_ld_32(o_addr + c0, *reinterpret_cast<uint32_t(*)[32]>(&ov[c0]));
       tmem_ld_wait();
-      if (r < rows && nparts > 1) {
+      if (BAL && r < rows && nparts > 1) {
         __half* dst = reinterpret_cast<__half*>(a.ws) + ((size_t)blockIdx.x * a.bm + r) * S::kInboxPitch;
 #pragma unroll
         for (int c = 0; c < D; c += 8) {
@@ -665,9 +667,9 @@ template <int WG>
 static int tc_max_active_clusters_impl(int cluster) {
   const int smem = tc_smem_bytes<WG>();
   static DeviceMemo limit;
-  if (ensure_smem_limit((const void*)attn_tc_kernel<128, WG>, smem, limit) != cudaSuccess)
+  if (ensure_smem_limit((const void*)attn_tc_kernel<128, WG, false>, smem, limit) != cudaSuccess)
     return 0;
-  if (cluster > 8 && cudaFuncSetAttribute(attn_tc_kernel<128, WG>,
+  if (cluster > 8 && cudaFuncSetAttribute(attn_tc_kernel<128, WG, false>,
                                           cudaFuncAttributeNonPortableClusterSizeAllowed,
                                           1) != cudaSuccess)
     return 0;
@@ -683,7 +685,7 @@ static int tc_max_active_clusters_impl(int cluster) {
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<128, WG>, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<128, WG, false>, &cfg) != cudaSuccess) {
     cudaGetLastError();
     return 0;
   }
@@ -695,24 +697,25 @@ int attention_tc_max_active_clusters(int cluster, int rows_per_cta) {
                             : tc_max_active_clusters_impl<1>(cluster);
 }
 
-template <int WG>
+template <int WG, bool BAL>
 static cudaError_t launch_tc(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl) {
   const int smem = tc_smem_bytes<WG>();
   static DeviceMemo limit;
   static DeviceMemo nonportable;
-  cudaError_t e = ensure_smem_limit((const void*)attn_tc_kernel<128, WG>, smem, limit);
+  cudaError_t e = ensure_smem_limit((const void*)attn_tc_kernel<128, WG, BAL>, smem, limit);
   if (e != cudaSuccess) return e;
   if (a.splits > 8) {
-    e = ensure_nonportable_cluster((const void*)attn_tc_kernel<128, WG>, nonportable);
+    e = ensure_nonportable_cluster((const void*)attn_tc_kernel<128, WG, BAL>, nonportable);
     if (e != cudaSuccess) return e;
   }
-  const dim3 grid(a.items > 0 ? a.items : a.B * a.Hkv * a.rb_count * a.splits);
-  return launch_ex(attn_tc_kernel<128, WG>, grid, dim3(TcShape<WG>::kThreads), smem, s, a.splits,
-                   pdl, m.q, m.tk, m.tv, m.ck, m.cv, a);
+  const dim3 grid(BAL ? a.items : a.B * a.Hkv * a.rb_count * a.splits);
+  return launch_ex(attn_tc_kernel<128, WG, BAL>, grid, dim3(TcShape<WG>::kThreads), smem, s,
+                   a.splits, pdl, m.q, m.tk, m.tv, m.ck, m.cv, a);
 }
 
 cudaError_t launch_attention_tc(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl) {
-  return a.bm > 128 ? launch_tc<2>(a, m, s, pdl) : launch_tc<1>(a, m, s, pdl);
+  if (a.items > 0) return a.bm > 128 ? launch_tc<2, true>(a, m, s, pdl) : launch_tc<1, true>(a, m, s, pdl);
+  return a.bm > 128 ? launch_tc<2, false>(a, m, s, pdl) : launch_tc<1, false>(a, m, s, pdl);
 }
 
 }  // namespace pf

@@ -93,31 +93,6 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t
   return mbar_wait_limit(bar, parity, err, kWaitLimitNs);
 }
 
-// Like mbar_wait, but gives up at once if *abort is set and sets *abort on
-// its own timeout, so that every role of a CTA stops waiting after the first
-// failure while still running through the same number of loop iterations.
-__device__ __forceinline__ bool mbar_wait_abortable(uint32_t bar, uint32_t parity, int32_t* err,
-                                                    volatile int* abort) {
-  if (*abort) return false;
-  if (mbar_try_wait(bar, parity)) return true;
-  const unsigned long long t0 = globaltimer();
-  while (true) {
-    for (int i = 0; i < 64; ++i)
-      if (mbar_try_wait(bar, parity)) return true;
-    if (*abort) return false;
-    if (globaltimer() - t0 > kWaitLimitNs) {
-      flag_error(err, PF_DEVERR_TIMEOUT);
-      *abort = 1;
-      return false;
-    }
-  }
-}
-
-// Named barrier over `count` threads (a multiple of 32).
-__device__ __forceinline__ void named_bar_sync(uint32_t id, uint32_t count) {
-  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
-}
-
 // ---------------------------------------------------------------- TMA
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");

@@ -35,7 +35,15 @@ if ROOT not in sys.path:
 METRIC = "verify-step µs/layer & accepted tokens/s; achieved HBM GB/s vs ~8 TB/s peak"
 DEFAULT_WORKLOAD = "2b-bf16-chain16"
 L2_FLUSH_BYTES = 256 << 20
-PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "lmhead_traffic.txt")
+CSRC = os.path.join(ROOT, "paper_2609_32166_gb300", "csrc")
+# Committed ncu DRAM-traffic summaries, each valid only for the kernel sources
+# it was captured on (a fingerprint of the files that define the kernel and
+# its launch shape).
+LMHEAD_TRAFFIC = (os.path.join(ROOT, "profiles", "lmhead_traffic.txt"),
+                  ("lmhead.cu", "pf_ptx.cuh"))
+ATTENTION_TRAFFIC = (os.path.join(ROOT, "profiles", "attention_traffic.txt"),
+                     ("api.cu", "attention.cu", "attention_tc.cu", "attention_tc2.cu",
+                      "attn_common.cuh", "pf_internal.h", "pf_ptx.cuh"))
 
 
 def parse():
@@ -73,24 +81,37 @@ def step_bytes(w, batch, accept_lens):
     return attn, lm, commit
 
 
-def lmhead_source_fingerprint():
+def attention_flops(w, batch):
+    """FLOPs of one layer's tree attention: QK^T and PV over every prefix row
+    and every proposal row (the masked tree part counted dense), i.e.
+    4 * N * Hq * (P + N) * D summed over the sequences."""
+    return float(sum(4 * len(par) * w.hq * (int(p) + len(par)) * w.d
+                     for par, p in zip(batch.parents, batch.prefix_lens)))
+
+
+def lmhead_flops(w, batch):
+    return 2.0 * batch.total_nodes * w.vocab * w.hidden
+
+
+def source_fingerprint(files):
     h = hashlib.sha256()
-    for f in ("lmhead.cu", "pf_ptx.cuh"):
-        h.update(open(os.path.join(ROOT, "paper_2609_32166_gb300", "csrc", f), "rb").read())
+    for f in files:
+        h.update(open(os.path.join(CSRC, f), "rb").read())
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(workload):
-    """dram bytes per LM-head launch from the committed ncu summary, if it was
-    taken on the current kernel source for this workload; else None."""
-    if not os.path.exists(PROFILE_TRAFFIC):
+def profiled_traffic(spec, workload):
+    """dram bytes per launch from a committed ncu summary, if it was taken on
+    the current kernel sources for this workload; else None."""
+    path, files = spec
+    if not os.path.exists(path):
         return None
     kv = {}
-    for line in open(PROFILE_TRAFFIC):
+    for line in open(path):
         if ":" in line and not line.startswith("#"):
             k, v = line.split(":", 1)
             kv[k.strip()] = v.strip()
-    if kv.get("source_fingerprint") != lmhead_source_fingerprint():
+    if kv.get("source_fingerprint") != source_fingerprint(files):
         return None
     if kv.get("workload") != workload:
         return None
@@ -98,6 +119,49 @@ def profiled_traffic(workload):
         return float(kv["dram_bytes_per_launch"])
     except (KeyError, ValueError):
         return None
+
+
+def kernel_roofline(kernel, dtype, bytes_per_launch, flops_per_launch, seconds_per_launch,
+                    launches_per_step, step_seconds, peaks, traffic):
+    """Roofline of one kernel from its algorithmic bytes and FLOPs per launch
+    and its mean in-step launch time.  The bound is the tensor pipe when the
+    arithmetic intensity of a bf16 kernel lies above the ridge of the two
+    measured peaks (bf16 sustained, since every kernel here is timed inside a
+    long run, over copy bandwidth), else HBM."""
+    hbm = peaks.get("hbm_gbs")
+    tc = peaks.get("bf16_tflops_sustained")
+    hbm_src = "measured copy bandwidth" if hbm else "fallback copy bandwidth"
+    tc_src = "measured bf16 sustained" if tc else "fallback bf16 sustained"
+    hbm = hbm or 6800.0
+    tc = tc or 1700.0
+    ridge = tc * 1e12 / (hbm * 1e9)
+    intensity = flops_per_launch / bytes_per_launch if bytes_per_launch else 0.0
+    if dtype == "bf16" and intensity > ridge:
+        achieved = flops_per_launch / seconds_per_launch / 1e12
+        out = {"bound": "tensor", "achieved": achieved, "peak": tc, "unit": "TFLOP/s",
+               "frac": achieved / tc, "peak_source": tc_src}
+    else:
+        achieved = bytes_per_launch / seconds_per_launch / 1e9
+        out = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+               "frac": achieved / hbm, "peak_source": hbm_src}
+    out.update({"kernel": kernel, "traffic": traffic,
+                "algorithmic_bytes": bytes_per_launch, "algorithmic_flops": flops_per_launch,
+                "intensity_flop_per_byte": intensity, "ridge_flop_per_byte": ridge,
+                "us_per_launch": seconds_per_launch * 1e6,
+                "launches_per_step": launches_per_step,
+                "share_of_step": seconds_per_launch * launches_per_step / step_seconds})
+    return out
+
+
+def step_rooflines(w, batch, attn_bytes, attn_s_per_layer, lm_bytes, lm_s, step_s, peaks):
+    """(dominant, other): the roofline of the kernel with the larger share of
+    the step's time, and that of the other one."""
+    attn = kernel_roofline("pf_verify_attention", w.dtype, attn_bytes,
+                           attention_flops(w, batch), attn_s_per_layer, w.layers, step_s, peaks,
+                           profiled_traffic(ATTENTION_TRAFFIC, w.name))
+    lm = kernel_roofline("pf_lmhead_accept", w.dtype, lm_bytes, lmhead_flops(w, batch), lm_s, 1,
+                         step_s, peaks, profiled_traffic(LMHEAD_TRAFFIC, w.name))
+    return (attn, lm) if attn["share_of_step"] >= lm["share_of_step"] else (lm, attn)
 
 
 # ---------------------------------------------------------------------------
@@ -506,8 +570,9 @@ def main():
     if os.path.exists(pk):
         peaks = json.load(open(pk))
     hbm_peak = peaks.get("hbm_gbs", 6800.0)
-    peak_src = "measured" if "hbm_gbs" in peaks else "fallback"
-    lm_gbs = lm_b / (lm_ms * 1e-3) / 1e9
+    roofline, other_roofline = step_rooflines(w, batch, attn_b_layer,
+                                              attn_ms * 1e-3 / w.layers, lm_b, lm_ms * 1e-3,
+                                              ms_step * 1e-3, peaks)
 
     e2e = None if args.no_e2e else run_e2e(vs, w, batch, K, stream, flush, world, tok_table,
                                            planned)
@@ -528,14 +593,8 @@ def main():
         "step_hbm_gbs": step_b / (ms_step * 1e-3) / 1e9,
         "step_hbm_frac": step_b / (ms_step * 1e-3) / 1e9 / hbm_peak,
         "step_bytes": step_b,
-        "roofline": {"kernel": "pf_lmhead_accept", "bound": "hbm", "achieved": lm_gbs,
-                     "peak": hbm_peak, "unit": "GB/s", "frac": lm_gbs / hbm_peak,
-                     "peak_source": f"{peak_src} (copy bandwidth)",
-                     "algorithmic_bytes": lm_b,
-                     "traffic": profiled_traffic(w.name)},
-        "attention_roofline": {"achieved": attn_b_layer * w.layers / (attn_ms * 1e-3) / 1e9,
-                               "unit": "GB/s", "frac": attn_b_layer * w.layers /
-                               (attn_ms * 1e-3) / 1e9 / hbm_peak},
+        "roofline": roofline,
+        "other_roofline": other_roofline,
         "gpu_launches": K * vs.launches_per_step(),
         "timing": ("CUDA graphs of %d steps; event nodes at every step boundary, and around "
                    "the attention / LM-head / commit parts of the first step of each graph "

@@ -1,0 +1,82 @@
+"""Host-side arithmetic of bench.py's roofline objects (no GPU)."""
+import os
+
+import pytest
+
+from paper_2609_32166_gb300 import inputs
+
+PEAKS = {"hbm_gbs": 6000.0, "bf16_tflops_sustained": 1500.0}   # ridge 250 FLOP/B
+
+
+def _bench():
+    import bench
+    return bench
+
+
+def test_attention_flops_counts_every_row_of_every_sequence():
+    b = _bench()
+    w = inputs.WORKLOADS["2b-bf16-chain16"]
+    batch = inputs.make_batch(w, 0)
+    assert b.attention_flops(w, batch) == 4 * 17 * 12 * (1800 + 17) * 128
+    w8 = inputs.WORKLOADS["7b-bf16-batch8-paged"]
+    b8 = inputs.make_batch(w8, 0)
+    expect = sum(4 * 32 * 28 * (int(p) + 32) * 128 for p in b8.prefix_lens)
+    assert b.attention_flops(w8, b8) == expect
+    assert b.lmhead_flops(w, batch) == 2 * 17 * 151936 * 1536
+
+
+def test_bound_follows_the_ridge():
+    b = _bench()
+    # 100 FLOP/B: below the ridge, HBM-bound; 1 MB in 1 us = 1000 GB/s.
+    r = b.kernel_roofline("k", "bf16", 1e6, 1e8, 1e-6, 1, 1e-5, PEAKS, None)
+    assert r["bound"] == "hbm" and r["unit"] == "GB/s"
+    assert r["achieved"] == pytest.approx(1000.0)
+    assert r["frac"] == pytest.approx(1000.0 / 6000.0)
+    assert r["ridge_flop_per_byte"] == pytest.approx(250.0)
+    # 1000 FLOP/B: above it, tensor-bound; 1 GFLOP in 1 us = 1000 TFLOP/s.
+    r = b.kernel_roofline("k", "bf16", 1e6, 1e9, 1e-6, 1, 1e-5, PEAKS, None)
+    assert r["bound"] == "tensor" and r["unit"] == "TFLOP/s"
+    assert r["achieved"] == pytest.approx(1000.0)
+    assert r["frac"] == pytest.approx(1000.0 / 1500.0)
+    # fp32 never takes the bf16 tensor peak.
+    r = b.kernel_roofline("k", "f32", 1e6, 1e9, 1e-6, 1, 1e-5, PEAKS, None)
+    assert r["bound"] == "hbm"
+
+
+def test_peaks_fall_back_when_unmeasured():
+    b = _bench()
+    r = b.kernel_roofline("k", "bf16", 1e6, 1e6, 1e-6, 1, 1e-5, {}, None)
+    assert r["peak"] == 6800.0 and r["peak_source"].startswith("fallback")
+
+
+def test_dominant_kernel_is_the_larger_share_of_the_step():
+    b = _bench()
+    w = inputs.WORKLOADS["2b-bf16-chain16"]
+    batch = inputs.make_batch(w, 0)
+    # 28 layers x 7 us = 196 us of attention against 88 us of LM head.
+    dom, other = b.step_rooflines(w, batch, 1.97e6, 7e-6, 4.67e8, 88e-6, 290e-6, PEAKS)
+    assert dom["kernel"] == "pf_verify_attention" and other["kernel"] == "pf_lmhead_accept"
+    assert dom["share_of_step"] == pytest.approx(196 / 290)
+    assert dom["launches_per_step"] == 28
+    # 28 x 2 us = 56 us of attention: the LM head dominates.
+    dom, other = b.step_rooflines(w, batch, 1.97e6, 2e-6, 4.67e8, 88e-6, 150e-6, PEAKS)
+    assert dom["kernel"] == "pf_lmhead_accept"
+
+
+def test_traffic_only_for_matching_sources_and_workload(tmp_path):
+    b = _bench()
+    files = ("lmhead.cu", "pf_ptx.cuh")
+    path = os.path.join(tmp_path, "t.txt")
+
+    def write(fp, wl):
+        with open(path, "w") as f:
+            f.write("# comment: ignored\nworkload: %s\nsource_fingerprint: %s\n"
+                    "dram_bytes_per_launch: 1234\n" % (wl, fp))
+
+    write(b.source_fingerprint(files), "2b-bf16-chain16")
+    assert b.profiled_traffic((path, files), "2b-bf16-chain16") == 1234.0
+    assert b.profiled_traffic((path, files), "7b-bf16-tree64") is None
+    write("0000000000000000", "2b-bf16-chain16")
+    assert b.profiled_traffic((path, files), "2b-bf16-chain16") is None
+    assert b.profiled_traffic((os.path.join(tmp_path, "missing.txt"), files),
+                              "2b-bf16-chain16") is None

@@ -531,6 +531,13 @@ __global__ void __launch_bounds__(TcShape<WG>::kThreads, 1)
     for (int c0 = 0; c0 < D; c0 += 32)
       tmem_ld_32(o_addr + c0, *reinterpret_cast<uint32_t(*)[32]>(&ov[c0]));
     tmem_ld_wait();
+    if (!(inv_l > 0.f)) {
+      // no column reached this row in this split (a split without tiles
+      // never writes O): its partial is 0 with lse = -inf, whatever the
+      // unwritten accumulator holds (0 * NaN would poison the merge)
+#pragma unroll
+      for (int c = 0; c < D; ++c) ov[c] = 0u;
+    }
     if (r < rows) {
       __half* dst = stage_rows + r * S::kInboxPitch;
 #pragma unroll

@@ -80,3 +80,10 @@ def test_traffic_only_for_matching_sources_and_workload(tmp_path):
     assert b.profiled_traffic((path, files), "2b-bf16-chain16") is None
     assert b.profiled_traffic((os.path.join(tmp_path, "missing.txt"), files),
                               "2b-bf16-chain16") is None
+
+
+def test_reference_steps_stop_at_the_wall_budget():
+    b = _bench()
+    spec = dict(workload="tiny-f32-chain8", seed=0, layers_sample=1, steps=50, warmup=0)
+    assert b.cpu_worker(dict(spec, wall_budget_s=0.0))["steps"] == 1
+    assert b.cpu_worker(dict(spec, steps=3, wall_budget_s=60.0))["steps"] == 3

@@ -251,7 +251,7 @@ __device__ __forceinline__ Cand score_round(const int8_t* keys, const int* list,
       if (cand_better(cand, best)) best = cand;
     }
   }
-  __syncwarp();  // the stage is refilled by the next round
+  __syncwarp();  // the stage is refilled in the next pass
   return best;
 }
 

@@ -3,16 +3,18 @@ greedy acceptance, KV commit) on seeded synthetic inputs.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
     python bench.py --impl reference ...      # the fp64 CPU oracle, timed
+    python bench.py --ell-sweep               # verify latency vs proposal length
 
 Prints one JSON line.  The metric is accepted tokens/s of whole verify steps
 (sum over sequences of accepted drafts + 1 bonus token, divided by the step
 time), with the attention time per layer and the step's achieved HBM
-bandwidth alongside.  Every step is one CUDA-graph segment: L attention
-launches, one LM-head launch, one commit launch.  Between steps a 256 MB
-memset evicts L2; each step is bracketed by its own CUDA events, so the
-flush is outside the measured time.  Multi-GPU runs are independent
-replicas (one process per GPU under torchrun); the value is the sum of
-tokens over ranks divided by the slowest rank's time.
+bandwidth alongside.  The headline workload is the largest single-GPU one
+(the 8-sequence paged 7B batch); `per_workload` times the other bf16
+workloads in the same run.  Steps run as CUDA graphs of L attention calls,
+one LM-head call and one commit call; a 256 MB memset between steps (outside
+the per-step events) evicts L2.  Multi-GPU runs are independent replicas
+(one process per GPU under torchrun); the value is the sum of tokens over
+ranks divided by the slowest rank's time.
 """
 from __future__ import annotations
 
@@ -33,23 +35,28 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "verify-step µs/layer & accepted tokens/s; achieved HBM GB/s vs ~8 TB/s peak"
-DEFAULT_WORKLOAD = "2b-bf16-chain16"
+DEFAULT_WORKLOAD = "7b-bf16-batch8-paged"
+# the other bf16 workloads, timed in the same run (`per_workload`)
+PER_WORKLOAD = ("7b-bf16-tree64", "7b-bf16-32k-tree128", "2b-bf16-chain16")
 L2_FLUSH_BYTES = 256 << 20
+# per-part (attention / LM head / commit) breakdown: at least this much
+# replay time, whatever --steps is
+PARTS_MIN_SECONDS = 0.5
 # the reference arm (the fp64 oracle on the host cores) times the requested
 # steps, or as many as fit this much wall time
 REFERENCE_WALL_BUDGET_S = 150.0
 CSRC = os.path.join(ROOT, "paper_2609_32166_gb300", "csrc")
 # Committed ncu DRAM-traffic summaries, each valid only for the kernel sources
 # it was captured on (a fingerprint of the files that define the kernel and
-# its launch shape).
+# its launch shape) and for the workload it names.
 LMHEAD_TRAFFIC = (os.path.join(ROOT, "profiles", "lmhead_traffic.txt"),
                   ("lmhead.cu", "pf_ptx.cuh"))
 ATTENTION_TRAFFIC = (os.path.join(ROOT, "profiles", "attention_traffic.txt"),
                      ("api.cu", "attention.cu", "attention_tc.cu", "attention_tc2.cu",
-                      "attn_common.cuh", "pf_internal.h", "pf_ptx.cuh"))
+                      "attention_pair.cu", "attn_common.cuh", "pf_internal.h", "pf_ptx.cuh"))
 
 
-def parse():
+def parse(argv=None):
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
     p.add_argument("--steps", type=int, default=400)
@@ -63,17 +70,23 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-next-rows", action="store_true",
-                   help="skip the key re-rotation and retrieval measurements")
+                   help="skip the re-rotation, retrieval, prefix and ell-sweep measurements")
+    p.add_argument("--no-per-workload", action="store_true",
+                   help="time the headline workload only")
     p.add_argument("--ell-sweep", action="store_true",
-                   help="verify-step latency vs proposal length on the workload's chain shape")
+                   help="only the verify-step latency vs proposal length curve")
     p.add_argument("--cpu-worker", default=None, help=argparse.SUPPRESS)
-    return p.parse_args()
+    return p.parse_args(argv)
 
 
 # ---------------------------------------------------------------------------
-# algorithmic bytes
+# algorithmic bytes and FLOPs
 # ---------------------------------------------------------------------------
 def step_bytes(w, batch, accept_lens):
+    """(attention bytes per layer, LM-head bytes, commit bytes) of one step:
+    every prefix K/V row, the proposal's K/V, q and out read or written once;
+    the LM weight and hidden states once; the committed rows read and written
+    in every layer."""
     es = 2 if w.dtype == "bf16" else 4
     T = batch.total_nodes
     prefix = int(np.sum(batch.prefix_lens))
@@ -124,6 +137,14 @@ def profiled_traffic(spec, workload):
         return None
 
 
+def peak_values(peaks):
+    hbm = peaks.get("hbm_gbs")
+    tc = peaks.get("bf16_tflops_sustained")
+    return (hbm or 6800.0, tc or 1700.0,
+            "measured copy bandwidth" if hbm else "fallback copy bandwidth",
+            "measured bf16 sustained" if tc else "fallback bf16 sustained")
+
+
 def kernel_roofline(kernel, dtype, bytes_per_launch, flops_per_launch, seconds_per_launch,
                     launches_per_step, step_seconds, peaks, traffic):
     """Roofline of one kernel from its algorithmic bytes and FLOPs per launch
@@ -131,12 +152,7 @@ def kernel_roofline(kernel, dtype, bytes_per_launch, flops_per_launch, seconds_p
     arithmetic intensity of a bf16 kernel lies above the ridge of the two
     measured peaks (bf16 sustained, since every kernel here is timed inside a
     long run, over copy bandwidth), else HBM."""
-    hbm = peaks.get("hbm_gbs")
-    tc = peaks.get("bf16_tflops_sustained")
-    hbm_src = "measured copy bandwidth" if hbm else "fallback copy bandwidth"
-    tc_src = "measured bf16 sustained" if tc else "fallback bf16 sustained"
-    hbm = hbm or 6800.0
-    tc = tc or 1700.0
+    hbm, tc, hbm_src, tc_src = peak_values(peaks)
     ridge = tc * 1e12 / (hbm * 1e9)
     intensity = flops_per_launch / bytes_per_launch if bytes_per_launch else 0.0
     if dtype == "bf16" and intensity > ridge:
@@ -165,6 +181,31 @@ def step_rooflines(w, batch, attn_bytes, attn_s_per_layer, lm_bytes, lm_s, step_
     lm = kernel_roofline("pf_lmhead_accept", w.dtype, lm_bytes, lmhead_flops(w, batch), lm_s, 1,
                          step_s, peaks, profiled_traffic(LMHEAD_TRAFFIC, w.name))
     return (attn, lm) if attn["share_of_step"] >= lm["share_of_step"] else (lm, attn)
+
+
+def combined_step_roofline(w, batch, attn_bytes, lm_bytes, commit_bytes, step_s, peaks):
+    """The step's ideal time with each part at its own bound -- attention per
+    layer and the LM head each at max(bytes / HBM, FLOPs / bf16 tensor peak),
+    the commit at bytes / HBM -- against the measured step; and the HBM-only
+    ideal (all algorithmic bytes at the copy bandwidth)."""
+    hbm, tc, _, _ = peak_values(peaks)
+    B, F = hbm * 1e9, tc * 1e12
+    attn_ideal = max(attn_bytes / B, attention_flops(w, batch) / F) * w.layers
+    lm_ideal = max(lm_bytes / B, lmhead_flops(w, batch) / F)
+    commit_ideal = commit_bytes / B
+    ideal = attn_ideal + lm_ideal + commit_ideal
+    hbm_ideal = (attn_bytes * w.layers + lm_bytes + commit_bytes) / B
+    return {"ideal_us": ideal * 1e6, "frac": ideal / step_s,
+            "attention_ideal_us": attn_ideal * 1e6, "lmhead_ideal_us": lm_ideal * 1e6,
+            "commit_ideal_us": commit_ideal * 1e6,
+            "hbm_only_ideal_us": hbm_ideal * 1e6, "hbm_only_frac": hbm_ideal / step_s,
+            "rule": "sum over parts of max(bytes / measured copy bandwidth, FLOPs / measured "
+                    "bf16 sustained peak), divided by the measured step time"}
+
+
+def load_peaks():
+    pk = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    return json.load(open(pk)) if os.path.exists(pk) else {}
 
 
 # ---------------------------------------------------------------------------
@@ -232,6 +273,11 @@ class ClockSampler:
 # interpreter so its BLAS thread count is set before numpy loads
 # ---------------------------------------------------------------------------
 def cpu_worker(spec: dict) -> dict:
+    """Times the fp64 oracle on one workload.  mode "whole": whole verify
+    steps, every layer and sequence.  mode "layer": one sampled step =
+    attention and commit of layer 0 for every sequence, the full LM head and
+    the acceptance walks; the whole-step time is projected as
+    L * (attention + commit of one layer) + LM head + walks."""
     from oracle import accept as OAcc
     from oracle import attention as OA
     from oracle import commit as OC
@@ -245,7 +291,7 @@ def cpu_worker(spec: dict) -> dict:
     f = (lambda x: I.bf16_bits_to_f32(x)) if w.dtype == "bf16" else (lambda x: x)
     hidden = f(I.hidden_states(w, batch))
     weight = f(I.lm_weight(w, batch.seed))
-    nl = spec["layers_sample"]
+    nl = w.layers if spec["mode"] == "whole" else 1
     layers = []
     for l in range(nl):
         q = f(I.layer_q(w, batch, l))
@@ -283,54 +329,77 @@ def cpu_worker(spec: dict) -> dict:
                 OC.commit_rows(rows, P, acc[s][1], tk[c0:c1])
                 OC.commit_rows(rows, P, acc[s][1], tv[c0:c1])
         t_commit = time.perf_counter() - t2
-        scale = w.layers / nl
-        est = (t_attn + t_commit) * scale + t_lm
-        return est, sum(a[0] + 1 for a in acc)
+        measured = t_attn + t_lm + t_commit
+        whole = (t_attn + t_commit) * (w.layers / nl) + t_lm
+        return measured, whole, sum(a[0] + 1 for a in acc)
 
-    times, toks = [], []
+    meas, whole, toks = [], [], []
     n = spec.get("steps")
-    if n is None:   # time-bounded sample for cpu_baseline
-        t_start = time.perf_counter()
-        while (time.perf_counter() - t_start < spec["budget_s"] or not times) and len(times) < 50:
-            est, tok = one_step()
-            times.append(est)
-            toks.append(tok)
-    else:
-        for _ in range(spec["warmup"]):
-            one_step()
-        counter[0] = 0
-        # the requested steps, or as many as fit the wall budget (at least one)
-        t_start = time.perf_counter()
-        budget = spec.get("wall_budget_s")
-        for _ in range(n):
-            if times and budget is not None and time.perf_counter() - t_start > budget:
-                break
-            est, tok = one_step()
-            times.append(est)
-            toks.append(tok)
-    return dict(step_s=float(np.mean(times)), steps=len(times),
-                tokens_per_step=float(np.mean(toks)))
+    budget = spec.get("wall_budget_s")
+    for _ in range(spec.get("warmup", 0)):
+        one_step()
+    counter[0] = 0
+    t_start = time.perf_counter()
+    # the requested steps, or as many as fit the wall budget (at least one)
+    while len(meas) < (n if n is not None else 1 << 30):
+        if meas and budget is not None and time.perf_counter() - t_start > budget:
+            break
+        m, wh, tok = one_step()
+        meas.append(m)
+        whole.append(wh)
+        toks.append(tok)
+    return dict(measured_s=float(np.mean(meas)), step_s=float(np.mean(whole)), steps=len(meas),
+                tokens_per_step=float(np.mean(toks)), layers_timed=nl)
 
 
-def run_cpu_worker(spec: dict) -> dict:
+def run_cpu_worker(spec: dict, threads: int = None) -> dict:
     cores = os.cpu_count() or 1
+    threads = threads or cores
     env = dict(os.environ)
     for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
-        env[k] = str(cores)
+        env[k] = str(threads)
     env["CUDA_VISIBLE_DEVICES"] = ""
     r = subprocess.run([sys.executable, os.path.abspath(__file__), "--cpu-worker", json.dumps(spec)],
                        capture_output=True, text=True, env=env, cwd=ROOT)
     if r.returncode != 0:
         raise RuntimeError("CPU oracle worker failed:\n" + r.stderr[-2000:])
     out = json.loads(r.stdout.strip().splitlines()[-1])
-    out["cores"] = cores
+    out["cores"] = threads
+    out["host_cores"] = cores
     return out
 
 
-def cpu_sample_text(w, nl):
-    return (f"whole verify steps of {w.name} in fp64 numpy: attention of {nl} of {w.layers} "
-            f"layers (time scaled by {w.layers}/{nl}), full LM head ({w.vocab}x{w.hidden}), "
-            f"acceptance, commit")
+def cpu_mode(w):
+    """Whole steps where one fits a few seconds of fp64 numpy (the 2B chain
+    and smaller), else a one-layer sample."""
+    return "whole" if (w.hq * w.nodes * w.batch <= 256 and w.prefix[1] <= 4096) else "layer"
+
+
+def cpu_sample_text(w, r):
+    if r["layers_timed"] == w.layers:
+        what = (f"whole verify steps of {w.name} in fp64 numpy: attention of all {w.layers} "
+                f"layers, full LM head ({w.vocab}x{w.hidden}), acceptance, commit")
+    else:
+        what = (f"one sampled step of {w.name} in fp64 numpy: attention and commit of layer 0 "
+                f"for all {w.batch} sequence(s), full LM head ({w.vocab}x{w.hidden}), acceptance; "
+                f"whole-step time projected as {w.layers} x (attention + commit of one layer) "
+                f"+ LM head + acceptance")
+    return what + f"; {r['steps']} step(s) timed, {r['cores']} thread(s)"
+
+
+def cpu_baseline_entry(w, spec_base):
+    """The oracle on all host cores and on one core; value = accepted
+    tokens per (projected) whole-step second."""
+    out = {}
+    for label, threads in (("all_cores", None), ("single_thread", 1)):
+        r = run_cpu_worker(dict(spec_base, mode=cpu_mode(w)), threads=threads)
+        out[label] = {"value": r["tokens_per_step"] / r["step_s"], "unit": "tokens/s",
+                      "cores": r["cores"], "kind": "oracle", "ms_per_step": r["step_s"] * 1e3,
+                      "measured_ms_per_sample": r["measured_s"] * 1e3,
+                      "sample": cpu_sample_text(w, r)}
+    base = dict(out["all_cores"])
+    base["single_thread"] = out["single_thread"]
+    return base
 
 
 # ---------------------------------------------------------------------------
@@ -364,9 +433,9 @@ def run_reference(args):
         return
     from paper_2609_32166_gb300 import inputs as I
     w = I.WORKLOADS[args.workload]
-    nl = 1
-    spec = dict(workload=args.workload, seed=args.seed, layers_sample=nl, steps=args.steps,
-                warmup=args.warmup, wall_budget_s=REFERENCE_WALL_BUDGET_S)
+    mode = cpu_mode(w)
+    spec = dict(workload=args.workload, seed=args.seed, mode=mode, steps=args.steps,
+                warmup=min(args.warmup, 1), wall_budget_s=REFERENCE_WALL_BUDGET_S)
     t0 = time.perf_counter()
     r = run_cpu_worker(spec)
     wall = time.perf_counter() - t0
@@ -375,12 +444,16 @@ def run_reference(args):
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
         "n_gpus": args.gpus, "steps": r["steps"], "steps_requested": args.steps,
         "warmup": args.warmup,
-        "ms_per_step": r["step_s"] * 1e3, "higher_is_better": True, "scaling": "weak",
+        # the measured time of the steps this run executed (for a one-layer
+        # sample: the sample, not the projected whole step)
+        "ms_per_step": r["measured_s"] * 1e3,
+        "projected_ms_per_whole_step": r["step_s"] * 1e3,
+        "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded generator)",
         "config": config_dict(w, args),
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": r["cores"],
                          "kind": "oracle",
-                         "sample": cpu_sample_text(w, nl) +
+                         "sample": cpu_sample_text(w, r) +
                          f"; {r['steps']} of {args.steps} steps timed (the steps that fit "
                          f"{REFERENCE_WALL_BUDGET_S:.0f} s of wall time)"},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
@@ -400,232 +473,257 @@ def config_dict(w, args):
 
 
 # ---------------------------------------------------------------------------
-# our arm
+# our arm: one workload, device-timed
 # ---------------------------------------------------------------------------
-def main():
-    args = parse()
-    if args.cpu_worker is not None:
-        print(json.dumps(cpu_worker(json.loads(args.cpu_worker))))
-        return
-    if args.impl == "reference":
-        run_reference(args)
-        return
-    if args.ell_sweep:
-        run_ell_sweep(args)
-        return
-
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-
-    cpu_base = None
-    from paper_2609_32166_gb300 import inputs as I
-    w = I.WORKLOADS[args.workload]
-    if args.layers is not None:
-        w = I.scaled(w, layers=max(1, min(args.layers, w.layers)))
-    nl_cpu = 1
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        # before any CUDA call in this process
-        cpu_base = run_cpu_worker(dict(workload=args.workload, seed=args.seed,
-                                       layers_sample=nl_cpu, budget_s=12.0, layers=w.layers))
-
+def _graph_events_supported():
     import torch
-    import torch.distributed as dist
-    torch.cuda.set_device(local)
-    if world > 1:
-        dist.init_process_group("nccl")
+    try:
+        torch.cuda.Event(enable_timing=True, external=True)
+        return True
+    except TypeError:
+        return False
 
-    import __graft_entry__
-    __graft_entry__.build()
+
+def prepare_workload(w, seed, weight_dev=None):
+    """Device state of a workload (bulk tensors drawn on the device), draft
+    tokens planted from the GPU's own greedy predictions for a seeded
+    sequence of per-step accepted paths."""
+    import torch
+    from paper_2609_32166_gb300 import inputs as I
     from paper_2609_32166_gb300.step import VerifyStep
-
-    batch = I.make_batch(w, args.seed)
-    vs = VerifyStep(w, batch, np.zeros(batch.total_nodes, np.int32))
-    # plant the draft tokens from the model's own greedy predictions so the
-    # accepted length is the planted one
+    batch = I.make_batch(w, seed)
+    vs = VerifyStep(w, batch, np.zeros(batch.total_nodes, np.int32), fill="device",
+                    weight_dev=weight_dev)
     vs.lmhead()
     torch.cuda.synchronize()
     greedy = vs.argmax.cpu().numpy()
-    # every step verifies a new proposal: the planted accepted path of step k
-    # follows the workload's rule, drawn from a seeded per-step stream
-    K = args.steps
-    G = max(d for d in range(1, min(K, 50) + 1) if K % d == 0)
+    G = 50
     ends = I.step_forced_ends(batch, G)
     depth = [I.node_depths(p) for p in batch.parents]
     planned = [int(sum(depth[b][e[b]] + 1 for b in range(w.batch))) for e in ends]
     tok_table = torch.from_numpy(np.stack([I.plant_tokens(batch, greedy, e, salt=g)
                                            for g, e in enumerate(ends)])).cuda()
-    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    return vs, batch, tok_table, planned
 
-    stream = torch.cuda.Stream()
-    torch.cuda.synchronize()
+
+def time_steps(vs, tok_table, planned, K, warmup, stream, flush, parts, world=1, dist=None):
+    """K verify steps in CUDA graphs of up to 50 steps, events at every step
+    boundary (parts=False) or also around the attention / LM head / commit
+    of every step (parts=True; those events split the programmatic-launch
+    chain between the parts).  Returns (per-step ms, per-part ms lists,
+    accepted tokens per step)."""
+    import torch
+    G_tab = tok_table.shape[0]
     with torch.cuda.stream(stream):
-        for k in range(max(args.warmup, 3)):
+        for k in range(max(warmup, 3)):
             flush.zero_()
-            vs.tokens.copy_(tok_table[k % G])
+            vs.tokens.copy_(tok_table[k % G_tab])
             vs.step()
             stream.synchronize()
             got = int((vs.accept_len + 1).sum().item())
-            assert got == planned[k % G], (k, got, planned[k % G])
-    accepted_steps = [planned[k % G] for k in range(K)]
-
-    # one graph = G steps; each step: flush, tokens | e0 attention e1 lmhead e2 commit e3
-    per_step, attn_t, lm_t, commit_t = [], [], [], []
-
-    def collect(e, parts=True):
-        per_step.append(e[0].elapsed_time(e[3]))
-        if parts:
-            attn_t.append(e[0].elapsed_time(e[1]))
-            lm_t.append(e[1].elapsed_time(e[2]))
-            commit_t.append(e[2].elapsed_time(e[3]))
-
-    try:
-        torch.cuda.Event(enable_timing=True, external=True)
-        graph_events = True
-    except TypeError:
-        graph_events = False
-    clocks = ClockSampler(torch.cuda.current_device())
-    if graph_events:
-        R = K // G
-        # step boundaries carry events in every step; the part boundaries
-        # (which break the programmatic-dependent-launch chain between the
-        # last layer, the LM head and the commit) only in the first step of
-        # each graph, which provides the per-kernel breakdown
-        ev = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(4)]
-              for _ in range(G)]
-        graph = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(graph, stream=stream):
-            s = torch.cuda.current_stream()
-            for g in range(G):
-                flush.zero_()
-                vs.tokens.copy_(tok_table[g])
-                ev[g][0].record(s)
-                for l in range(vs.L):
-                    vs.attention(l, s.cuda_stream)
-                if g == 0:
-                    ev[g][1].record(s)
-                vs.lmhead(s.cuda_stream)
-                if g == 0:
-                    ev[g][2].record(s)
-                vs.commit(s.cuda_stream)
-                ev[g][3].record(s)
-        with torch.cuda.stream(stream):
-            graph.replay()   # untimed: uploads the graph
-        stream.synchronize()
-        clocks.start()
-        time.sleep(0.3)
-        if world > 1:
-            dist.barrier()
-        torch.cuda.synchronize()
-        with torch.cuda.stream(stream):
-            for r in range(R):
+            assert got == planned[k % G_tab], (k, got, planned[k % G_tab])
+    per_step, attn_t, lm_t, commit_t, toks = [], [], [], [], []
+    done = 0
+    graph_events = _graph_events_supported()
+    while done < K:
+        n = min(50, K - done)
+        if graph_events:
+            ev = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(4)]
+                  for _ in range(n)]
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=stream):
+                s = torch.cuda.current_stream()
+                for g in range(n):
+                    flush.zero_()
+                    vs.tokens.copy_(tok_table[(done + g) % G_tab])
+                    ev[g][0].record(s)
+                    for l in range(vs.L):
+                        vs.attention(l, s.cuda_stream)
+                    if parts:
+                        ev[g][1].record(s)
+                    vs.lmhead(s.cuda_stream)
+                    if parts:
+                        ev[g][2].record(s)
+                    vs.commit(s.cuda_stream)
+                    ev[g][3].record(s)
+            with torch.cuda.stream(stream):
+                graph.replay()   # untimed: uploads the graph
+            stream.synchronize()
+            if dist is not None and world > 1:
+                dist.barrier()
+            torch.cuda.synchronize()
+            with torch.cuda.stream(stream):
                 graph.replay()
-                # the event nodes hold this replay's timestamps: read them
-                # before the next replay overwrites them
-                stream.synchronize()
-                for g in range(G):
-                    collect(ev[g], parts=(g == 0))
-    else:
-        # torch without external graph events: one graph per part, events
-        # recorded between graph launches
-        parts = []
-        for fn in (lambda st: [vs.attention(l, st) for l in range(vs.L)],
-                   lambda st: vs.lmhead(st), lambda st: vs.commit(st)):
-            gr = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(gr, stream=stream):
-                fn(torch.cuda.current_stream().cuda_stream)
-            parts.append(gr)
-        with torch.cuda.stream(stream):
-            for gr in parts:
-                gr.replay()
-        stream.synchronize()
-        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
-        clocks.start()
-        time.sleep(0.3)
-        if world > 1:
-            dist.barrier()
-        torch.cuda.synchronize()
-        with torch.cuda.stream(stream):
-            for k in range(K):
-                flush.zero_()
-                vs.tokens.copy_(tok_table[k % G])
-                ev[k][0].record(stream)
-                parts[0].replay()
-                ev[k][1].record(stream)
-                parts[1].replay()
-                ev[k][2].record(stream)
-                parts[2].replay()
-                ev[k][3].record(stream)
-        stream.synchronize()
-        for k in range(K):
-            collect(ev[k])
-    torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
-    clk = clocks.stop()
-    assert len(per_step) == K
-    t_total_ms = max_over_ranks(float(np.sum(per_step)), world, "cuda")
+            stream.synchronize()
+            del graph
+        else:
+            ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(n)]
+            with torch.cuda.stream(stream):
+                for g in range(n):
+                    flush.zero_()
+                    vs.tokens.copy_(tok_table[(done + g) % G_tab])
+                    ev[g][0].record(stream)
+                    for l in range(vs.L):
+                        vs.attention(l, stream.cuda_stream)
+                    ev[g][1].record(stream)
+                    vs.lmhead(stream.cuda_stream)
+                    ev[g][2].record(stream)
+                    vs.commit(stream.cuda_stream)
+                    ev[g][3].record(stream)
+            stream.synchronize()
+        for g in range(n):
+            per_step.append(ev[g][0].elapsed_time(ev[g][3]))
+            if parts or not graph_events:
+                attn_t.append(ev[g][0].elapsed_time(ev[g][1]))
+                lm_t.append(ev[g][1].elapsed_time(ev[g][2]))
+                commit_t.append(ev[g][2].elapsed_time(ev[g][3]))
+            toks.append(planned[(done + g) % G_tab])
+        done += n
     res = vs.results()
     assert res["err"] == 0, f"device error flag {res['err']}"
-    assert int(np.sum(res["accept_len"] + 1)) == accepted_steps[-1]
+    assert int(np.sum(res["accept_len"] + 1)) == toks[-1]
+    return per_step, (attn_t, lm_t, commit_t), toks
 
+
+def measure_workload(w, args, K, stream, flush, peaks, weight_dev=None, world=1, dist=None,
+                     clocks=None):
+    """Device-timed steps of one workload: the step time over exactly K
+    steps (step-boundary events only), then a per-part pass of at least
+    PARTS_MIN_SECONDS of replays with events around every step's parts."""
+    import torch
+    vs, batch, tok_table, planned = prepare_workload(w, args.seed, weight_dev)
+    if clocks is not None:
+        clocks.start()
+        time.sleep(0.3)
+    per_step, _, toks = time_steps(vs, tok_table, planned, K, args.warmup, stream, flush,
+                                   parts=False, world=world, dist=dist)
+    clk = clocks.stop() if clocks is not None else None
+    t_total_ms = max_over_ranks(float(np.sum(per_step)), world, "cuda")
     ms_step = t_total_ms / K
-    accepted = float(np.mean(accepted_steps))
-    value = whole_job_rate(float(np.sum(accepted_steps)), t_total_ms / 1e3, world)
+    k_parts = max(20, int(np.ceil(PARTS_MIN_SECONDS / (ms_step * 1e-3))))
+    _, (attn_t, lm_t, commit_t), _ = time_steps(vs, tok_table, planned, k_parts, 0, stream,
+                                                flush, parts=True)
+    res = vs.results()
     attn_b, lm_b, commit_b = step_bytes(w, batch, res["accept_len"])
-    attn_b_layer = attn_b
     step_b = attn_b * w.layers + lm_b + commit_b
-    lm_ms = float(np.mean(lm_t))
     attn_ms = float(np.mean(attn_t))
-    peaks = {}
-    pk = os.path.join(ROOT, "MEASURED_PEAKS.json")
-    if os.path.exists(pk):
-        peaks = json.load(open(pk))
-    hbm_peak = peaks.get("hbm_gbs", 6800.0)
-    roofline, other_roofline = step_rooflines(w, batch, attn_b_layer,
-                                              attn_ms * 1e-3 / w.layers, lm_b, lm_ms * 1e-3,
-                                              ms_step * 1e-3, peaks)
-
-    e2e = None if args.no_e2e else run_e2e(vs, w, batch, K, stream, flush, world, tok_table,
-                                           planned)
-    if rank != 0:
-        if world > 1:
-            dist.destroy_process_group()
-        return
-    next_rows = None if args.no_next_rows else measure_next_rows(stream, flush, hbm_peak)
-    line = {
-        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
-        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
-        "data": "synthetic (seeded generator, shapes of the named workload)",
-        "config": config_dict(w, args),
-        "accepted_tokens_per_step": accepted,
+    lm_ms = float(np.mean(lm_t))
+    hbm = peak_values(peaks)[0]
+    roof, other = step_rooflines(w, batch, attn_b, attn_ms * 1e-3 / w.layers, lm_b, lm_ms * 1e-3,
+                                 ms_step * 1e-3, peaks)
+    out = {
+        "workload": w.name, "steps": K, "ms_per_step": ms_step,
+        "value": whole_job_rate(float(np.sum(toks)), t_total_ms / 1e3, world),
+        "unit": "tokens/s", "accepted_tokens_per_step": float(np.mean(toks)),
         "us_per_layer_attention": attn_ms * 1e3 / w.layers,
         "us_lmhead": lm_ms * 1e3, "us_commit": float(np.mean(commit_t)) * 1e3,
+        "parts": {"steps": len(attn_t), "seconds": float(np.sum(attn_t) + np.sum(lm_t) +
+                                                         np.sum(commit_t)) * 1e-3,
+                  "ms_per_step_with_part_events": float(np.mean(attn_t) + np.mean(lm_t) +
+                                                        np.mean(commit_t)),
+                  "attention_us_per_layer_sd": float(np.std(attn_t)) * 1e3 / w.layers,
+                  "lmhead_us_sd": float(np.std(lm_t)) * 1e3},
         "step_hbm_gbs": step_b / (ms_step * 1e-3) / 1e9,
-        "step_hbm_frac": step_b / (ms_step * 1e-3) / 1e9 / hbm_peak,
+        "step_hbm_frac": step_b / (ms_step * 1e-3) / 1e9 / hbm,
         "step_bytes": step_b,
-        "roofline": roofline,
-        "other_roofline": other_roofline,
-        "gpu_launches": K * vs.launches_per_step(),
-        "timing": ("CUDA graphs of %d steps; event nodes at every step boundary, and around "
-                   "the attention / LM-head / commit parts of the first step of each graph "
-                   "(those give the per-part times)" % G
-                   if graph_events else "one CUDA graph per part, events between graph launches"),
-        "clocks": clk,
-        "e2e": e2e,
-        "next_rows": next_rows,
+        "step_roofline": combined_step_roofline(w, batch, attn_b, lm_b, commit_b, ms_step * 1e-3,
+                                                peaks),
+        "roofline": roof,
+        "other_roofline": other,
+        "gpu_launches_per_step": vs.launches_per_step(),
     }
-    if cpu_base is not None:
-        line["cpu_baseline"] = {"value": cpu_base["tokens_per_step"] / cpu_base["step_s"],
-                                "unit": "tokens/s", "cores": cpu_base["cores"], "kind": "oracle",
-                                "sample": cpu_sample_text(w, nl_cpu) +
-                                f"; {cpu_base['steps']} step(s) timed"}
-    print(json.dumps(line))
-    if world > 1:
-        dist.destroy_process_group()
+    if clk is not None:
+        out["clocks"] = clk
+    return out, vs, batch, tok_table, planned
 
 
+# ---------------------------------------------------------------------------
+# end to end through the library's calls
+# ---------------------------------------------------------------------------
+def run_e2e(vs, w, K, stream, flush, world, tok_table, planned):
+    """The same metric end to end, as a caller of the library sees it, timed
+    on the host wall clock: every step copies its inputs (queries, proposal
+    K/V of every layer, hidden states, tokens, tree and lengths: one packed
+    arena) from pinned host memory, issues the C-ABI calls eagerly -- the
+    device tree bitmaps (pf_tree_prepare_device), L attention calls, the LM
+    head, the commit -- reads its outputs (accepted lengths, tokens, new
+    lengths: one arena) back and synchronises.  The L2 flush between steps
+    is outside the timed region.  A second figure replays the same step as
+    one CUDA graph between the copies (device events)."""
+    import torch
+    host_in = vs.in_arena.detach().cpu().pin_memory()
+    host_out = torch.empty(vs.out_arena.numel(), dtype=torch.uint8).pin_memory()
+    tok_off = vs.tokens.data_ptr() - vs.in_arena.data_ptr()
+    tok_bytes = vs.tokens.numel() * vs.tokens.element_size()
+    host_tokens = [t.cpu().contiguous().view(torch.uint8) for t in tok_table]
+    acc_off = vs.accept_len.data_ptr() - vs.out_arena.data_ptr()
+    h2d, d2h = host_in.numel(), host_out.numel()
+    n = min(K, 200)
+    sp = stream.cuda_stream
+
+    def one(k, graph=None, events=None):
+        host_in[tok_off:tok_off + tok_bytes].copy_(host_tokens[k % len(host_tokens)])
+        with torch.cuda.stream(stream):
+            flush.zero_()
+        stream.synchronize()
+        t0 = time.perf_counter()
+        with torch.cuda.stream(stream):
+            if events:
+                events[0].record(stream)
+            vs.in_arena.copy_(host_in, non_blocking=True)
+            if graph is None:
+                vs.step(sp, tree_prepare=True)
+            else:
+                graph.replay()
+            host_out.copy_(vs.out_arena, non_blocking=True)
+            if events:
+                events[1].record(stream)
+        stream.synchronize()
+        t = time.perf_counter() - t0
+        got = int((host_out[acc_off:acc_off + 4 * w.batch].view(torch.int32) + 1).sum())
+        assert got == planned[k % len(planned)]
+        return t, got
+
+    for k in range(3):
+        one(k)
+    wall, tok = [], 0
+    for k in range(n):
+        t, got = one(k)
+        wall.append(t)
+        tok += got
+    t_wall = max_over_ranks(float(np.sum(wall)), world, "cuda")
+    # graph variant
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        vs.step(torch.cuda.current_stream().cuda_stream, tree_prepare=True)
+    with torch.cuda.stream(stream):
+        g.replay()
+    stream.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    gt, gtok = [], 0
+    for k in range(n):
+        _, got = one(k, graph=g, events=(e0, e1))
+        gt.append(e0.elapsed_time(e1))
+        gtok += got
+    t_graph = max_over_ranks(float(np.sum(gt)), world, "cuda")
+    res = vs.results()
+    assert res["err"] == 0
+    return {"value": whole_job_rate(tok, t_wall, world), "unit": "tokens/s",
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n,
+            "ms_per_step": t_wall * 1e3 / n,
+            "timing": "host wall clock (time.perf_counter) around H2D, eager C-ABI calls "
+                      "(pf_tree_prepare_device, %d x pf_verify_attention, pf_lmhead_accept, "
+                      "pf_kv_commit), D2H and a stream synchronise, per step" % vs.L,
+            "copies_per_step": {"h2d": 1, "d2h": 1},
+            "graph": {"value": whole_job_rate(gtok, t_graph * 1e-3, world),
+                      "ms_per_step": t_graph / n,
+                      "timing": "the same step as one CUDA-graph replay between the copies, "
+                                "device events around copies and replay"}}
+
+
+# ---------------------------------------------------------------------------
+# widened rows and the verify latency curve
+# ---------------------------------------------------------------------------
 def _time_events(stream, flush, fn, iters, warmup=3):
     """Mean device time (ms) of fn(i) over iters calls, L2 flushed before each
     call outside the events.  The calls are captured in one CUDA graph with
@@ -637,12 +735,9 @@ def _time_events(stream, flush, fn, iters, warmup=3):
             flush.zero_()
             fn(i)
     stream.synchronize()
-    try:
+    if _graph_events_supported():
         ev = [(torch.cuda.Event(enable_timing=True, external=True),
                torch.cuda.Event(enable_timing=True, external=True)) for _ in range(iters)]
-    except TypeError:
-        ev = None
-    if ev is not None:
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
             s = torch.cuda.current_stream()
@@ -670,11 +765,12 @@ def _time_events(stream, flush, fn, iters, warmup=3):
 
 
 def measure_next_rows(stream, flush, hbm_peak, reps=4):
-    """Rolling-image key re-rotation and decoding-memory retrieval, each on a
-    workload of the paper's shape, timed with CUDA events on the launching
-    stream.  Each timed iteration makes `reps` calls on `reps` disjoint
-    buffers (every call cold in L2; L2 flushed between iterations), so the
-    fixed cost of the event pair is spread over several calls."""
+    """Rolling-image key re-rotation, decoding-memory retrieval and prompt-
+    prefix carryover, each on a workload of the paper's shape, timed with
+    CUDA events on the launching stream.  Each timed iteration makes `reps`
+    calls on `reps` disjoint buffers (every call cold in L2; L2 flushed
+    between iterations), so the fixed cost of the event pair is spread over
+    several calls."""
     import torch
     from paper_2609_32166_gb300 import binding as pb
     from paper_2609_32166_gb300 import inputs as I
@@ -806,77 +902,36 @@ def measure_next_rows(stream, flush, hbm_peak, reps=4):
 
 
 ELL_POINTS = (0, 1, 2, 3, 4, 6, 8, 12, 16, 24, 32, 48, 64, 96, 127)
+ELL_RATES = (0.3, 0.6, 0.8, 0.9, 0.95, 0.99)
 
 
-def run_ell_sweep(args):
+def ell_sweep(base, seed, stream, flush, steps=50, weight_dev=None):
     """Verify-step latency T(l) for chain proposals of l drafts (N = l + 1
-    nodes) on the workload's model shape and prefix: L attention launches,
-    the LM head with acceptance, the commit; CUDA-graph steps with events
-    at every step boundary, L2 flushed between steps (outside the events),
-    accepted length drawn per step as in the main benchmark.  Prints one
-    JSON line with the curve and a log-quadratic least-squares fit
-    log T = c0 + c1 l + c2 l^2 (the latency model of eq. 1's controller)."""
+    nodes) on the workload's model shape with one sequence and its largest
+    prefix: L attention launches, the LM head with acceptance, the commit;
+    CUDA-graph steps with events at every step boundary, L2 flushed between
+    steps (outside the events), accepted length drawn per step as in the
+    main benchmark.  Returns the curve, a log-quadratic least-squares fit
+    log T = c0 + c1 l + c2 l^2 (the latency model of eq. 1's controller) and
+    the library controller's choices on it at fixed per-token acceptance."""
     import torch
-    import __graft_entry__
-    __graft_entry__.build()
+    from paper_2609_32166_gb300 import binding as pb
     from paper_2609_32166_gb300 import inputs as I
-    from paper_2609_32166_gb300.step import VerifyStep
-    base = I.WORKLOADS[args.workload]
-    weight = I.lm_weight(base, args.seed)
-    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
-    stream = torch.cuda.Stream()
-    K = max(10, args.steps)
-    G = max(d for d in range(1, min(K, 50) + 1) if K % d == 0)
     points = []
     for ell in ELL_POINTS:
         w = I.scaled(base, nodes=ell + 1, max_depth=ell, tree="chain", accept="chain", batch=1,
-                     layout="contiguous")
-        batch = I.make_batch(w, args.seed)
-        vs = VerifyStep(w, batch, np.zeros(batch.total_nodes, np.int32), weight=weight)
-        vs.lmhead()
-        torch.cuda.synchronize()
-        greedy = vs.argmax.cpu().numpy()
-        ends = I.step_forced_ends(batch, G)
-        toks = torch.from_numpy(np.stack([I.plant_tokens(batch, greedy, e, salt=g)
-                                          for g, e in enumerate(ends)])).cuda()
-        with torch.cuda.stream(stream):
-            for k in range(max(args.warmup, 3)):
-                flush.zero_()
-                vs.tokens.copy_(toks[k % G])
-                vs.step(stream.cuda_stream)
-        stream.synchronize()
-        ev = [(torch.cuda.Event(enable_timing=True, external=True),
-               torch.cuda.Event(enable_timing=True, external=True)) for _ in range(G)]
-        gr = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(gr, stream=stream):
-            st = torch.cuda.current_stream()
-            for g in range(G):
-                flush.zero_()
-                vs.tokens.copy_(toks[g])
-                ev[g][0].record(st)
-                vs.step(st.cuda_stream)
-                ev[g][1].record(st)
-        times = []
-        with torch.cuda.stream(stream):
-            gr.replay()   # untimed: uploads the graph
-            stream.synchronize()
-            for r in range(K // G):
-                gr.replay()
-                stream.synchronize()
-                times.extend(a.elapsed_time(b) for a, b in ev)
-        res = vs.results()
-        assert res["err"] == 0
-        del vs, gr
+                     layout="contiguous", prefix=(base.prefix[1], base.prefix[1]))
+        vs, batch, tok_table, planned = prepare_workload(w, seed, weight_dev)
+        if weight_dev is None:
+            weight_dev = vs.weight
+        per_step, _, _ = time_steps(vs, tok_table, planned, steps, 3, stream, flush, parts=False)
+        points.append({"ell": ell, "nodes": ell + 1, "us_step": float(np.mean(per_step)) * 1e3})
+        del vs
         torch.cuda.empty_cache()
-        points.append({"ell": ell, "nodes": ell + 1, "us_step": float(np.mean(times)) * 1e3})
     ell = np.array([p["ell"] for p in points], dtype=np.float64)
     logt = np.log(np.array([p["us_step"] for p in points]))
     A = np.stack([np.ones_like(ell), ell, ell * ell], axis=1)
     coef, *_ = np.linalg.lstsq(A, logt, rcond=None)
-    # eq. 1 driven by the measured curve: the library's controller fits its
-    # latency model to the points; for a per-token acceptance rate q (p1 =
-    # pc = q) the chosen length and the resulting tokens per second
-    from paper_2609_32166_gb300 import binding as pb
     l_max = ELL_POINTS[-1]
     ctl = pb.pf_controller_init(l_max, 0.05, 0.0)
     for p in points:
@@ -884,64 +939,131 @@ def run_ell_sweep(args):
     u = np.arange(l_max + 1) / l_max
     t_hat = np.exp(ctl.c[0] + ctl.c[1] * u + ctl.c[2] * u * u)
     choices = []
-    for q in (0.3, 0.6, 0.8, 0.9, 0.95, 0.99):
+    for q in ELL_RATES:
         best, obj = pb.pf_length_select(t_hat, np.full(l_max + 1, q), np.full(l_max + 1, q))
         choices.append({"per_token_acceptance": q, "chosen_length": best,
                         "us_per_token": obj, "tokens_per_s": 1e6 / obj})
-    print(json.dumps({"mode": "ell_sweep", "workload": base.name, "unit": "us per verify step",
-                      "steps_per_point": K, "points": points,
-                      "log_quadratic_fit": [float(c) for c in coef],
-                      "controller": {"l_max": l_max, "latency_model": list(ctl.c),
-                                     "choices": choices},
-                      "timing": "CUDA graphs of %d steps, events around every step; L2 "
-                                "flushed before every step, outside the events" % G}))
+    return {"workload": f"{base.name} shape, one sequence, prefix {base.prefix[1]}, chain of l "
+                        f"drafts", "unit": "us per verify step", "steps_per_point": steps,
+            "points": points, "log_quadratic_fit": [float(c) for c in coef],
+            "controller": {"l_max": l_max, "latency_model": list(ctl.c), "choices": choices},
+            "timing": "CUDA graphs, events around every step; L2 flushed before every step, "
+                      "outside the events"}
 
 
-def run_e2e(vs, w, batch, K, stream, flush, world, tok_table, planned):
-    """Same metric through host buffers: every step copies its inputs (the
-    queries, proposal K/V of every layer, hidden states, tokens, tree and
-    lengths: one packed arena) from pinned host memory, runs the step and
-    reads its outputs (accepted lengths, tokens, new lengths: one arena)
-    back."""
+def run_ell_sweep(args):
     import torch
-    host_in = vs.in_arena.detach().cpu().pin_memory()
-    host_out = torch.empty(vs.out_arena.numel(), dtype=torch.uint8).pin_memory()
-    tok_off = vs.tokens.data_ptr() - vs.in_arena.data_ptr()
-    tok_bytes = vs.tokens.numel() * vs.tokens.element_size()
-    host_tokens = [t.cpu().contiguous().view(torch.uint8) for t in tok_table]
-    acc_off = vs.accept_len.data_ptr() - vs.out_arena.data_ptr()
-    h2d = host_in.numel()
-    d2h = host_out.numel()
-    g = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g, stream=stream):
-        vs.step(torch.cuda.current_stream().cuda_stream)
-    with torch.cuda.stream(stream):
-        g.replay()
-    stream.synchronize()
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    times = []
-    tok = 0
-    n = min(K, 200)
-    with torch.cuda.stream(stream):
-        for k in range(n):
-            flush.zero_()
-            host_in[tok_off:tok_off + tok_bytes].copy_(host_tokens[k % len(host_tokens)])
-            e0.record(stream)
-            vs.in_arena.copy_(host_in, non_blocking=True)
-            g.replay()
-            host_out.copy_(vs.out_arena, non_blocking=True)
-            e1.record(stream)
-            stream.synchronize()
-            times.append(e0.elapsed_time(e1))
-            acc = host_out[acc_off:acc_off + 4 * w.batch].view(torch.int32)
-            got = int((acc + 1).sum())
-            assert got == planned[k % len(planned)]
-            tok += got
-    t = max_over_ranks(float(np.sum(times)), world, "cuda")
-    return {"value": whole_job_rate(tok, t * 1e-3, world), "unit": "tokens/s",
-            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n, "ms_per_step": t / n,
-            "copies_per_step": {"h2d": 1, "d2h": 1}}
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_32166_gb300 import inputs as I
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.Stream()
+    r = ell_sweep(I.WORKLOADS[args.workload], args.seed, stream, flush, max(10, args.steps))
+    print(json.dumps(dict(mode="ell_sweep", **r)))
+
+
+# ---------------------------------------------------------------------------
+# main
+# ---------------------------------------------------------------------------
+def main():
+    args = parse()
+    if args.cpu_worker is not None:
+        print(json.dumps(cpu_worker(json.loads(args.cpu_worker))))
+        return
+    if args.impl == "reference":
+        run_reference(args)
+        return
+    if args.ell_sweep:
+        run_ell_sweep(args)
+        return
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    from paper_2609_32166_gb300 import inputs as I
+    w = I.WORKLOADS[args.workload]
+    if args.layers is not None:
+        w = I.scaled(w, layers=max(1, min(args.layers, w.layers)))
+
+    import torch
+    import torch.distributed as dist
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl")
+
+    import __graft_entry__
+    __graft_entry__.build()
+
+    peaks = load_peaks()
+    hbm_peak = peak_values(peaks)[0]
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.Stream()
+    K = args.steps
+    clocks = ClockSampler(torch.cuda.current_device())
+    head, vs, batch, tok_table, planned = measure_workload(
+        w, args, K, stream, flush, peaks, world=world, dist=dist, clocks=clocks)
+    e2e = None if args.no_e2e else run_e2e(vs, w, K, stream, flush, world, tok_table, planned)
+    weight_7b = vs.weight if (w.vocab, w.hidden) == (152064, 3584) else None
+    if world > 1:
+        dist.barrier()
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+    launches = head["gpu_launches_per_step"]
+    del vs
+    torch.cuda.empty_cache()
+
+    per_workload = {}
+    if not args.no_per_workload and args.layers is None:
+        for name in PER_WORKLOAD:
+            if name == w.name:
+                continue
+            wo = I.WORKLOADS[name]
+            share = weight_7b if (wo.vocab, wo.hidden) == (152064, 3584) else None
+            k_w = max(20, min(K, 200))
+            r, vso, *_ = measure_workload(wo, args, k_w, stream, flush, peaks, weight_dev=share)
+            del vso
+            torch.cuda.empty_cache()
+            per_workload[name] = r
+    next_rows = None
+    if not args.no_next_rows:
+        next_rows = measure_next_rows(stream, flush, hbm_peak)
+        next_rows["ell_sweep"] = ell_sweep(w, args.seed, stream, flush, 50, weight_dev=weight_7b)
+    del weight_7b
+    torch.cuda.empty_cache()
+
+    line = {
+        "metric": METRIC, "value": head["value"], "unit": "tokens/s", "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": head["ms_per_step"], "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
+        "data": "synthetic (seeded device generator; shapes and distributions of the named "
+                "workload)",
+        "config": config_dict(w, args),
+    }
+    for k in ("accepted_tokens_per_step", "us_per_layer_attention", "us_lmhead", "us_commit",
+              "parts", "step_hbm_gbs", "step_hbm_frac", "step_bytes", "step_roofline",
+              "roofline", "other_roofline", "clocks"):
+        line[k] = head[k]
+    line["gpu_launches"] = K * launches
+    line["timing"] = ("step time: CUDA graphs of up to 50 steps with events at every step "
+                      "boundary, exactly %d steps; per-part times: a second pass of %d steps with "
+                      "events around every step's parts" % (K, head["parts"]["steps"]))
+    line["e2e"] = e2e
+    line["per_workload"] = per_workload
+    line["next_rows"] = next_rows
+    if not args.no_cpu_baseline and world == 1:
+        spec = dict(workload=w.name, seed=args.seed, layers=args.layers, warmup=0, steps=1)
+        line["cpu_baseline"] = cpu_baseline_entry(w, spec)
+        for name, r in per_workload.items():
+            wo = I.WORKLOADS[name]
+            if cpu_mode(wo) == "whole":
+                r["cpu_baseline"] = cpu_baseline_entry(
+                    wo, dict(workload=name, seed=args.seed, warmup=0, steps=1))
+    print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
 
 
 if __name__ == "__main__":

@@ -77,6 +77,9 @@ typedef enum pf_kv_layout { PF_KV_CONTIGUOUS = 0, PF_KV_PAGED = 1 } pf_kv_layout
 #define PF_DEVERR_BOUNDS 4     /* device-side sizes (cu_nodes, prefix_len,
                                   page_table) contradict the host bounds;
                                   the affected work was skipped            */
+#define PF_DEVERR_TREE 8       /* a device-side parent array is not a
+                                  topologically ordered tree
+                                  (pf_tree_prepare_device)                 */
 
 /* Message for the last non-OK status returned on this host thread. */
 PF_API const char* pf_last_error(void);
@@ -96,6 +99,33 @@ PF_API int32_t pf_version(void);
  */
 PF_API pf_status pf_tree_prepare(const int32_t* parent, int32_t n_nodes,
                           int32_t* depth_out, uint64_t* mask_out);
+
+/*
+ * pf_tree_prepare_device -- the same for a batch of proposal trees already
+ * in device memory, stream-ordered (no host synchronisation), for decode
+ * loops whose proposal changes every step (Section 3.2: a new proposal is
+ * retrieved and verified at every decoding iteration).
+ *   parent     device [total_nodes]: sequence b's tree at cu_nodes[b] ..
+ *              cu_nodes[b+1]-1, parent indices local to the sequence
+ *              (-1 at its root)
+ *   cu_nodes   device [batch+1], cu_nodes[0] = 0, cu_nodes[batch] =
+ *              total_nodes
+ *   depth_out  device [total_nodes] or NULL
+ *   mask_out   device [total_nodes][PF_MASK_WORDS], the layout
+ *              pf_verify_attention reads
+ *   error_flag optional device int32
+ * Host checks: batch >= 1, 1 <= max_nodes <= PF_MAX_NODES, total_nodes >= 1,
+ * mask_out 16-byte aligned.  Device checks: a sequence whose node count is
+ * outside 1..max_nodes or whose nodes fall outside 0..total_nodes-1 ORs
+ * PF_DEVERR_BOUNDS and is skipped; a sequence whose parent array is not a
+ * topologically ordered tree (parent[0] != -1, or parent[j] outside
+ * [0, j)) ORs PF_DEVERR_TREE and gets masks with only each node's own bit
+ * and depth -1, so no later kernel reads outside the tree.  One launch.
+ */
+PF_API pf_status pf_tree_prepare_device(const int32_t* parent, const int32_t* cu_nodes,
+                                        int32_t batch, int32_t total_nodes, int32_t max_nodes,
+                                        int32_t* depth_out, uint64_t* mask_out,
+                                        int32_t* error_flag, void* stream);
 
 /* One layer's prefix KV cache. */
 typedef struct pf_kv_view {
@@ -149,7 +179,32 @@ typedef struct pf_attn_desc {
   int32_t flags;               /* PF_ATTN_* bits, 0 = none                   */
   void* workspace;             /* optional device scratch (see below)        */
   size_t workspace_bytes;      /* its size                                   */
+  /* Launch choices (0 = the library's automatic choice for the shape).
+   * They change which kernel runs and how the work is split, never the
+   * result beyond floating-point rounding order. */
+  int32_t kernel;              /* pf_attn_kernel                             */
+  int32_t splits;              /* K/V splits per row block (cluster width):
+                                  1..16; 1..8 for PF_ATTN_KERNEL_PAIR        */
+  int32_t rows_per_cta;        /* PF_ATTN_KERNEL_TC64: 128 or 256            */
+  int32_t stages;              /* PF_ATTN_KERNEL_TC128 ring depth: 2 or 3    */
 } pf_attn_desc;
+
+/* Attention kernels (bf16; the fp32 path has one kernel and takes 0).
+ *   MMA    warp-level mma.sync tiles (D = 64 or 128)
+ *   TC64   tcgen05 tensor cores, 64-token K/V tiles, 128 or 256 query rows
+ *          per CTA; the only kernel for head sizes other than 128 on them
+ *   TC128  tcgen05, 128-token tiles with P kept in tensor memory, 128 rows
+ *          per CTA (no balanced batch mode: a workspace is ignored)
+ *   PAIR   tcgen05 on pairs of SMs (one 2-SM MMA of 256 query rows per
+ *          128-token tile, each SM loading half of every K/V tile)
+ * TC64, TC128 and PAIR need bf16 and D = 128. */
+typedef enum pf_attn_kernel {
+  PF_ATTN_KERNEL_AUTO = 0,
+  PF_ATTN_KERNEL_MMA = 1,
+  PF_ATTN_KERNEL_TC64 = 2,
+  PF_ATTN_KERNEL_TC128 = 3,
+  PF_ATTN_KERNEL_PAIR = 4
+} pf_attn_kernel;
 
 /* PF_ATTN_EARLY_PREFETCH: the prefix cache, page_table, cu_nodes, prefix_len
  * and mask were all written before the kernel that precedes this call in the
@@ -160,6 +215,9 @@ typedef struct pf_attn_desc {
  * read only after it finishes.  Leave it clear when the preceding kernel may
  * write any of those inputs. */
 #define PF_ATTN_EARLY_PREFETCH 1
+/* PF_ATTN_NO_PDL: launch without programmatic dependent launch (the kernel
+ * then starts only after the preceding kernel in the stream has finished). */
+#define PF_ATTN_NO_PDL 2
 
 /* Workspace (optional; batches of B > 1 sequences, bf16, head_dim 128):
  * with workspace != NULL and at least pf_verify_attention_workspace_size(d)
@@ -216,6 +274,9 @@ typedef struct pf_lm_desc {
   int32_t* last_node;          /* out device [B], optional                   */
   int32_t* error_flag;         /* optional device int32                      */
   int32_t flags;               /* PF_LM_* bits, 0 = none                     */
+  int32_t stages;              /* bf16 weight-tile pipeline depth: 0 = the
+                                  library's choice, else 2..16 (at most 12
+                                  are used, fewer if shared memory is short) */
 } pf_lm_desc;
 
 /* PF_LM_EARLY_WEIGHT: the weight was written before the kernel that precedes
@@ -224,6 +285,8 @@ typedef struct pf_lm_desc {
  * preceding kernel to finish (programmatic dependent launch); the hidden
  * states, tokens and tree are read only after it finishes. */
 #define PF_LM_EARLY_WEIGHT 1
+/* PF_LM_NO_PDL: launch without programmatic dependent launch. */
+#define PF_LM_NO_PDL 2
 
 PF_API size_t pf_lmhead_accept_workspace_size(const pf_lm_desc* d);
 PF_API pf_status pf_lmhead_accept(const pf_lm_desc* d, void* workspace, size_t workspace_bytes,
@@ -232,20 +295,22 @@ PF_API pf_status pf_lmhead_accept(const pf_lm_desc* d, void* workspace, size_t w
 /*
  * pf_lmhead_accept_noalloc -- pf_lmhead_accept without a workspace argument.
  * The paper has no counterpart: this exists for callers that cannot
- * allocate device memory where they verify, e.g. code running while a
- * stream is being captured into a CUDA graph (cudaMalloc is not allowed
- * there), plug-ins whose host framework owns every device allocation, and
- * loops that must never reach the allocator.  The scratch lives in a
- * file-scope device array of 2112 bytes (room for PF_MAX_LM_ROWS = 256
- * proposal rows) that every GPU loading this library holds until exit;
- * total_nodes above 256 is rejected with PF_ERR_SHAPE.  The first call on
- * each device looks up that array's device address (cudaGetSymbolAddress),
- * so make the first call on a device before any stream capture.  Every call
- * clears the array (cudaMemsetAsync on the given stream) and then runs
- * exactly pf_lmhead_accept; nothing is allocated or freed.  All calls share
- * the one array, so calls that overlap on the GPU (other streams, other
- * host threads) race: serialise them.  Same outputs and errors as
- * pf_lmhead_accept otherwise.
+ * allocate device memory where they verify -- plug-ins whose host framework
+ * owns every device allocation, and decode loops that must never reach an
+ * allocator (allocating can synchronise the device or fail under memory
+ * pressure).  The scratch lives in a file-scope device array of 2112 bytes
+ * (room for PF_MAX_LM_ROWS = 256 proposal rows) that every GPU loading this
+ * library holds until exit; total_nodes above 256 is rejected with
+ * PF_ERR_SHAPE.  The first call on each device looks up that array's device
+ * address (cudaGetSymbolAddress) and keeps it for the life of the process,
+ * so make the first call on a device before any stream capture, and make no
+ * call after cudaDeviceReset (the reset discards the array the kept address
+ * points to).  Every call checks its arguments, then clears the array
+ * (cudaMemsetAsync on the given stream) and runs exactly pf_lmhead_accept;
+ * a rejected call queues nothing, and nothing is allocated or freed.  All
+ * calls share the one array, so calls that overlap on the GPU (other
+ * streams, other host threads) race: serialise them.  Same outputs and
+ * errors as pf_lmhead_accept otherwise.
  */
 PF_API pf_status pf_lmhead_accept_noalloc(const pf_lm_desc* d, void* stream);
 

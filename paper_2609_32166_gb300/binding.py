@@ -25,9 +25,11 @@ PF_ERR_CAPACITY, PF_ERR_ALIGN, PF_ERR_CUDA, PF_ERR_WORKSPACE = 5, 6, 7, 8
 PF_F32, PF_BF16 = 0, 1
 PF_KV_CONTIGUOUS, PF_KV_PAGED = 0, 1
 PF_MAX_NODES, PF_MASK_WORDS, PF_PAGE_SIZE, PF_MAX_LM_ROWS = 128, 2, 16, 256
-PF_DEVERR_TIMEOUT, PF_DEVERR_CAPACITY, PF_DEVERR_BOUNDS = 1, 2, 4
-PF_ATTN_EARLY_PREFETCH = 1
-PF_LM_EARLY_WEIGHT = 1
+PF_DEVERR_TIMEOUT, PF_DEVERR_CAPACITY, PF_DEVERR_BOUNDS, PF_DEVERR_TREE = 1, 2, 4, 8
+PF_ATTN_EARLY_PREFETCH, PF_ATTN_NO_PDL = 1, 2
+PF_LM_EARLY_WEIGHT, PF_LM_NO_PDL = 1, 2
+(PF_ATTN_KERNEL_AUTO, PF_ATTN_KERNEL_MMA, PF_ATTN_KERNEL_TC64, PF_ATTN_KERNEL_TC128,
+ PF_ATTN_KERNEL_PAIR) = 0, 1, 2, 3, 4
 
 STATUS_NAMES = {0: "PF_OK", 1: "PF_ERR_NULL", 2: "PF_ERR_SHAPE", 3: "PF_ERR_DTYPE",
                 4: "PF_ERR_TREE", 5: "PF_ERR_CAPACITY", 6: "PF_ERR_ALIGN", 7: "PF_ERR_CUDA",
@@ -58,7 +60,9 @@ class pf_attn_desc(C.Structure):
                 ("prefix_len", C.c_void_p), ("q", C.c_void_p), ("tree_k", C.c_void_p),
                 ("tree_v", C.c_void_p), ("mask", C.c_void_p), ("cache", pf_kv_view),
                 ("out", C.c_void_p), ("error_flag", C.c_void_p), ("flags", C.c_int32),
-                ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t)]
+                ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t),
+                ("kernel", C.c_int32), ("splits", C.c_int32), ("rows_per_cta", C.c_int32),
+                ("stages", C.c_int32)]
 
 
 class pf_lm_desc(C.Structure):
@@ -69,7 +73,7 @@ class pf_lm_desc(C.Structure):
                 ("argmax", C.c_void_p), ("max_logit", C.c_void_p),
                 ("accept_len", C.c_void_p), ("path", C.c_void_p),
                 ("out_tokens", C.c_void_p), ("last_node", C.c_void_p),
-                ("error_flag", C.c_void_p), ("flags", C.c_int32)]
+                ("error_flag", C.c_void_p), ("flags", C.c_int32), ("stages", C.c_int32)]
 
 
 class pf_commit_desc(C.Structure):
@@ -137,6 +141,9 @@ def lib() -> C.CDLL:
     L.pf_version.restype = C.c_int32
     L.pf_tree_prepare.restype = C.c_int
     L.pf_tree_prepare.argtypes = [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p]
+    L.pf_tree_prepare_device.restype = C.c_int
+    L.pf_tree_prepare_device.argtypes = [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_int32,
+                                         C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]
     L.pf_verify_attention.restype = C.c_int
     L.pf_verify_attention.argtypes = [C.POINTER(pf_attn_desc), C.c_void_p]
     L.pf_verify_attention_workspace_size.restype = C.c_size_t
@@ -206,6 +213,17 @@ def pf_tree_prepare(parent) -> tuple:
     mask = np.zeros((max(n, 1), PF_MASK_WORDS), dtype=np.uint64)
     _check(lib().pf_tree_prepare(p.ctypes.data, n, depth.ctypes.data, mask.ctypes.data))
     return depth[:n], mask[:n]
+
+
+def pf_tree_prepare_device(parent: int, cu_nodes: int, batch: int, total_nodes: int,
+                           max_nodes: int, depth_out: int, mask_out: int, error_flag: int = 0,
+                           stream: int = 0) -> None:
+    """Device call (pointers are device addresses; depth_out and error_flag
+    may be 0): ancestor bitmaps and depths of a batch of trees."""
+    _check(lib().pf_tree_prepare_device(C.c_void_p(parent), C.c_void_p(cu_nodes), batch,
+                                        total_nodes, max_nodes, C.c_void_p(depth_out or None),
+                                        C.c_void_p(mask_out), C.c_void_p(error_flag or None),
+                                        C.c_void_p(stream)))
 
 
 def pf_verify_attention_workspace_size(desc: pf_attn_desc) -> int:

@@ -37,14 +37,6 @@ pf_status cuda_fail(cudaError_t e, const char* what) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-bool pdl_enabled() {
-  static const bool on = [] {
-    const char* e = getenv("PF_PDL");
-    return !(e && e[0] == '0');
-  }();
-  return on;
-}
-
 int num_sms() {
   static pf::DeviceMemo cache;
   int dev = 0;
@@ -110,14 +102,17 @@ pf_status check_cache_view(const pf_kv_view& c, int need_rows, const char* who) 
   return PF_OK;
 }
 
-// Launch shape of the bf16 attention: query rows per CTA (32, 64 or 128)
-// and KV splits per cluster (<= 16).  Small problems take small row blocks
-// and wide clusters so that enough SMs stream the cache; large ones keep
-// 128-row blocks so each K/V tile serves more rows.  A cluster wider than 8
-// is used only if the device can schedule it.
-// kernel index 0..2: mma.sync BM 32/64/128; 3: tcgen05
+// ---------------------------------------------------------------------------
+// Attention launch shape.  Which kernel runs and how a layer's work is split
+// (query rows per CTA, K/V splits per row block, the balanced batch mode)
+// follows from the shape, unless the descriptor's launch fields ask for
+// something specific; nothing is read from the environment.
+// ---------------------------------------------------------------------------
+enum class AttnKernel { F32, MMA, TC64, TC128, PAIR };
+
+// kernel index 0..2: mma.sync BM 32/64/128
 int max_cluster_for(int kernel, int D, int want) {
-  static std::atomic<int> cache[64][4][2][17];
+  static std::atomic<int> cache[64][3][2][17];
   int dev = 0;
   cudaGetDevice(&dev);
   const int di = D == 64 ? 0 : 1;
@@ -131,131 +126,212 @@ int max_cluster_for(int kernel, int D, int want) {
       slot.store(c, std::memory_order_release);
     }
     if (c > 0) break;
-    w -= kernel == 3 ? 2 : 1;
+    w -= 1;
   }
   return w;
 }
 
-int tc_max_active_clusters(int cluster, int bm) {
-  static std::atomic<int> cache[64][2][17];
+// How many clusters of `cluster` CTAs fit on the device at once, per kernel
+// variant (memoised per device): 0 tc64 128 rows, 1 tc64 256 rows, 2 tc128
+// 3 stages, 3 tc128 2 stages, 4 pair.
+int max_active_clusters(int variant, int cluster) {
+  static std::atomic<int> cache[64][5][17];
   int dev = 0;
   cudaGetDevice(&dev);
-  std::atomic<int>& slot = cache[dev & 63][bm > 128 ? 1 : 0][cluster];
+  std::atomic<int>& slot = cache[dev & 63][variant][cluster];
   int c = slot.load(std::memory_order_acquire);
   if (c == 0) {
-    c = std::max(1, pf::attention_tc_max_active_clusters(cluster, bm)) + 1;
-    slot.store(c, std::memory_order_release);
-  }
-  return c - 1;
-}
-
-int tc2_max_active_clusters(int cluster) {
-  static std::atomic<int> cache[64][17];
-  int dev = 0;
-  cudaGetDevice(&dev);
-  std::atomic<int>& slot = cache[dev & 63][cluster];
-  int c = slot.load(std::memory_order_acquire);
-  if (c == 0) {
-    c = std::max(1, pf::attention_tc2_max_active_clusters(cluster)) + 1;
-    slot.store(c, std::memory_order_release);
-  }
-  return c - 1;
-}
-
-// The tcgen05 kernels serve bf16 with D = 128 (PF_ATTN_IMPL=mma selects the
-// mma.sync kernel instead).
-bool use_tc_attention(const pf::AttnArgs& a) {
-  const char* e = getenv("PF_ATTN_IMPL");
-  return a.D == 128 && !(e && strcmp(e, "mma") == 0);
-}
-
-// 128-token tiles (attn_tc2_kernel) for 128-row CTAs outside the balanced
-// batch mode once a CTA holds at least four 64-token tiles: per tile the
-// wider S MMA halves the UMMA instructions per key, while a CTA with one or
-// two tiles gains more from starting on a first, smaller tile (2B chain:
-// 6.70 us per layer with 64-token tiles, 6.95 with 128).  PF_ATTN_IMPL=tc64
-// or tc128 forces either.  `max_tiles` counts 64-token tiles.
-bool use_tc2_attention(const pf::AttnArgs& a, int max_prefix_len) {
-  if (!use_tc_attention(a) || a.bm != 128 || a.items != 0) return false;
-  const char* e = getenv("PF_ATTN_IMPL");
-  if (e && strcmp(e, "tc64") == 0) return false;
-  if (e && strcmp(e, "tc128") == 0) return true;
-  const int max_tiles = (max_prefix_len + 63) / 64 + (a.max_nodes + 63) / 64;
-  return (max_tiles + a.splits - 1) / a.splits >= 4;
-}
-
-// Splits for attn_tc2_kernel: the widest even cluster, at most the tile
-// count, whose clusters all fit on the GPU at once.
-void choose_tc2_splits(pf::AttnArgs& a, int max_prefix_len) {
-  const int max_tiles = (max_prefix_len + 127) / 128 + (a.max_nodes + 127) / 128;
-  const int groups = a.B * a.Hkv * a.rb_count;
-  int splits = std::min(16, max_tiles);
-  if (splits > 1) splits &= ~1;
-  for (; splits > 1; splits -= 2)
-    if (tc2_max_active_clusters(splits) >= groups) break;
-  if (const char* e = getenv("PF_ATTN_SPLITS")) splits = std::max(1, std::min(16, atoi(e)));
-  a.splits = std::max(1, splits);
-}
-
-void choose_attention_shape(pf::AttnArgs& a, int max_prefix_len, int sms) {
-  const int max_tiles = (max_prefix_len + 63) / 64 + (a.max_nodes + 63) / 64;
-  if (use_tc_attention(a)) {
-    // Two 128-row blocks per CTA (each K/V tile serves 256 rows, two
-    // softmax warpgroups) when that covers all of a KV head's rows; beyond
-    // 256 rows the tensor pipe of one SM, not the tile reads, bounds a CTA,
-    // and 128-row CTAs spread the work over more SMs.
-    const int head_rows = a.G * a.max_nodes;
-    a.bm = head_rows > 128 && head_rows <= 256 ? 256 : 128;
-    if (const char* e = getenv("PF_ATTN_BM")) a.bm = atoi(e) > 128 ? 256 : 128;
-    a.nb = a.bm / a.G;
-    a.rb_count = (a.max_nodes + a.nb - 1) / a.nb;
-    // One CTA per SM (shared memory), clusters must be co-resident: take the
-    // widest even split whose clusters all fit on the GPU at once, so the
-    // grid runs in one wave (odd cluster sizes strand SMs of an SM pair).
-    const int groups = a.B * a.Hkv * a.rb_count;
-    int splits = std::min(16, max_tiles);
-    if (splits > 1) splits &= ~1;
-    for (; splits > 1; splits -= 2)
-      if (tc_max_active_clusters(splits, a.bm) >= groups) break;
-    if (const char* e = getenv("PF_ATTN_SPLITS")) splits = std::max(1, std::min(16, atoi(e)));
-    a.splits = std::max(1, splits);
-    return;
-  }
-  const int bms[3] = {128, 64, 32};
-  int pick = 32;
-  for (int bm : bms) {
-    if (a.G > bm) break;
-    const int rb = (a.max_nodes + bm / a.G - 1) / (bm / a.G);
-    const int base = a.B * a.Hkv * rb;
-    const int per_sm = bm == 128 ? 1 : 2;
-    if (base * std::min(16, max_tiles) >= sms * per_sm || bm == 32) {
-      pick = bm;
-      break;
+    int n = 0;
+    switch (variant) {
+      case 0: n = pf::attention_tc_max_active_clusters(cluster, 128); break;
+      case 1: n = pf::attention_tc_max_active_clusters(cluster, 256); break;
+      case 2: n = pf::attention_tc2_max_active_clusters(cluster, 3); break;
+      case 3: n = pf::attention_tc2_max_active_clusters(cluster, 2); break;
+      default: n = pf::attention_pair_max_active_clusters(cluster, false); break;
     }
+    c = std::max(1, n) + 1;
+    slot.store(c, std::memory_order_release);
   }
-  if (a.G > pick) pick = 128;
-  if (const char* e = getenv("PF_ATTN_BM")) pick = atoi(e);
-  a.bm = pick;
-  a.nb = pick / a.G;
-  a.rb_count = (a.max_nodes + a.nb - 1) / a.nb;
-  const int base = a.B * a.Hkv * a.rb_count;
-  const int per_sm = pick == 128 ? 1 : 2;
-  int splits = (sms * per_sm) / base;
-  if (const char* e = getenv("PF_ATTN_SPLITS")) splits = atoi(e);
-  if (splits > 16) splits = 16;
-  if (splits > max_tiles) splits = max_tiles;
-  if (splits < 1) splits = 1;
-  if (splits > 8) splits = max_cluster_for(pick == 32 ? 0 : pick == 64 ? 1 : 2, a.D, splits);
-  a.splits = splits;
+  return c - 1;
 }
 
-// Balanced batch mode (tcgen05 path, B > 1): one CTA per SM, provided the
-// plan can give every (sequence, KV head, row block) group at least one.
-int balanced_items(const pf::AttnArgs& a, int sms) {
-  if (a.B < 2 || !use_tc_attention(a)) return 0;
+// The widest even cluster of at most `cap` CTAs (and at most `tiles`)
+// whose clusters all fit on the GPU at once, so the grid runs in one wave
+// (odd cluster sizes strand SMs of an SM pair); `step` CTAs per split.
+int widest_split(int variant, int groups, int tiles, int cap, int step) {
+  int splits = std::min(cap, tiles);
+  if (step == 1 && splits > 1) splits &= ~1;
+  for (; splits > 1; splits -= step == 1 ? 2 : 1)
+    if (max_active_clusters(variant, splits * step) >= groups) break;
+  return std::max(1, splits);
+}
+
+struct AttnChoice {
+  AttnKernel kernel;
+  int stages;       // TC128 ring depth
+  size_t ws_need;   // workspace bytes the balanced batch mode needs (0: not used)
+};
+
+// Validates the launch fields and fills a.bm, a.nb, a.rb_count, a.splits
+// and, when `ws_ok` and the shape allows, the balanced batch mode (a.items).
+pf_status choose_attention(const pf_attn_desc* d, pf::AttnArgs& a, int sms, bool ws_ok,
+                           AttnChoice* out, const char* who) {
+  const int D = a.D, G = a.G;
+  out->stages = d->stages == 2 ? 2 : 3;
+  out->ws_need = 0;
+  if (d->dtype == PF_F32) {
+    out->kernel = AttnKernel::F32;
+    a.nb = 0;
+    a.rb_count = (a.max_nodes * G + 31) / 32;
+    a.splits = 1;
+    return PF_OK;
+  }
+  AttnKernel k;
+  if (d->kernel == PF_ATTN_KERNEL_AUTO && d->rows_per_cta != 0) {
+    k = AttnKernel::TC64;
+  } else if (d->kernel == PF_ATTN_KERNEL_AUTO) {
+    // Tensor cores for D = 128: 128-row CTAs on 128-token tiles once a CTA
+    // holds several of them (wider S MMAs), else on 64-token tiles (a CTA
+    // with one or two tiles starts sooner on a smaller first tile); KV heads
+    // of 129..256 rows in two-block CTAs of the 64-token kernel.
+    k = D != 128 ? AttnKernel::MMA : AttnKernel::TC64;  // may become TC128 below
+  } else {
+    k = d->kernel == PF_ATTN_KERNEL_MMA    ? AttnKernel::MMA
+        : d->kernel == PF_ATTN_KERNEL_TC64 ? AttnKernel::TC64
+        : d->kernel == PF_ATTN_KERNEL_TC128 ? AttnKernel::TC128
+                                            : AttnKernel::PAIR;
+  }
+  const int tiles64 = (a.max_prefix + 63) / 64 + (a.max_nodes + 63) / 64;
+  const int tiles128 = (a.max_prefix + 127) / 128 + (a.max_nodes + 127) / 128;
+  const bool batch_ws = ws_ok && a.B > 1;
+
+  if (k == AttnKernel::MMA) {
+    const int bms[3] = {128, 64, 32};
+    int pick = 32;
+    for (int bm : bms) {
+      if (G > bm) break;
+      const int rb = (a.max_nodes + bm / G - 1) / (bm / G);
+      const int base = a.B * a.Hkv * rb;
+      const int per_sm = bm == 128 ? 1 : 2;
+      if (base * std::min(16, tiles64) >= sms * per_sm || bm == 32) {
+        pick = bm;
+        break;
+      }
+    }
+    if (G > pick) pick = 128;
+    a.bm = pick;
+    a.nb = pick / G;
+    a.rb_count = (a.max_nodes + a.nb - 1) / a.nb;
+    const int base = a.B * a.Hkv * a.rb_count;
+    const int per_sm = pick == 128 ? 1 : 2;
+    int splits = d->splits > 0 ? d->splits : (sms * per_sm) / base;
+    splits = std::max(1, std::min(std::min(16, tiles64), splits));
+    if (splits > 8) splits = max_cluster_for(pick == 32 ? 0 : pick == 64 ? 1 : 2, D, splits);
+    a.splits = splits;
+    out->kernel = k;
+    return PF_OK;
+  }
+
+  if (k == AttnKernel::PAIR) {
+    const int nbh = 128 / G;  // nodes per CTA (G <= 128)
+    a.bm = 256;
+    a.nb = 2 * nbh;
+    a.rb_count = (a.max_nodes + a.nb - 1) / a.nb;
+    const int groups = a.B * a.Hkv * a.rb_count;
+    const int items = sms / 2;  // one pair per SM pair
+    if (batch_ws && d->splits == 0 && groups <= items && groups <= pf::kPlanMaxGroups) {
+      a.splits = 1;
+      a.items = items;
+      out->ws_need = pf::attention_balanced_ws_bytes(items, a.bm, D);
+    } else {
+      a.splits = d->splits > 0 ? std::min(d->splits, std::max(1, tiles128))
+                               : widest_split(4, groups, tiles128, 8, 2);
+    }
+    out->kernel = k;
+    return PF_OK;
+  }
+
+  // TC64 / TC128: one 128-row block per CTA, or two (256 rows, TC64 only)
+  // where that covers all of a KV head's rows
+  const int head_rows = G * a.max_nodes;
+  a.bm = (k == AttnKernel::TC64 && head_rows > 128 && head_rows <= 256) ? 256 : 128;
+  if (d->rows_per_cta != 0) a.bm = d->rows_per_cta;
+  a.nb = a.bm / G;  // >= 1: G <= 128
+  a.rb_count = (a.max_nodes + a.nb - 1) / a.nb;
   const int groups = a.B * a.Hkv * a.rb_count;
-  if (groups > sms || groups > pf::kPlanMaxGroups) return 0;
-  return sms;
+  if (k == AttnKernel::TC64 && batch_ws && d->splits == 0 && groups <= sms &&
+      groups <= pf::kPlanMaxGroups) {
+    a.splits = 1;
+    a.items = sms;
+    out->ws_need = pf::attention_balanced_ws_bytes(sms, a.bm, D);
+    out->kernel = k;
+    return PF_OK;
+  }
+  a.splits = d->splits > 0 ? std::min(d->splits, tiles64)
+                           : widest_split(a.bm > 128 ? 1 : 0, groups, tiles64, 16, 1);
+  if (d->kernel == PF_ATTN_KERNEL_AUTO && a.bm == 128 &&
+      (tiles64 + a.splits - 1) / a.splits >= 4)
+    k = AttnKernel::TC128;
+  if (k == AttnKernel::TC128) {
+    a.splits = d->splits > 0 ? std::min(d->splits, tiles128)
+                             : widest_split(out->stages == 2 ? 3 : 2, groups, tiles128, 16, 1);
+  }
+  out->kernel = k;
+  return PF_OK;
+}
+
+// The fields of pf_attn_desc that the launch shape depends on, validated.
+pf_status attention_args(const pf_attn_desc* d, pf::AttnArgs& a, const char* who) {
+  if (d->dtype != PF_BF16 && d->dtype != PF_F32)
+    return fail(PF_ERR_DTYPE, "%s: dtype %d unsupported", who, d->dtype);
+  if (d->batch < 1 || d->n_kv_heads < 1 || d->n_q_heads < 1 ||
+      d->n_q_heads % d->n_kv_heads != 0)
+    return fail(PF_ERR_SHAPE, "%s: need batch >= 1 and n_q_heads a multiple of n_kv_heads", who);
+  const int D = d->head_dim;
+  const int G = d->n_q_heads / d->n_kv_heads;
+  if (d->dtype == PF_BF16 && D != 64 && D != 128)
+    return fail(PF_ERR_SHAPE, "%s: bf16 head_dim must be 64 or 128 (got %d)", who, D);
+  if (d->dtype == PF_F32 && (D < 1 || D > 128))
+    return fail(PF_ERR_SHAPE, "%s: fp32 head_dim must be in 1..128 (got %d)", who, D);
+  if (d->dtype == PF_BF16 && G > 128)
+    return fail(PF_ERR_SHAPE, "%s: query heads per KV head must be <= 128", who);
+  if (d->max_nodes < 1 || d->max_nodes > PF_MAX_NODES || d->total_nodes < 1)
+    return fail(PF_ERR_SHAPE, "%s: max_nodes must be in 1..%d and total_nodes >= 1", who,
+                PF_MAX_NODES);
+  if (d->max_prefix_len < 0) return fail(PF_ERR_SHAPE, "%s: max_prefix_len < 0", who);
+  if (d->flags & ~(PF_ATTN_EARLY_PREFETCH | PF_ATTN_NO_PDL))
+    return fail(PF_ERR_SHAPE, "%s: unknown flags 0x%x", who, d->flags);
+  // launch fields
+  if (d->kernel < PF_ATTN_KERNEL_AUTO || d->kernel > PF_ATTN_KERNEL_PAIR)
+    return fail(PF_ERR_SHAPE, "%s: unknown kernel %d", who, d->kernel);
+  if (d->dtype == PF_F32 && (d->kernel != PF_ATTN_KERNEL_AUTO || d->splits != 0 ||
+                             d->rows_per_cta != 0 || d->stages != 0))
+    return fail(PF_ERR_DTYPE, "%s: the fp32 path has one kernel and takes no launch fields",
+                who);
+  const bool tc_kernel = d->kernel == PF_ATTN_KERNEL_TC64 || d->kernel == PF_ATTN_KERNEL_TC128 ||
+                         d->kernel == PF_ATTN_KERNEL_PAIR;
+  if (tc_kernel && D != 128)
+    return fail(PF_ERR_SHAPE, "%s: the tcgen05 kernels need head_dim 128", who);
+  if (d->splits < 0 || d->splits > (d->kernel == PF_ATTN_KERNEL_PAIR ? 8 : 16))
+    return fail(PF_ERR_SHAPE, "%s: splits must be 0 (automatic) or 1..16 (1..8 for pairs)", who);
+  if (d->rows_per_cta != 0 &&
+      ((d->rows_per_cta != 128 && d->rows_per_cta != 256) || D != 128 ||
+       (d->kernel != PF_ATTN_KERNEL_AUTO && d->kernel != PF_ATTN_KERNEL_TC64) ||
+       G > d->rows_per_cta))
+    return fail(PF_ERR_SHAPE,
+                "%s: rows_per_cta (128 or 256, at least G) applies to the 64-token kernel", who);
+  if (d->stages != 0 && ((d->stages != 2 && d->stages != 3) || d->kernel != PF_ATTN_KERNEL_TC128))
+    return fail(PF_ERR_SHAPE, "%s: stages (2 or 3) applies to the 128-token kernel", who);
+  a.B = d->batch;
+  a.Hq = d->n_q_heads;
+  a.Hkv = d->n_kv_heads;
+  a.D = D;
+  a.G = G;
+  a.T = d->total_nodes;
+  a.max_nodes = d->max_nodes;
+  a.max_prefix = d->max_prefix_len;
+  a.flags = d->flags & PF_ATTN_EARLY_PREFETCH;
+  return PF_OK;
 }
 
 }  // namespace
@@ -272,11 +348,41 @@ pf_status set_error(pf_status s, const char* fmt, ...) {
 }
 }  // namespace pf
 
+namespace pf {
+// Every argument check of pf_lmhead_accept that does not involve the
+// workspace (pf_lmhead_accept_noalloc runs them before it touches its
+// scratch, so that a rejected call queues nothing).
+pf_status lmhead_check_desc(const pf_lm_desc* d, const char* who) {
+  if (!d) return fail(PF_ERR_NULL, "%s: desc is NULL", who);
+  if (!d->cu_nodes || !d->hidden_states || !d->weight || !d->tokens || !d->parent ||
+      !d->argmax || !d->accept_len || !d->path || !d->out_tokens)
+    return fail(PF_ERR_NULL, "%s: a required pointer is NULL", who);
+  if (d->dtype != PF_BF16 && d->dtype != PF_F32)
+    return fail(PF_ERR_DTYPE, "%s: dtype %d unsupported", who, d->dtype);
+  if (d->batch < 1 || d->hidden < 1 || d->vocab < 1)
+    return fail(PF_ERR_SHAPE, "%s: batch, hidden and vocab must be >= 1", who);
+  if (d->total_nodes < 1 || d->total_nodes > PF_MAX_LM_ROWS)
+    return fail(PF_ERR_SHAPE, "%s: total_nodes = %d outside 1..%d", who, d->total_nodes,
+                PF_MAX_LM_ROWS);
+  if (d->max_nodes < 1 || d->max_nodes > PF_MAX_NODES)
+    return fail(PF_ERR_SHAPE, "%s: max_nodes outside 1..%d", who, PF_MAX_NODES);
+  if (d->dtype == PF_BF16 && d->hidden % 8 != 0)
+    return fail(PF_ERR_ALIGN, "%s: bf16 hidden size must be a multiple of 8", who);
+  if (!aligned16(d->hidden_states) || !aligned16(d->weight))
+    return fail(PF_ERR_ALIGN, "%s: hidden and weight must be 16-byte aligned", who);
+  if (d->flags & ~(PF_LM_EARLY_WEIGHT | PF_LM_NO_PDL))
+    return fail(PF_ERR_SHAPE, "%s: unknown flags", who);
+  if (d->stages < 0 || d->stages == 1 || d->stages > 16)
+    return fail(PF_ERR_SHAPE, "%s: stages must be 0 (automatic) or 2..16", who);
+  return PF_OK;
+}
+}  // namespace pf
+
 extern "C" {
 
 const char* pf_last_error(void) { return g_last_error.c_str(); }
 
-int32_t pf_version(void) { return 100; }
+int32_t pf_version(void) { return 200; }
 
 pf_status pf_tree_prepare(const int32_t* parent, int32_t n_nodes, int32_t* depth_out,
                           uint64_t* mask_out) {
@@ -306,24 +412,41 @@ pf_status pf_tree_prepare(const int32_t* parent, int32_t n_nodes, int32_t* depth
   return PF_OK;
 }
 
+pf_status pf_tree_prepare_device(const int32_t* parent, const int32_t* cu_nodes, int32_t batch,
+                                 int32_t total_nodes, int32_t max_nodes, int32_t* depth_out,
+                                 uint64_t* mask_out, int32_t* error_flag, void* stream) {
+  static const char* who = "pf_tree_prepare_device";
+  if (!parent || !cu_nodes || !mask_out)
+    return fail(PF_ERR_NULL, "%s: parent, cu_nodes and mask_out are required", who);
+  if (batch < 1 || batch > 65535 || total_nodes < 1)
+    return fail(PF_ERR_SHAPE, "%s: need 1 <= batch <= 65535 and total_nodes >= 1", who);
+  if (max_nodes < 1 || max_nodes > PF_MAX_NODES)
+    return fail(PF_ERR_SHAPE, "%s: max_nodes outside 1..%d", who, PF_MAX_NODES);
+  if (!aligned16(mask_out)) return fail(PF_ERR_ALIGN, "%s: mask_out must be 16-byte aligned", who);
+  if (num_sms() <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
+  pf::TreeArgs a = {};
+  a.B = batch;
+  a.T = total_nodes;
+  a.max_nodes = max_nodes;
+  a.parent = parent;
+  a.cu_nodes = cu_nodes;
+  a.depth = depth_out;
+  a.mask = mask_out;
+  a.err = error_flag;
+  cudaError_t e = pf::launch_tree_prepare(a, static_cast<cudaStream_t>(stream), true);
+  return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
+}
+
 size_t pf_verify_attention_workspace_size(const pf_attn_desc* d) {
-  if (!d || d->dtype != PF_BF16 || d->batch < 2 || d->n_kv_heads < 1 || d->n_q_heads < 1 ||
-      d->n_q_heads % d->n_kv_heads != 0 || d->max_nodes < 1 || d->max_nodes > PF_MAX_NODES ||
-      d->max_prefix_len < 0)
-    return 0;
-  const int sms = num_sms();
-  if (sms <= 0) return 0;
+  if (!d) return 0;
+  const std::string saved = g_last_error;  // a size query leaves the last error alone
   pf::AttnArgs a = {};
-  a.B = d->batch;
-  a.Hq = d->n_q_heads;
-  a.Hkv = d->n_kv_heads;
-  a.D = d->head_dim;
-  a.G = a.Hq / a.Hkv;
-  a.max_nodes = d->max_nodes;
-  if (!use_tc_attention(a) || a.G > 128) return 0;
-  choose_attention_shape(a, d->max_prefix_len, sms);
-  const int items = balanced_items(a, sms);
-  return items > 0 ? pf::attention_balanced_ws_bytes(items, a.bm, a.D) : 0;
+  AttnChoice ch;
+  const int sms = num_sms();
+  const bool ok = sms > 0 && attention_args(d, a, "") == PF_OK &&
+                  choose_attention(d, a, sms, true, &ch, "") == PF_OK;
+  g_last_error = saved;
+  return ok ? ch.ws_need : 0;
 }
 
 pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
@@ -331,38 +454,15 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
   if (!d) return fail(PF_ERR_NULL, "%s: desc is NULL", who);
   if (!d->cu_nodes || !d->prefix_len || !d->q || !d->tree_k || !d->tree_v || !d->mask || !d->out)
     return fail(PF_ERR_NULL, "%s: a required pointer is NULL", who);
-  if (d->dtype != PF_BF16 && d->dtype != PF_F32)
-    return fail(PF_ERR_DTYPE, "%s: dtype %d unsupported", who, d->dtype);
-  if (d->batch < 1 || d->n_kv_heads < 1 || d->n_q_heads < 1 ||
-      d->n_q_heads % d->n_kv_heads != 0)
-    return fail(PF_ERR_SHAPE, "%s: need batch >= 1 and n_q_heads a multiple of n_kv_heads", who);
-  const int D = d->head_dim;
-  const int G = d->n_q_heads / d->n_kv_heads;
-  if (d->dtype == PF_BF16 && D != 64 && D != 128)
-    return fail(PF_ERR_SHAPE, "%s: bf16 head_dim must be 64 or 128 (got %d)", who, D);
-  if (d->dtype == PF_F32 && (D < 1 || D > 128))
-    return fail(PF_ERR_SHAPE, "%s: fp32 head_dim must be in 1..128 (got %d)", who, D);
-  if (d->dtype == PF_BF16 && G > 128)
-    return fail(PF_ERR_SHAPE, "%s: query heads per KV head must be <= 128", who);
-  if (d->max_nodes < 1 || d->max_nodes > PF_MAX_NODES || d->total_nodes < 1)
-    return fail(PF_ERR_SHAPE, "%s: max_nodes must be in 1..%d and total_nodes >= 1", who,
-                PF_MAX_NODES);
-  if (d->max_prefix_len < 0) return fail(PF_ERR_SHAPE, "%s: max_prefix_len < 0", who);
-  pf_status st = check_cache_view(d->cache, d->max_prefix_len, who);
+  pf::AttnArgs a = {};
+  pf_status st = attention_args(d, a, who);
+  if (st != PF_OK) return st;
+  st = check_cache_view(d->cache, d->max_prefix_len, who);
   if (st != PF_OK) return st;
   if (!aligned16(d->q) || !aligned16(d->tree_k) || !aligned16(d->tree_v) || !aligned16(d->out) ||
       !aligned16(d->mask))
     return fail(PF_ERR_ALIGN, "%s: tensor pointers must be 16-byte aligned", who);
-
-  pf::AttnArgs a = {};
-  a.B = d->batch;
-  a.Hq = d->n_q_heads;
-  a.Hkv = d->n_kv_heads;
-  a.D = D;
-  a.G = G;
-  a.T = d->total_nodes;
-  a.max_nodes = d->max_nodes;
-  a.max_prefix = d->max_prefix_len;
+  const int D = a.D, G = a.G;
   a.scale = d->scale > 0.f ? d->scale : 1.0f / sqrtf((float)D);
   a.scale_log2 = a.scale * 1.4426950408889634f;
   a.cu_nodes = d->cu_nodes;
@@ -381,58 +481,53 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
   a.ck = d->cache.k;
   a.cv = d->cache.v;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const bool pdl = (d->flags & PF_ATTN_NO_PDL) == 0;
   const int sms = num_sms();
   if (sms <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
 
-  if (d->dtype == PF_F32) {
-    a.nb = 0;
-    a.rb_count = (d->max_nodes * G + 31) / 32;
-    a.splits = 1;
-    cudaError_t e = pf::launch_attention_f32(a, s, pdl_enabled());
+  AttnChoice ch;
+  st = choose_attention(d, a, sms, d->workspace != nullptr, &ch, who);
+  if (st != PF_OK) return st;
+  if (ch.kernel == AttnKernel::F32) {
+    cudaError_t e = pf::launch_attention_f32(a, s, pdl);
     return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
   }
-
-  if (d->flags & ~PF_ATTN_EARLY_PREFETCH)
-    return fail(PF_ERR_SHAPE, "%s: unknown flags 0x%x", who, d->flags);
-  a.flags = d->flags;
-  choose_attention_shape(a, d->max_prefix_len, sms);
-  if (d->workspace) {
-    const int items = balanced_items(a, sms);
-    if (items > 0) {
-      const size_t need = pf::attention_balanced_ws_bytes(items, a.bm, a.D);
-      if (d->workspace_bytes < need)
-        return fail(PF_ERR_WORKSPACE, "%s: workspace needs %zu bytes", who, need);
-      if (!aligned16(d->workspace))
-        return fail(PF_ERR_ALIGN, "%s: workspace must be 16-byte aligned", who);
-      a.splits = 1;
-      a.items = items;
-      a.ws = d->workspace;
-    }
+  if (a.items > 0) {
+    if (d->workspace_bytes < ch.ws_need)
+      return fail(PF_ERR_WORKSPACE, "%s: workspace needs %zu bytes", who, ch.ws_need);
+    if (!aligned16(d->workspace))
+      return fail(PF_ERR_ALIGN, "%s: workspace must be 16-byte aligned", who);
+    a.ws = d->workspace;
   }
-  const bool tc2 = use_tc2_attention(a, d->max_prefix_len);
-  if (tc2) choose_tc2_splits(a, d->max_prefix_len);
-  const cuuint32_t tile_rows = tc2 ? 128 : 64;  // K/V tile height of the chosen kernel
+  // Tensor maps: K/V boxes of the chosen kernel's tile (the pair kernel
+  // loads half a tile per CTA: 64 K rows, 128 V rows of 64 columns).
+  const bool pair = ch.kernel == AttnKernel::PAIR;
+  const cuuint32_t k_rows = pair ? 64 : ch.kernel == AttnKernel::TC128 ? 128 : 64;
+  const cuuint32_t v_rows = pair ? 128 : k_rows;
+  const cuuint32_t q_nodes = pair ? (cuuint32_t)(a.nb / 2) : (cuuint32_t)a.nb;
   pf::AttnMaps m;
   const cuuint64_t es = 2;
   {
     cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)a.Hq, (cuuint64_t)a.T};
     cuuint64_t str[2] = {D * es, (cuuint64_t)a.Hq * D * es};
-    cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)a.nb};  // nb * G <= bm rows
+    cuuint32_t box[3] = {64, (cuuint32_t)G, q_nodes};  // q_nodes * G <= 128 rows
     if ((st = make_map(&m.q, 3, d->q, dims, str, box, "q")) != PF_OK) return st;
   }
   {
     cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)a.Hkv, (cuuint64_t)a.T};
     cuuint64_t str[2] = {D * es, (cuuint64_t)a.Hkv * D * es};
-    cuuint32_t box[3] = {64, 1, tile_rows};
-    if ((st = make_map(&m.tk, 3, d->tree_k, dims, str, box, "tree_k")) != PF_OK) return st;
-    if ((st = make_map(&m.tv, 3, d->tree_v, dims, str, box, "tree_v")) != PF_OK) return st;
+    cuuint32_t kbox[3] = {64, 1, k_rows};
+    cuuint32_t vbox[3] = {64, 1, v_rows};
+    if ((st = make_map(&m.tk, 3, d->tree_k, dims, str, kbox, "tree_k")) != PF_OK) return st;
+    if ((st = make_map(&m.tv, 3, d->tree_v, dims, str, vbox, "tree_v")) != PF_OK) return st;
   }
   if (a.layout == PF_KV_CONTIGUOUS) {
     cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)a.max_seq, (cuuint64_t)a.B * a.Hkv};
     cuuint64_t str[2] = {D * es, (cuuint64_t)a.max_seq * D * es};
-    cuuint32_t box[3] = {64, tile_rows, 1};
-    if ((st = make_map(&m.ck, 3, d->cache.k, dims, str, box, "cache.k")) != PF_OK) return st;
-    if ((st = make_map(&m.cv, 3, d->cache.v, dims, str, box, "cache.v")) != PF_OK) return st;
+    cuuint32_t kbox[3] = {64, k_rows, 1};
+    cuuint32_t vbox[3] = {64, v_rows, 1};
+    if ((st = make_map(&m.ck, 3, d->cache.k, dims, str, kbox, "cache.k")) != PF_OK) return st;
+    if ((st = make_map(&m.cv, 3, d->cache.v, dims, str, vbox, "cache.v")) != PF_OK) return st;
   } else {
     cuuint64_t dims[4] = {(cuuint64_t)D, PF_PAGE_SIZE, (cuuint64_t)a.Hkv,
                           (cuuint64_t)a.num_pages};
@@ -441,37 +536,29 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
     if ((st = make_map(&m.ck, 4, d->cache.k, dims, str, box, "cache.k")) != PF_OK) return st;
     if ((st = make_map(&m.cv, 4, d->cache.v, dims, str, box, "cache.v")) != PF_OK) return st;
   }
-  cudaError_t e = tc2 ? pf::launch_attention_tc2(a, m, s, pdl_enabled())
-                 : use_tc_attention(a) ? pf::launch_attention_tc(a, m, s, pdl_enabled())
-                                       : pf::launch_attention_bf16(a, m, s, sms, pdl_enabled());
-  if (e == cudaSuccess && a.items > 0) e = pf::launch_attention_combine(a, s, pdl_enabled());
+  cudaError_t e;
+  switch (ch.kernel) {
+    case AttnKernel::PAIR: e = pf::launch_attention_pair(a, m, s, pdl); break;
+    case AttnKernel::TC128: e = pf::launch_attention_tc2(a, m, s, pdl, ch.stages); break;
+    case AttnKernel::TC64: e = pf::launch_attention_tc(a, m, s, pdl); break;
+    default: e = pf::launch_attention_bf16(a, m, s, sms, pdl); break;
+  }
+  if (e == cudaSuccess && a.items > 0) e = pf::launch_attention_combine(a, s, pdl);
   return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
 }
 
 size_t pf_lmhead_accept_workspace_size(const pf_lm_desc*) { return pf::kLmWorkspaceBytes; }
 
+
 pf_status pf_lmhead_accept(const pf_lm_desc* d, void* workspace, size_t workspace_bytes,
                            void* stream) {
   static const char* who = "pf_lmhead_accept";
-  if (!d) return fail(PF_ERR_NULL, "%s: desc is NULL", who);
-  if (!d->cu_nodes || !d->hidden_states || !d->weight || !d->tokens || !d->parent ||
-      !d->argmax || !d->accept_len || !d->path || !d->out_tokens)
-    return fail(PF_ERR_NULL, "%s: a required pointer is NULL", who);
+  const pf_status chk = pf::lmhead_check_desc(d, who);
+  if (chk != PF_OK) return chk;
   if (!workspace || workspace_bytes < pf::kLmWorkspaceBytes)
     return fail(PF_ERR_WORKSPACE, "%s: workspace needs %zu bytes", who, pf::kLmWorkspaceBytes);
-  if (d->dtype != PF_BF16 && d->dtype != PF_F32)
-    return fail(PF_ERR_DTYPE, "%s: dtype %d unsupported", who, d->dtype);
-  if (d->batch < 1 || d->hidden < 1 || d->vocab < 1)
-    return fail(PF_ERR_SHAPE, "%s: batch, hidden and vocab must be >= 1", who);
-  if (d->total_nodes < 1 || d->total_nodes > PF_MAX_LM_ROWS)
-    return fail(PF_ERR_SHAPE, "%s: total_nodes = %d outside 1..%d", who, d->total_nodes,
-                PF_MAX_LM_ROWS);
-  if (d->max_nodes < 1 || d->max_nodes > PF_MAX_NODES)
-    return fail(PF_ERR_SHAPE, "%s: max_nodes outside 1..%d", who, PF_MAX_NODES);
-  if (d->dtype == PF_BF16 && d->hidden % 8 != 0)
-    return fail(PF_ERR_ALIGN, "%s: bf16 hidden size must be a multiple of 8", who);
-  if (!aligned16(d->hidden_states) || !aligned16(d->weight) || !aligned16(workspace))
-    return fail(PF_ERR_ALIGN, "%s: hidden, weight and workspace must be 16-byte aligned", who);
+  if (!aligned16(workspace))
+    return fail(PF_ERR_ALIGN, "%s: workspace must be 16-byte aligned", who);
 
   pf::LmArgs a = {};
   a.T = d->total_nodes;
@@ -494,8 +581,8 @@ pf_status pf_lmhead_accept(const pf_lm_desc* d, void* workspace, size_t workspac
   a.best = static_cast<unsigned long long*>(workspace);
   a.ticket = reinterpret_cast<unsigned int*>(static_cast<char*>(workspace) + 8 * PF_MAX_LM_ROWS);
   a.err = d->error_flag;
-  if (d->flags & ~PF_LM_EARLY_WEIGHT) return fail(PF_ERR_SHAPE, "%s: unknown flags", who);
-  a.flags = d->flags;
+  a.flags = d->flags & PF_LM_EARLY_WEIGHT;
+  const bool pdl = (d->flags & PF_LM_NO_PDL) == 0;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int sms = num_sms();
   if (sms <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
@@ -503,10 +590,10 @@ pf_status pf_lmhead_accept(const pf_lm_desc* d, void* workspace, size_t workspac
   if (d->dtype == PF_F32) {
     a.hidden_f32 = static_cast<const float*>(d->hidden_states);
     a.weight_f32 = static_cast<const float*>(d->weight);
-    cudaError_t e = pf::launch_lmhead_f32(a, s, sms, pdl_enabled());
+    cudaError_t e = pf::launch_lmhead_f32(a, s, sms, pdl);
     return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
   }
-  a.stages = pf::lmhead_bf16_stages(a.npad);
+  a.stages = pf::lmhead_bf16_stages(a.npad, d->stages);
   CUtensorMap wm, hm;
   pf_status st;
   {
@@ -521,7 +608,7 @@ pf_status pf_lmhead_accept(const pf_lm_desc* d, void* workspace, size_t workspac
     cuuint32_t box[2] = {64, (cuuint32_t)a.npad};
     if ((st = make_map(&hm, 2, d->hidden_states, dims, str, box, "hidden")) != PF_OK) return st;
   }
-  cudaError_t e = pf::launch_lmhead_bf16(a, wm, hm, s, sms, pdl_enabled());
+  cudaError_t e = pf::launch_lmhead_bf16(a, wm, hm, s, sms, pdl);
   return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
 }
 
@@ -581,7 +668,7 @@ pf_status pf_kv_commit(const pf_commit_desc* d, void* stream) {
   a.err = d->error_flag;
   const int sms = num_sms();
   if (sms <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
-  cudaError_t e = pf::launch_kv_commit(a, static_cast<cudaStream_t>(stream), sms, pdl_enabled());
+  cudaError_t e = pf::launch_kv_commit(a, static_cast<cudaStream_t>(stream), sms, true);
   return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
 }
 
@@ -635,7 +722,7 @@ pf_status pf_kv_shift(const pf_shift_desc* d, void* stream) {
   }
   const int sms = num_sms();
   if (sms <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
-  cudaError_t e = pf::launch_kv_shift(a, static_cast<cudaStream_t>(stream), sms, pdl_enabled());
+  cudaError_t e = pf::launch_kv_shift(a, static_cast<cudaStream_t>(stream), sms, true);
   return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
 }
 
@@ -665,7 +752,7 @@ pf_status pf_retrieval_key(const pf_key_desc* d, void* workspace, size_t workspa
   a.ticket = reinterpret_cast<unsigned*>(static_cast<char*>(workspace) + pf::kRetrievalKeyTicketOff);
   a.err = d->error_flag;
   if (num_sms() <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
-  cudaError_t e = pf::launch_retrieval_key(a, static_cast<cudaStream_t>(stream), pdl_enabled());
+  cudaError_t e = pf::launch_retrieval_key(a, static_cast<cudaStream_t>(stream), true);
   return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
 }
 
@@ -701,7 +788,7 @@ pf_status pf_retrieve(const pf_retrieval_desc* d, void* workspace, size_t worksp
   a.err = d->error_flag;
   const int sms = num_sms();
   if (sms <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
-  cudaError_t e = pf::launch_retrieve(a, static_cast<cudaStream_t>(stream), sms, pdl_enabled());
+  cudaError_t e = pf::launch_retrieve(a, static_cast<cudaStream_t>(stream), sms, true);
   return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
 }
 
@@ -734,7 +821,7 @@ pf_status pf_prefix_match(const pf_prefix_desc* d, void* stream) {
   a.lcp = d->lcp;
   a.cache_len = d->cache_len;
   if (num_sms() <= 0) return fail(PF_ERR_CUDA, "%s: no CUDA device", who);
-  cudaError_t e = pf::launch_prefix_match(a, static_cast<cudaStream_t>(stream), pdl_enabled());
+  cudaError_t e = pf::launch_prefix_match(a, static_cast<cudaStream_t>(stream), true);
   return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
 }
 

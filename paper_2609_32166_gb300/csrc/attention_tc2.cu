@@ -64,28 +64,6 @@ struct W2Smem {
   static_assert(kTotal + 1024 <= 232448, "shared memory budget");
 };
 
-// Page-table entries of the eight 16-token pages of prefix tile t (-1 past
-// the prefix end), loaded together.
-struct Pages8 {
-  int4 lo, hi;
-};
-
-__device__ __forceinline__ Pages8 w2_tile_pages(const AttnArgs& a, int t, int n_ptiles, int b,
-                                                int P) {
-  Pages8 pg{make_int4(-1, -1, -1, -1), make_int4(-1, -1, -1, -1)};
-  if (a.layout != PF_KV_CONTIGUOUS && t < n_ptiles) {
-    const int tok0 = t * kW;
-    const int npages = min(kW / PF_PAGE_SIZE, (P - tok0 + PF_PAGE_SIZE - 1) / PF_PAGE_SIZE);
-    const int32_t* pt = a.page_table + (size_t)b * a.pages_per_seq + tok0 / PF_PAGE_SIZE;
-    int v[8];
-#pragma unroll
-    for (int p = 0; p < 8; ++p) v[p] = p < npages ? pt[p] : -1;
-    pg.lo = make_int4(v[0], v[1], v[2], v[3]);
-    pg.hi = make_int4(v[4], v[5], v[6], v[7]);
-  }
-  return pg;
-}
-
 // TMA loads of one 128-token K/V tile into a ring stage: K then V, each two
 // 64-column halves of 128 rows.  Prefix cache: one 3-D box of 128 rows per
 // half (contiguous) or one 4-D box per 16-token page holding prefix rows
@@ -227,8 +205,8 @@ __global__ void __launch_bounds__(kW2Threads, 1)
     Pages8 pg[kW2Stages];  // every first tile's page entries in one round trip
 #pragma unroll
     for (int i = 0; i < kW2Stages; ++i)
-      pg[i] = i < first ? w2_tile_pages(a, tile_at(i), n_ptiles, b, P)
-                        : Pages8{make_int4(-1, -1, -1, -1), make_int4(-1, -1, -1, -1)};
+      pg[i] = i < first ? kv_tile_pages8(a, tile_at(i), n_ptiles, b, P)
+                        : no_pages8();
 #pragma unroll
     for (int i = 0; i < kW2Stages; ++i)
       if (i < first && i < my_ptiles)
@@ -246,7 +224,7 @@ __global__ void __launch_bounds__(kW2Threads, 1)
       if (i >= my_ptiles)  // proposal tiles: no page entries
         w2_issue_tile(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
                       smem_u32(&kv_full[i]), tile_at(i), n_ptiles, b, g, node0, P,
-                      Pages8{make_int4(-1, -1, -1, -1), make_int4(-1, -1, -1, -1)});
+                      no_pages8());
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), kW2TmemCols);
@@ -268,7 +246,7 @@ __global__ void __launch_bounds__(kW2Threads, 1)
       for (int i = kW2Stages; i < my_tiles; ++i) {
         const int st = i % kW2Stages;
         const int t = tile_at(i);
-        const Pages8 pg = w2_tile_pages(a, t, n_ptiles, b, P);  // in flight during the wait
+        const Pages8 pg = kv_tile_pages8(a, t, n_ptiles, b, P);  // in flight during the wait
         if (!mbar_wait(smem_u32(&kv_empty[st]), ((i / kW2Stages) & 1) ^ 1, a.err)) break;
         w2_issue_tile(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + st * S::kStageBytes,
                       smem_u32(&kv_full[st]), t, n_ptiles, b, g, node0, P, pg);
@@ -626,19 +604,15 @@ static cudaError_t launch_tc2(const AttnArgs& a, const AttnMaps& m, cudaStream_t
 }
 
 // Ring depth: 3 stages (inbox in the ring, peers send after every CTA of
-// the cluster has left its loop) unless PF_ATTN_W2_STAGES=2.
-static int tc2_stages() {
-  const char* e = getenv("PF_ATTN_W2_STAGES");
-  return e && atoi(e) == 2 ? 2 : 3;
+// the cluster has left its loop) unless the caller asks for 2.
+int attention_tc2_max_active_clusters(int cluster, int stages) {
+  return stages == 2 ? tc2_max_active_clusters_impl<2>(cluster)
+                     : tc2_max_active_clusters_impl<3>(cluster);
 }
 
-int attention_tc2_max_active_clusters(int cluster) {
-  return tc2_stages() == 2 ? tc2_max_active_clusters_impl<2>(cluster)
-                           : tc2_max_active_clusters_impl<3>(cluster);
-}
-
-cudaError_t launch_attention_tc2(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl) {
-  return tc2_stages() == 2 ? launch_tc2<2>(a, m, s, pdl) : launch_tc2<3>(a, m, s, pdl);
+cudaError_t launch_attention_tc2(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl,
+                                 int stages) {
+  return stages == 2 ? launch_tc2<2>(a, m, s, pdl) : launch_tc2<3>(a, m, s, pdl);
 }
 
 }  // namespace pf

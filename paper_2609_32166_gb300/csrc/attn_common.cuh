@@ -39,6 +39,33 @@ __device__ __forceinline__ int4 kv_tile_pages(const AttnArgs& a, int t, int n_pt
   return pg;
 }
 
+// Page-table entries of the eight 16-token pages of 128-token prefix tile
+// t (-1 past the prefix end, and for a contiguous cache or a proposal
+// tile), loaded together.
+struct Pages8 {
+  int4 lo, hi;
+};
+
+__device__ __forceinline__ Pages8 no_pages8() {
+  return Pages8{make_int4(-1, -1, -1, -1), make_int4(-1, -1, -1, -1)};
+}
+
+__device__ __forceinline__ Pages8 kv_tile_pages8(const AttnArgs& a, int t, int n_ptiles, int b,
+                                                 int P) {
+  Pages8 pg = no_pages8();
+  if (a.layout != PF_KV_CONTIGUOUS && t < n_ptiles) {
+    const int tok0 = t * 128;
+    const int npages = min(128 / PF_PAGE_SIZE, (P - tok0 + PF_PAGE_SIZE - 1) / PF_PAGE_SIZE);
+    const int32_t* pt = a.page_table + (size_t)b * a.pages_per_seq + tok0 / PF_PAGE_SIZE;
+    int v[8];
+#pragma unroll
+    for (int p = 0; p < 8; ++p) v[p] = p < npages ? pt[p] : -1;
+    pg.lo = make_int4(v[0], v[1], v[2], v[3]);
+    pg.hi = make_int4(v[4], v[5], v[6], v[7]);
+  }
+  return pg;
+}
+
 // TMA loads of one 64-token K/V tile into a ring stage (K then V, each two
 // 64-column halves): from the prefix cache (contiguous: one 3-D box per
 // half; paged: one 4-D box per 16-token page that holds prefix rows, pages
@@ -174,8 +201,8 @@ __device__ __forceinline__ void cluster_merge(const AttnArgs& a,
 
 // ---- balanced batch mode: the work plan.  Group q = (b * Hkv + g) *
 // rb_count + rb (sequence b, KV head g, row block rb) holds
-//   tiles_q = ceil(P_b / 64) + ceil(nn_b / 64)
-// K/V tiles if its row block has nodes (rb * nb < nn_b), else none.  With
+//   tiles_q = ceil(P_b / W) + ceil(nn_b / W)
+// K/V tiles of W tokens (the kernel's tile width) if its row block has nodes (rb * nb < nn_b), else none.  With
 // the smallest T for which sum_q ceil(tiles_q / T) <= items, group q gets
 // k_q = ceil(tiles_q / T) consecutive items (CTAs), which split its tiles
 // evenly, so no CTA holds more than T tiles while every group is served in
@@ -189,7 +216,7 @@ struct PlanItem {
   int first;  // the group's first item
 };
 
-__device__ __forceinline__ int plan_tiles(const AttnArgs& a, int q) {
+__device__ __forceinline__ int plan_tiles(const AttnArgs& a, int q, int tile_tokens) {
   const int b = q / (a.Hkv * a.rb_count);
   const int rb = q % a.rb_count;
   const int node0 = a.cu_nodes[b];
@@ -200,7 +227,7 @@ __device__ __forceinline__ int plan_tiles(const AttnArgs& a, int q) {
     return 0;
   }
   if (rb * a.nb >= nn) return 0;
-  return (P + kBN - 1) / kBN + (nn + kBN - 1) / kBN;
+  return (P + tile_tokens - 1) / tile_tokens + (nn + tile_tokens - 1) / tile_tokens;
 }
 
 // The plan's per-group table in the workspace, after the partials: (first
@@ -214,7 +241,7 @@ __device__ __forceinline__ int4* plan_table(const AttnArgs& a) {
 // Warp-collective (all 32 lanes, warp-uniform arguments): the plan entry
 // of item `item`, and in *grp that of group `group` (j = 0) if group >= 0.
 static __device__ __noinline__ PlanItem balanced_plan(const AttnArgs& a, int item, int group,
-                                                      PlanItem* grp) {
+                                                      PlanItem* grp, int tile_tokens = kBN) {
   const int lane = threadIdx.x & 31;
   const int n_groups = a.B * a.Hkv * a.rb_count;  // <= kPlanMaxGroups and <= items (host)
   constexpr int kPer = kPlanMaxGroups / 32;
@@ -224,7 +251,7 @@ static __device__ __noinline__ PlanItem balanced_plan(const AttnArgs& a, int ite
 #pragma unroll
   for (int s = 0; s < kPer; ++s) {
     const int q = lane + 32 * s;
-    t[s] = q < n_groups ? plan_tiles(a, q) : 0;
+    t[s] = q < n_groups ? plan_tiles(a, q, tile_tokens) : 0;
     U += t[s];
     n_active += t[s] > 0 ? 1 : 0;
     t_max = max(t_max, t[s]);

@@ -326,12 +326,12 @@ int lmhead_bf16_smem_bytes(int npad, int stages) {
 }
 
 // Ring depth: as many stages as about 200 KB of shared memory holds (at
-// most kMaxStages, at least 2); PF_LM_STAGES overrides it within what the
-// 227 KB per-CTA limit allows.
-int lmhead_bf16_stages(int npad) {
+// most kMaxStages, at least 2); a caller's request (`want` > 0) overrides it
+// within what the 227 KB per-CTA limit allows.
+int lmhead_bf16_stages(int npad, int want) {
   const int stage = kABytes + npad * 128;
   int ns = (200 * 1024) / stage;
-  if (const char* e = getenv("PF_LM_STAGES")) ns = atoi(e);
+  if (want > 0) ns = want;
   if (ns > kMaxStages) ns = kMaxStages;
   while (ns > 2 && lmhead_bf16_smem_bytes(npad, ns) > 232448) --ns;
   if (ns < 2) ns = 2;

@@ -2,14 +2,15 @@
 // a fixed, file-scope device array instead of a caller-provided workspace.
 //
 // Some callers cannot allocate device memory at the point where they verify
-// a proposal: code that runs while a CUDA stream is being captured into a
-// graph (cudaMalloc is not allowed there), plug-ins whose host framework
-// owns every device allocation, and latency-critical loops that must never
-// reach the allocator.  This entry point needs no workspace argument: the
-// LM head's scratch (one packed maximum per proposal row and a completion
-// ticket, kLmWorkspaceBytes = 2112 bytes, enough for PF_MAX_LM_ROWS = 256
-// rows) lives in g_lm_scratch below, which every GPU that loads this library
-// holds until the process exits.
+// a proposal: plug-ins whose host framework owns every device allocation
+// (they get tensors handed to them and have no allocator of their own), and
+// latency-critical decode loops that must never reach an allocator, which
+// can synchronise the device or fail under memory pressure.  This entry
+// point needs no workspace argument: the LM head's scratch (one packed
+// maximum per proposal row and a completion ticket, kLmWorkspaceBytes =
+// 2112 bytes, enough for PF_MAX_LM_ROWS = 256 rows) lives in g_lm_scratch
+// below, which every GPU that loads this library holds until the process
+// exits.
 #include <cuda_runtime.h>
 
 #include <mutex>
@@ -27,12 +28,15 @@ void* g_scratch_ptr[64] = {};
 
 extern "C" PF_API pf_status pf_lmhead_accept_noalloc(const pf_lm_desc* d, void* stream) {
   static const char* who = "pf_lmhead_accept_noalloc";
-  if (!d) return pf::set_error(PF_ERR_NULL, "%s: desc is NULL", who);
-  if (d->total_nodes > PF_MAX_LM_ROWS)
+  // Every argument check comes first, so that a rejected call queues
+  // nothing; the scratch's capacity first of all, with its own message.
+  if (d && d->total_nodes > PF_MAX_LM_ROWS)
     return pf::set_error(PF_ERR_SHAPE,
                          "%s: total_nodes = %d exceeds the %d rows its fixed %zu-byte scratch "
                          "holds",
                          who, d->total_nodes, PF_MAX_LM_ROWS, pf::kLmWorkspaceBytes);
+  const pf_status chk = pf::lmhead_check_desc(d, who);
+  if (chk != PF_OK) return chk;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return pf::set_error(PF_ERR_CUDA, "%s: %s", who, cudaGetErrorString(e));
@@ -43,7 +47,7 @@ extern "C" PF_API pf_status pf_lmhead_accept_noalloc(const pf_lm_desc* d, void* 
     if (!g_scratch_ptr[dev]) {
       // In host code g_lm_scratch names a host-side stand-in, not the
       // device array: its device address is looked up once per device,
-      // with that device current.
+      // with that device current, and kept for the life of the process.
       void* p = nullptr;
       e = cudaGetSymbolAddress(&p, g_lm_scratch);
       if (e != cudaSuccess || !p)

@@ -64,8 +64,16 @@ cudaError_t launch_attention_tc(const AttnArgs& a, const AttnMaps& m, cudaStream
 // tcgen05 variant with 128-token K/V tiles and P in tensor memory (bf16,
 // D = 128, a.bm = 128, cluster split-KV only); its tensor maps hold
 // 128-row cache boxes and 128-node proposal boxes.
-cudaError_t launch_attention_tc2(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl);
-int attention_tc2_max_active_clusters(int cluster);
+cudaError_t launch_attention_tc2(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl,
+                                 int stages);
+int attention_tc2_max_active_clusters(int cluster, int stages);
+// tcgen05 variant on SM pairs (2-SM MMA, M = 256 rows per pair, 128-token
+// tiles; bf16, D = 128): a.bm = 256, a.nb = 2 * floor(128 / G) nodes per
+// pair; a.splits pairs per cluster (<= 8), or a.items pairs in the balanced
+// batch mode.  Tensor maps: K boxes of 64 rows, V boxes of 128 rows (cache),
+// tree K boxes of 64 nodes, tree V boxes of 128, Q boxes of a.nb / 2 nodes.
+cudaError_t launch_attention_pair(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl);
+int attention_pair_max_active_clusters(int cluster, bool balanced);
 // Merge of the balanced batch mode's partials (launched after the tcgen05
 // kernel when a.items > 0).
 cudaError_t launch_attention_combine(const AttnArgs& a, cudaStream_t s, bool pdl);
@@ -106,10 +114,22 @@ struct LmArgs {
 cudaError_t launch_lmhead_bf16(const LmArgs& a, const CUtensorMap& w_map,
                                const CUtensorMap& h_map, cudaStream_t s, int num_sms, bool pdl);
 cudaError_t launch_lmhead_f32(const LmArgs& a, cudaStream_t s, int num_sms, bool pdl);
-int lmhead_bf16_stages(int npad);
+int lmhead_bf16_stages(int npad, int want);
 int lmhead_bf16_smem_bytes(int npad, int stages);
 
 constexpr size_t kLmWorkspaceBytes = 8 * PF_MAX_LM_ROWS + 64;
+
+// ------------------------------------------------------------ device tree prepare
+struct TreeArgs {
+  int B, T, max_nodes;
+  const int32_t* parent;
+  const int32_t* cu_nodes;
+  int32_t* depth;
+  uint64_t* mask;
+  int32_t* err;
+};
+
+cudaError_t launch_tree_prepare(const TreeArgs& a, cudaStream_t s, bool pdl);
 
 // ------------------------------------------------------------ commit
 struct CommitArgs {
@@ -205,6 +225,9 @@ cudaError_t launch_prefix_match(const PrefixArgs& a, cudaStream_t s, bool pdl);
 
 cudaError_t launch_selftest_wait(int32_t* err, unsigned long long limit_ns, int signal,
                                  int32_t* waited_ok, cudaStream_t s);
+
+// pf_lmhead_accept's argument checks that do not involve the workspace.
+pf_status lmhead_check_desc(const pf_lm_desc* d, const char* who);
 
 // Record the message pf_last_error() returns on this thread; returns s.
 pf_status set_error(pf_status s, const char* fmt, ...);

@@ -48,13 +48,25 @@ class VerifyStep:
     """One workload's device state.  ``layers`` may restrict the layer count
     (parity tests use a few layers of a full-size workload).  ``balanced``
     gives the attention calls a workspace, with which a batch of several
-    sequences is dealt out to the SMs in proportion to their lengths."""
+    sequences is dealt out to the SMs in proportion to their lengths.
+
+    ``fill="host"`` (the default) uploads the seeded host generator's values,
+    which the oracle also receives; ``fill="device"`` draws the bulk tensors
+    (queries, proposal K/V, caches, hidden states, LM weight) with torch's
+    seeded device generator instead -- the same shapes and distributions
+    (N(0, 1), weight N(0, 0.02), bf16), minutes faster for the 32K-token
+    cache, for measurements that are not compared with the oracle.
+    ``weight_dev`` shares an LM-head weight already on the device."""
 
     def __init__(self, w: I.Workload, batch: I.Batch, tokens: np.ndarray, layers: int = None,
                  device: str = "cuda", weight: np.ndarray = None, hidden: np.ndarray = None,
-                 balanced: bool = True):
+                 balanced: bool = True, attn_launch: dict = None, fill: str = "host",
+                 weight_dev: torch.Tensor = None):
         self.w, self.batch = w, batch
         self.balanced = balanced
+        # pf_attn_desc launch fields (kernel, splits, rows_per_cta, stages):
+        # empty = the library's automatic choice
+        self.attn_launch = dict(attn_launch or {})
         self.L = layers if layers is not None else w.layers
         self.device = device
         td = _torch_dtype(w.dtype)
@@ -82,7 +94,15 @@ class VerifyStep:
         self.tree_v = torch.empty_like(self.tree_k)
         self.cache_k = torch.zeros((self.L,) + shp, dtype=td, device=device)
         self.cache_v = torch.zeros_like(self.cache_k)
-        for l in range(self.L):
+        gen = None
+        if fill == "device":
+            gen = torch.Generator(device=device)
+            gen.manual_seed(int(batch.seed) * 7919 + 17)
+            for t in (self.q, self.tree_k, self.tree_v, self.cache_k, self.cache_v):
+                t.normal_(0.0, 1.0, generator=gen)
+        elif fill != "host":
+            raise ValueError(f"fill must be 'host' or 'device', not {fill!r}")
+        for l in (range(self.L) if fill == "host" else ()):
             self.q[l] = _dev(I.layer_q(w, batch, l), w.dtype, device)
             tk, tv = I.layer_tree_kv(w, batch, l)
             self.tree_k[l] = _dev(tk, w.dtype, device)
@@ -96,12 +116,21 @@ class VerifyStep:
             self.cache_k[l] = _dev(ck, w.dtype, device)
             self.cache_v[l] = _dev(cv, w.dtype, device)
         self.attn_out = torch.zeros_like(self.q)
-        if hidden is None:
-            hidden = I.hidden_states(w, batch)
-        if weight is None:
-            weight = I.lm_weight(w, batch.seed)
-        self.hidden = _dev(hidden, w.dtype, device)
-        self.weight = _dev(weight, w.dtype, device)
+        if fill == "device" and hidden is None:
+            self.hidden = torch.empty((T, w.hidden), dtype=td, device=device)
+            self.hidden.normal_(0.0, 1.0, generator=gen)
+        else:
+            self.hidden = _dev(I.hidden_states(w, batch) if hidden is None else hidden, w.dtype,
+                               device)
+        if weight_dev is not None:
+            assert tuple(weight_dev.shape) == (w.vocab, w.hidden) and weight_dev.dtype == td
+            self.weight = weight_dev
+        elif fill == "device" and weight is None:
+            self.weight = torch.empty((w.vocab, w.hidden), dtype=td, device=device)
+            self.weight.normal_(0.0, 0.02, generator=gen)
+        else:
+            self.weight = _dev(I.lm_weight(w, batch.seed) if weight is None else weight, w.dtype,
+                               device)
 
         i32 = dict(dtype=torch.int32, device=device)
         self.argmax = torch.full((T,), -1, **i32)
@@ -117,8 +146,10 @@ class VerifyStep:
         # A step's inputs and outputs each live in one contiguous arena (the
         # tensors above become views of it), so that a host round trip is
         # one copy each way.
+        # (the ancestor bitmaps are derived on the device from the parent
+        # array by pf_tree_prepare_device, so they are not among the inputs)
         self.in_arena = self._arena(("q", "tree_k", "tree_v", "hidden", "tokens", "parent",
-                                     "mask", "cu_nodes", "prefix_len"), device)
+                                     "cu_nodes", "prefix_len"), device)
         self.out_arena = self._arena(("accept_len", "out_tokens", "new_len"), device)
         self._build_descs()
 
@@ -175,6 +206,8 @@ class VerifyStep:
             # after the last layer: every layer but the first may request its
             # cache tiles while the previous layer is still finishing.
             d.flags = pb.PF_ATTN_EARLY_PREFETCH if l > 0 else 0
+            for k, v in self.attn_launch.items():
+                setattr(d, k, int(v))
             self.attn_descs.append(d)
         # one attention workspace serves every layer (calls run in stream order)
         self.attn_ws_bytes = (pb.pf_verify_attention_workspace_size(self.attn_descs[0])
@@ -225,8 +258,19 @@ class VerifyStep:
     def commit(self, stream=None):
         pb.pf_kv_commit(self.commit_desc, self._stream(stream))
 
-    def step(self, stream=None):
+    def tree_prepare(self, stream=None):
+        """Ancestor bitmaps of this step's trees, on the device, from the
+        parent array (pf_tree_prepare_device)."""
+        pb.pf_tree_prepare_device(self.parent.data_ptr(), self.cu_nodes.data_ptr(), self.w.batch,
+                                  self.T, self.max_nodes, 0, self.mask.data_ptr(),
+                                  self.err.data_ptr(), self._stream(stream))
+
+    def step(self, stream=None, tree_prepare: bool = False):
+        """One verify step: (optionally the device tree bitmaps,) L attention
+        calls, the LM head with acceptance, the commit."""
         s = self._stream(stream)
+        if tree_prepare:
+            self.tree_prepare(s)
         for l in range(self.L):
             pb.pf_verify_attention(self.attn_descs[l], s)
         pb.pf_lmhead_accept(self.lm_desc, self.workspace.data_ptr(), self.ws_bytes, s)

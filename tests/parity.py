@@ -33,7 +33,7 @@ class Case:
     """A generated workload, the oracle's greedy predictions and a device step."""
 
     def __init__(self, w: I.Workload, seed: int = 0, layers: int = None, batch: I.Batch = None,
-                 balanced: bool = True):
+                 balanced: bool = True, attn_launch: dict = None):
         self.w = w
         self.batch = batch if batch is not None else I.make_batch(w, seed)
         self.L = layers if layers is not None else w.layers
@@ -44,7 +44,8 @@ class Case:
         del lg
         self.tokens = I.plant_tokens(self.batch, self.o_argmax)
         self.vs = VerifyStep(w, self.batch, self.tokens, layers=self.L,
-                             weight=self.weight, hidden=self.hidden, balanced=balanced)
+                             weight=self.weight, hidden=self.hidden, balanced=balanced,
+                             attn_launch=attn_launch)
 
     # --------------------------------------------------------------- attention
     def oracle_attention(self, layer: int, seq: int, nodes=None) -> np.ndarray:
@@ -62,6 +63,18 @@ class Case:
         sel = range(c1 - c0) if nodes is None else nodes
         err = max(float(np.abs(got[n] - ref[n]).max()) for n in sel)
         assert np.isfinite(got[list(sel)]).all()
+        assert err <= ATTN_TOL[self.w.dtype], (layer, seq, err)
+        return err
+
+    def compare_attention(self, layer: int, seq: int, ref: dict) -> float:
+        """Max error against precomputed oracle rows {node: [Hq, D]}."""
+        c0 = int(self.batch.cu_nodes[seq])
+        got = self.vs.attn_out[layer].float().cpu().numpy().astype(np.float64)
+        err = 0.0
+        for n, r in ref.items():
+            g = got[c0 + n]
+            assert np.isfinite(g).all(), (layer, seq, n)
+            err = max(err, float(np.abs(g - r).max()))
         assert err <= ATTN_TOL[self.w.dtype], (layer, seq, err)
         return err
 

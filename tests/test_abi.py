@@ -130,6 +130,21 @@ def _attn_desc(**kw):
     (dict(cache_layout=1, cache_page_table=0x10000, cache_num_pages=4, cache_pages_per_seq=1,
           max_prefix_len=17), pb.PF_ERR_CAPACITY),
     (dict(q=0x10008), pb.PF_ERR_ALIGN),
+    # launch fields
+    (dict(kernel=5), pb.PF_ERR_SHAPE),
+    (dict(kernel=-1), pb.PF_ERR_SHAPE),
+    (dict(kernel=pb.PF_ATTN_KERNEL_PAIR, splits=9), pb.PF_ERR_SHAPE),
+    (dict(kernel=pb.PF_ATTN_KERNEL_TC64, splits=17), pb.PF_ERR_SHAPE),
+    (dict(splits=-1), pb.PF_ERR_SHAPE),
+    (dict(kernel=pb.PF_ATTN_KERNEL_PAIR, head_dim=64), pb.PF_ERR_SHAPE),
+    (dict(kernel=pb.PF_ATTN_KERNEL_TC128, rows_per_cta=128), pb.PF_ERR_SHAPE),
+    (dict(rows_per_cta=192), pb.PF_ERR_SHAPE),
+    (dict(rows_per_cta=128, n_q_heads=258, n_kv_heads=2), pb.PF_ERR_SHAPE),
+    (dict(kernel=pb.PF_ATTN_KERNEL_TC64, stages=2), pb.PF_ERR_SHAPE),
+    (dict(kernel=pb.PF_ATTN_KERNEL_TC128, stages=4), pb.PF_ERR_SHAPE),
+    (dict(dtype=pb.PF_F32, kernel=pb.PF_ATTN_KERNEL_MMA), pb.PF_ERR_DTYPE),
+    (dict(dtype=pb.PF_F32, splits=2), pb.PF_ERR_DTYPE),
+    (dict(flags=8), pb.PF_ERR_SHAPE),
 ])
 def test_attention_rejects_bad_arguments(kw, status):
     with pytest.raises(pb.PfError) as e:
@@ -301,3 +316,32 @@ def test_prefix_match_rejects_bad_arguments():
         with pytest.raises(pb.PfError) as e:
             pb.pf_prefix_match(desc(**kw), 0)
         assert e.value.status == status
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(parent=0), pb.PF_ERR_NULL),
+    (dict(cu_nodes=0), pb.PF_ERR_NULL),
+    (dict(mask_out=0), pb.PF_ERR_NULL),
+    (dict(batch=0), pb.PF_ERR_SHAPE),
+    (dict(total_nodes=0), pb.PF_ERR_SHAPE),
+    (dict(max_nodes=0), pb.PF_ERR_SHAPE),
+    (dict(max_nodes=129), pb.PF_ERR_SHAPE),
+    (dict(mask_out=0x10008), pb.PF_ERR_ALIGN),
+])
+def test_tree_prepare_device_rejects_bad_arguments(kw, status):
+    """Host checks of the device tree call: they return before any launch
+    (here, with no GPU, before the library would notice there is none)."""
+    a = dict(parent=0x10000, cu_nodes=0x10000, batch=2, total_nodes=9, max_nodes=8,
+             depth_out=0, mask_out=0x10000)
+    a.update(kw)
+    with pytest.raises(pb.PfError) as e:
+        pb.pf_tree_prepare_device(**a)
+    assert e.value.status == status
+
+
+def test_launch_fields_reach_the_library():
+    """The launch fields sit after the workspace in pf_attn_desc and the
+    stage request at the end of pf_lm_desc, as the header declares them."""
+    names = [f[0] for f in pb.pf_attn_desc._fields_]
+    assert names[-4:] == ["kernel", "splits", "rows_per_cta", "stages"]
+    assert [f[0] for f in pb.pf_lm_desc._fields_][-1] == "stages"

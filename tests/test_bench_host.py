@@ -84,6 +84,37 @@ def test_traffic_only_for_matching_sources_and_workload(tmp_path):
 
 def test_reference_steps_stop_at_the_wall_budget():
     b = _bench()
-    spec = dict(workload="tiny-f32-chain8", seed=0, layers_sample=1, steps=50, warmup=0)
+    spec = dict(workload="tiny-f32-chain8", seed=0, mode="whole", steps=50, warmup=0)
     assert b.cpu_worker(dict(spec, wall_budget_s=0.0))["steps"] == 1
-    assert b.cpu_worker(dict(spec, steps=3, wall_budget_s=60.0))["steps"] == 3
+    r = b.cpu_worker(dict(spec, steps=3, wall_budget_s=60.0))
+    assert r["steps"] == 3
+    # whole steps: nothing is projected
+    assert r["layers_timed"] == 1 and r["step_s"] == pytest.approx(r["measured_s"])
+
+
+def test_combined_step_roofline_takes_each_part_at_its_own_bound():
+    b = _bench()
+    w = inputs.WORKLOADS["7b-bf16-32k-tree128"]
+    batch = inputs.make_batch(w, 0)
+    attn_b, lm_b, commit_b = 69.2e6, 1.09e9, 2.0e6
+    r = b.combined_step_roofline(w, batch, attn_b, lm_b, commit_b, 2e-3, PEAKS)
+    flops = b.attention_flops(w, batch)
+    # the 32K tree's attention is tensor-bound (about 870 FLOP/B, ridge 250)
+    attn = max(attn_b / 6000e9, flops / 1500e12) * w.layers
+    assert attn == pytest.approx(flops / 1500e12 * w.layers)
+    lm = max(lm_b / 6000e9, b.lmhead_flops(w, batch) / 1500e12)
+    ideal = attn + lm + commit_b / 6000e9
+    assert r["ideal_us"] == pytest.approx(ideal * 1e6)
+    assert r["frac"] == pytest.approx(ideal / 2e-3)
+    hbm = (attn_b * w.layers + lm_b + commit_b) / 6000e9
+    assert r["hbm_only_frac"] == pytest.approx(hbm / 2e-3)
+    assert r["ideal_us"] > r["hbm_only_ideal_us"]
+
+
+def test_cpu_baseline_mode_is_whole_steps_only_where_they_are_cheap():
+    b = _bench()
+    W = inputs.WORKLOADS
+    assert b.cpu_mode(W["tiny-f32-chain8"]) == "whole"
+    assert b.cpu_mode(W["2b-bf16-chain16"]) == "whole"
+    for name in ("7b-bf16-tree64", "7b-bf16-batch8-paged", "7b-bf16-32k-tree128"):
+        assert b.cpu_mode(W[name]) == "layer"

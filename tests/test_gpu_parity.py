@@ -7,8 +7,14 @@ import numpy as np
 import pytest
 import torch
 
+from paper_2609_32166_gb300 import binding as pb
 from paper_2609_32166_gb300 import inputs as I
 from tests.parity import Case
+
+MMA = dict(kernel=pb.PF_ATTN_KERNEL_MMA)
+TC64 = dict(kernel=pb.PF_ATTN_KERNEL_TC64)
+TC128 = dict(kernel=pb.PF_ATTN_KERNEL_TC128)
+PAIR = dict(kernel=pb.PF_ATTN_KERNEL_PAIR)
 
 pytestmark = pytest.mark.gpu
 
@@ -90,12 +96,90 @@ def test_edge_cases(name):
     c.check_commit(res)
 
 
+# ---------------------------------------------------------------------------
+# the SM-pair kernel (2-SM MMA, each CTA holding half of every K/V tile)
+# ---------------------------------------------------------------------------
+EDGE_PAIR = {k: EDGE[k] for k in ("root-only", "empty-prefix", "65-nodes", "g16-tiny-vocab",
+                                  "256-rows-paged", "two-blocks-one-tile")}
+
+
+@pytest.mark.parametrize("balanced", [False, True])
+@pytest.mark.parametrize("name", sorted(EDGE_PAIR))
+def test_pair_kernel_edges(name, balanced):
+    """Root only (the odd CTA of the pair has no rows), no prefix (one tile),
+    65 nodes with a one-row last prefix tile, G = 16 (the odd CTA holds one
+    node), 128-node paged trees, one tile for 192 rows; cluster mode and the
+    balanced batch mode (the latter only changes batches)."""
+    c = Case(EDGE_PAIR[name], seed=5, balanced=balanced, attn_launch=PAIR)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for l in range(c.L):
+        for s in range(c.w.batch):
+            c.check_attention(l, s)
+    c.check_lmhead(res)
+    c.check_commit(res)
+
+
+@pytest.mark.parametrize("splits", [1, 2, 3, 8])
+@pytest.mark.parametrize("name", ["7b-tree64-small", "7b-32k-tree128-small",
+                                  "7b-batch8-paged-small"])
+def test_pair_kernel_splits(name, splits):
+    """Pairs per cluster from 1 to 8 (cluster widths 2 to 16) on the three 7B
+    shapes, paged batch included (cluster mode: no workspace), every node."""
+    c = Case(SMALL[name], seed=14, balanced=False, attn_launch=dict(PAIR, splits=splits))
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for s in range(c.w.batch):
+        c.check_attention(0, s)
+
+
+@pytest.mark.parametrize("launch", ["tc64", "pair"])
+def test_splits_without_tiles(launch):
+    """A split count above a sequence's tile count: with 8 splits, a
+    sequence whose prefix is 20 rows has 2 tiles, so 6 splits (tc64) or 6
+    pairs (pair kernel) of its cluster get no tile and contribute zero
+    partials with lse = -inf to the merge."""
+    w = I.scaled(W["7b-bf16-batch8-paged"], layers=1, batch=3, prefix=(20, 1500), nodes=20,
+                 max_depth=6, vocab=600, hidden=128)
+    rng = np.random.default_rng(21)
+    parents = [I.random_tree(20, 3, rng) for _ in range(3)]
+    prefix = np.array([20, 1500, 700], dtype=np.int32)
+    ends = np.array([5, 11, 19], dtype=np.int32)
+    max_seq = int(prefix.max()) + 20
+    per_seq = -(-max_seq // I.PAGE_SIZE)
+    pt = rng.permutation(per_seq * 3).astype(np.int32).reshape(3, per_seq)
+    b = I.Batch(w, 3, parents, prefix, ends, pt, per_seq * 3, max_seq)
+    tile = 64 if launch == "tc64" else 128
+    n_tiles = -(-int(prefix[0]) // tile) + 1
+    assert n_tiles < 8   # the case under test occurs
+    launch_fields = dict(TC64, rows_per_cta=128) if launch == "tc64" else dict(PAIR)
+    c = Case(w, batch=b, balanced=False, attn_launch=dict(launch_fields, splits=8))
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for s in range(3):
+        c.check_attention(0, s)
+    c.check_lmhead(res)
+    c.check_commit(res)
+
+
+def test_two_block_kernel_one_tile():
+    """192 rows of one KV head in one two-block CTA of the 64-token kernel,
+    one KV tile (no split): that kernel's direct epilogue."""
+    c = Case(EDGE["two-blocks-one-tile"], seed=5, attn_launch=dict(TC64, rows_per_cta=256))
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    c.check_attention(0, 0)
+
+
 @pytest.mark.parametrize("name", ["7b-tree64-small", "7b-batch8-paged-small"])
-def test_mma_sync_kernel(name, monkeypatch):
-    """The mma.sync attention kernel (selected with PF_ATTN_IMPL=mma) stays
-    correct at D = 128, where the tcgen05 kernel is the default."""
-    monkeypatch.setenv("PF_ATTN_IMPL", "mma")
-    c = Case(SMALL[name], seed=6)
+def test_mma_sync_kernel(name):
+    """The mma.sync attention kernel (kernel = PF_ATTN_KERNEL_MMA) stays
+    correct at D = 128, where the tcgen05 kernels are the default."""
+    c = Case(SMALL[name], seed=6, attn_launch=MMA)
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0
@@ -104,11 +188,10 @@ def test_mma_sync_kernel(name, monkeypatch):
 
 
 @pytest.mark.parametrize("name", ["2b-chain16-small", "7b-tree64-small", "7b-32k-tree128-small"])
-def test_64_token_tile_kernel(name, monkeypatch):
-    """The tcgen05 kernel with 64-token tiles (PF_ATTN_IMPL=tc64), which the
-    balanced batch mode and 256-row CTAs use, on 128-row CTAs too."""
-    monkeypatch.setenv("PF_ATTN_IMPL", "tc64")
-    c = Case(SMALL[name], seed=7)
+def test_64_token_tile_kernel(name):
+    """The tcgen05 kernel with 64-token tiles (PF_ATTN_KERNEL_TC64), its
+    balanced batch mode and 256-row CTAs, on 128-row CTAs too."""
+    c = Case(SMALL[name], seed=7, attn_launch=dict(TC64, rows_per_cta=128))
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0
@@ -116,15 +199,13 @@ def test_64_token_tile_kernel(name, monkeypatch):
         c.check_attention(l, 0)
 
 
-@pytest.mark.parametrize("stages", ["2", "3"])
+@pytest.mark.parametrize("stages", [2, 3])
 @pytest.mark.parametrize("name", ["2b-chain16-small", "7b-tree64-small", "7b-32k-tree128-small"])
-def test_128_token_tile_kernel(name, stages, monkeypatch):
+def test_128_token_tile_kernel(name, stages):
     """The tcgen05 kernel with 128-token tiles and P in tensor memory
-    (PF_ATTN_IMPL=tc128) also where a CTA holds few tiles, with both ring
+    (PF_ATTN_KERNEL_TC128) also where a CTA holds few tiles, with both ring
     depths (3 stages: the merge inbox in the idle ring)."""
-    monkeypatch.setenv("PF_ATTN_IMPL", "tc128")
-    monkeypatch.setenv("PF_ATTN_W2_STAGES", stages)
-    c = Case(SMALL[name], seed=9)
+    c = Case(SMALL[name], seed=9, attn_launch=dict(TC128, stages=stages))
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0
@@ -137,9 +218,8 @@ EDGE_128 = {k: EDGE[k] for k in ("root-only", "empty-prefix", "65-nodes", "g16-t
 
 
 @pytest.mark.parametrize("name", sorted(EDGE_128))
-def test_128_token_tile_kernel_edges(name, monkeypatch):
-    monkeypatch.setenv("PF_ATTN_IMPL", "tc128")
-    c = Case(EDGE_128[name], seed=5)
+def test_128_token_tile_kernel_edges(name):
+    c = Case(EDGE_128[name], seed=5, attn_launch=TC128)
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0
@@ -148,14 +228,13 @@ def test_128_token_tile_kernel_edges(name, monkeypatch):
             c.check_attention(l, s)
 
 
-@pytest.mark.parametrize("stages", ["2", "3"])
-def test_128_token_tile_kernel_paged(stages, monkeypatch):
+@pytest.mark.parametrize("stages", [2, 3])
+def test_128_token_tile_kernel_paged(stages):
     """Paged cache (eight 16-token pages per 128-token tile, random page
     order, ragged last pages), two sequences with 128-node trees, on the
     128-token kernel (no workspace, so no balanced batch mode)."""
-    monkeypatch.setenv("PF_ATTN_IMPL", "tc128")
-    monkeypatch.setenv("PF_ATTN_W2_STAGES", stages)
-    c = Case(EDGE["256-rows-paged"], seed=10, balanced=False)
+    c = Case(EDGE["256-rows-paged"], seed=10, balanced=False,
+             attn_launch=dict(TC128, stages=stages))
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0
@@ -166,11 +245,10 @@ def test_128_token_tile_kernel_paged(stages, monkeypatch):
 
 
 @pytest.mark.parametrize("name", ["7b-tree64-small", "7b-32k-tree128-small"])
-def test_two_block_kernel_on_many_rows(name, monkeypatch):
-    """Two 128-row blocks per CTA (PF_ATTN_BM=256) where a KV head has more
-    than 256 rows, so several two-block CTAs share a head."""
-    monkeypatch.setenv("PF_ATTN_BM", "256")
-    c = Case(SMALL[name], seed=8)
+def test_two_block_kernel_on_many_rows(name):
+    """Two 128-row blocks per CTA (64-token kernel, rows_per_cta = 256) where
+    a KV head has more than 256 rows, so several two-block CTAs share a head."""
+    c = Case(SMALL[name], seed=8, attn_launch=dict(TC64, rows_per_cta=256))
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0
@@ -178,13 +256,16 @@ def test_two_block_kernel_on_many_rows(name, monkeypatch):
         c.check_attention(0, s)
 
 
+@pytest.mark.parametrize("kernel", ["auto", "pair"])
 @pytest.mark.parametrize("balanced", [False, True])
-def test_batch_work_split(balanced):
+def test_batch_work_split(balanced, kernel):
     """Eight sequences with prefixes from 100 to 700 rows, with an attention
-    workspace (tiles dealt out to the SMs in proportion to each sequence's
-    length, partials merged by a second kernel) and without one (every
-    sequence and KV head gets the same cluster)."""
-    c = Case(SMALL["7b-batch8-paged-small"], seed=11, balanced=balanced)
+    workspace (tiles dealt out to the SMs -- or SM pairs -- in proportion to
+    each sequence's length, partials merged by a second kernel) and without
+    one (every sequence and KV head gets the same cluster); on the automatic
+    choice and on the SM-pair kernel."""
+    c = Case(SMALL["7b-batch8-paged-small"], seed=11, balanced=balanced,
+             attn_launch=PAIR if kernel == "pair" else None)
     assert (c.vs.attn_ws is not None) == balanced
     assert c.vs.launches_per_step() == c.L * (2 if balanced else 1) + 2
     c.vs.step()
@@ -237,12 +318,11 @@ def test_batch_beyond_balanced_groups():
     c.check_commit(res)
 
 
-@pytest.mark.parametrize("impl", ["default", "tc128"])
-def test_mixed_tree_sizes(impl, monkeypatch):
+@pytest.mark.parametrize("impl", ["default", "tc128", "pair-clusters"])
+def test_mixed_tree_sizes(impl):
     """Sequences of 1, 17 and 128 nodes in one batch (variable cu_nodes), on
-    the default path (balanced batch mode) and on the 128-token kernel."""
-    if impl == "tc128":
-        monkeypatch.setenv("PF_ATTN_IMPL", "tc128")
+    the default path (balanced batch mode on SM pairs), on the 128-token
+    kernel and on SM pairs in cluster mode."""
     w = I.scaled(W["7b-bf16-batch8-paged"], layers=1, batch=3, prefix=(50, 400), nodes=128,
                  vocab=640, hidden=128)
     rng = np.random.default_rng(9)
@@ -253,7 +333,8 @@ def test_mixed_tree_sizes(impl, monkeypatch):
     per_seq = -(-max_seq // I.PAGE_SIZE)
     pt = rng.permutation(per_seq * 3).astype(np.int32).reshape(3, per_seq)
     b = I.Batch(w, 7, parents, prefix, ends, pt, per_seq * 3, max_seq)
-    c = Case(w, batch=b, balanced=impl == "default")
+    launch = {"default": None, "tc128": TC128, "pair-clusters": PAIR}[impl]
+    c = Case(w, batch=b, balanced=impl == "default", attn_launch=launch)
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0
@@ -293,7 +374,7 @@ def test_commit_capacity_flag_without_fault():
 
 
 # ---------------------------------------------------------------------------
-# full workload sizes (sampled checks)
+# full workload sizes, in the launch configuration bench.py times
 # ---------------------------------------------------------------------------
 FULL = {
     "2b-bf16-chain16": 28,
@@ -301,21 +382,48 @@ FULL = {
     "7b-bf16-batch8-paged": 1,
     "7b-bf16-32k-tree128": 1,
 }
+FULL_CASES = [("2b-bf16-chain16", 0), ("7b-bf16-tree64", 0), ("7b-bf16-tree64", 1),
+              ("7b-bf16-batch8-paged", 0), ("7b-bf16-32k-tree128", 0),
+              ("7b-bf16-32k-tree128", 1)]
 
 
-@pytest.mark.parametrize("name", sorted(FULL))
-def test_full_size_sampled(name):
+@pytest.fixture(scope="module")
+def oracle_pool():
+    from tests.oracle_pool import make_pool
+    pool = make_pool()
+    yield pool
+    pool.shutdown()
+
+
+@pytest.mark.parametrize("name,seed", FULL_CASES)
+def test_full_size(name, seed, oracle_pool):
+    """The workloads' real shapes with the library's automatic launch choice
+    (the balanced batch mode for the batch): every node and head of layer 0
+    of every sequence against the oracle (for the 32K tree's second seed,
+    four sampled nodes), sampled nodes of the middle and last layer, then the
+    LM head, acceptance and commit."""
+    import time
+    from tests.oracle_pool import oracle_attention_nodes
     w = W[name]
-    c = Case(w, seed=0, layers=FULL[name])
+    t0 = time.time()
+    c = Case(w, seed=seed, layers=FULL[name])
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0
+    every = not (name == "7b-bf16-32k-tree128" and seed == 1)
+    errs = []
+    for s in range(w.batch):
+        n = int(c.batch.cu_nodes[s + 1] - c.batch.cu_nodes[s])
+        nodes = range(n) if every else sorted({0, n - 1, n // 2, int(c.batch.forced_end[s])})
+        ref = oracle_attention_nodes(oracle_pool, w, seed, 0, s, nodes)
+        errs.append(c.compare_attention(0, s, ref))
     layers = sorted({0, c.L // 2, c.L - 1})
-    for l in layers:
+    for l in layers[1:]:
         for s in sorted({0, w.batch - 1}):
             n = int(c.batch.cu_nodes[s + 1] - c.batch.cu_nodes[s])
-            nodes = sorted({0, n - 1, n // 2, int(c.batch.forced_end[s])})
-            c.check_attention(l, s, nodes=nodes)
+            c.check_attention(l, s, nodes=sorted({0, n - 1, n // 2, int(c.batch.forced_end[s])}))
     flagged = c.check_lmhead(res)
-    print(f"{name}: flagged near-tie nodes {flagged}/{c.batch.total_nodes}")
     c.check_commit(res, layers=layers)
+    print(f"{name} seed {seed}: layer-0 max error {max(errs):.2e} over "
+          f"{'every node' if every else 'sampled nodes'}, flagged near-tie nodes "
+          f"{flagged}/{c.batch.total_nodes}, {time.time() - t0:.0f} s")

@@ -184,7 +184,7 @@ typedef struct pf_attn_desc {
    * result beyond floating-point rounding order. */
   int32_t kernel;              /* pf_attn_kernel                             */
   int32_t splits;              /* K/V splits per row block (cluster width):
-                                  1..16; 1..8 for PF_ATTN_KERNEL_PAIR        */
+                                  1..16; 0 for PF_ATTN_KERNEL_PAIR           */
   int32_t rows_per_cta;        /* PF_ATTN_KERNEL_TC64: 128 or 256            */
   int32_t stages;              /* PF_ATTN_KERNEL_TC128 ring depth: 2 or 3    */
 } pf_attn_desc;
@@ -196,14 +196,24 @@ typedef struct pf_attn_desc {
  *   TC128  tcgen05, 128-token tiles with P kept in tensor memory, 128 rows
  *          per CTA (no balanced batch mode: a workspace is ignored)
  *   PAIR   tcgen05 on pairs of SMs (one 2-SM MMA of 256 query rows per
- *          128-token tile, each SM loading half of every K/V tile)
- * TC64, TC128 and PAIR need bf16 and D = 128. */
+ *          128-token tile, each SM loading half of every K/V tile); all
+ *          sequences' tiles are laid end to end and cut into one equal range
+ *          per SM pair, pieces of a sequence merged by a second kernel; needs
+ *          the workspace
+ *   STREAM TC128's pipeline, one CTA per SM, with the same continuous split
+ *          (one equal range of all sequences' tiles per SM); needs the
+ *          workspace
+ * TC64, TC128, PAIR and STREAM need bf16 and D = 128.  The automatic choice
+ * is TC128 (128-row CTAs in clusters that split each row block's tiles)
+ * where a CTA holds several 128-token tiles, TC64 otherwise, MMA for other
+ * head sizes; it takes no workspace. */
 typedef enum pf_attn_kernel {
   PF_ATTN_KERNEL_AUTO = 0,
   PF_ATTN_KERNEL_MMA = 1,
   PF_ATTN_KERNEL_TC64 = 2,
   PF_ATTN_KERNEL_TC128 = 3,
-  PF_ATTN_KERNEL_PAIR = 4
+  PF_ATTN_KERNEL_PAIR = 4,
+  PF_ATTN_KERNEL_STREAM = 5
 } pf_attn_kernel;
 
 /* PF_ATTN_EARLY_PREFETCH: the prefix cache, page_table, cu_nodes, prefix_len
@@ -219,17 +229,21 @@ typedef enum pf_attn_kernel {
  * then starts only after the preceding kernel in the stream has finished). */
 #define PF_ATTN_NO_PDL 2
 
-/* Workspace (optional; batches of B > 1 sequences, bf16, head_dim 128):
- * with workspace != NULL and at least pf_verify_attention_workspace_size(d)
- * bytes (16-byte aligned), a batch's KV tiles are dealt out to one CTA per
- * SM in proportion to each sequence's length (prefix plus proposal tiles),
- * so long and short prefixes finish together; sequences spread over several
- * CTAs are merged by a second kernel in the same stream (the call then
- * launches two kernels).  Without it every (sequence, KV head) gets the
- * same number of CTAs.  The contents need no initialisation and are
- * scratch between calls; one workspace serves calls in stream order but
- * not concurrent calls.  A workspace that is too small is an error
- * (PF_ERR_WORKSPACE); for shapes that do not use it, it is ignored. */
+/* Workspace (bf16, head_dim 128; needed by PF_ATTN_KERNEL_PAIR and
+ * PF_ATTN_KERNEL_STREAM, optional for PF_ATTN_KERNEL_TC64): with workspace
+ * != NULL and at least pf_verify_attention_workspace_size(d) bytes (16-byte
+ * aligned), the KV tiles are dealt out in proportion to each sequence's
+ * length (prefix plus proposal tiles) -- on TC64 to one CTA per SM for
+ * batches of B > 1 sequences, on STREAM and PAIR in one equal range of all
+ * sequences' tiles per SM (pair) for any B -- so long and short prefixes
+ * finish together; sequences spread over several CTAs are merged by a
+ * second kernel in the same stream (the call then launches two kernels).
+ * Without it every (sequence, KV head) gets the same number of CTAs.  The
+ * size query returns 0 where the chosen kernel takes none (the automatic
+ * choice).  The contents need no initialisation and are scratch between
+ * calls; one workspace serves calls in stream order but not concurrent
+ * calls.  A workspace that is too small is an error (PF_ERR_WORKSPACE);
+ * for shapes that do not use it, it is ignored. */
 PF_API size_t pf_verify_attention_workspace_size(const pf_attn_desc* d);
 
 PF_API pf_status pf_verify_attention(const pf_attn_desc* d, void* stream);

@@ -29,7 +29,7 @@ PF_DEVERR_TIMEOUT, PF_DEVERR_CAPACITY, PF_DEVERR_BOUNDS, PF_DEVERR_TREE = 1, 2, 
 PF_ATTN_EARLY_PREFETCH, PF_ATTN_NO_PDL = 1, 2
 PF_LM_EARLY_WEIGHT, PF_LM_NO_PDL = 1, 2
 (PF_ATTN_KERNEL_AUTO, PF_ATTN_KERNEL_MMA, PF_ATTN_KERNEL_TC64, PF_ATTN_KERNEL_TC128,
- PF_ATTN_KERNEL_PAIR) = 0, 1, 2, 3, 4
+ PF_ATTN_KERNEL_PAIR, PF_ATTN_KERNEL_STREAM) = 0, 1, 2, 3, 4, 5
 
 STATUS_NAMES = {0: "PF_OK", 1: "PF_ERR_NULL", 2: "PF_ERR_SHAPE", 3: "PF_ERR_DTYPE",
                 4: "PF_ERR_TREE", 5: "PF_ERR_CAPACITY", 6: "PF_ERR_ALIGN", 7: "PF_ERR_CUDA",

@@ -108,7 +108,7 @@ pf_status check_cache_view(const pf_kv_view& c, int need_rows, const char* who) 
 // follows from the shape, unless the descriptor's launch fields ask for
 // something specific; nothing is read from the environment.
 // ---------------------------------------------------------------------------
-enum class AttnKernel { F32, MMA, TC64, TC128, PAIR };
+enum class AttnKernel { F32, MMA, TC64, TC128, PAIR, STREAM };
 
 // kernel index 0..2: mma.sync BM 32/64/128
 int max_cluster_for(int kernel, int D, int want) {
@@ -133,9 +133,9 @@ int max_cluster_for(int kernel, int D, int want) {
 
 // How many clusters of `cluster` CTAs fit on the device at once, per kernel
 // variant (memoised per device): 0 tc64 128 rows, 1 tc64 256 rows, 2 tc128
-// 3 stages, 3 tc128 2 stages, 4 pair.
+// 3 stages, 3 tc128 2 stages.
 int max_active_clusters(int variant, int cluster) {
-  static std::atomic<int> cache[64][5][17];
+  static std::atomic<int> cache[64][4][17];
   int dev = 0;
   cudaGetDevice(&dev);
   std::atomic<int>& slot = cache[dev & 63][variant][cluster];
@@ -146,8 +146,7 @@ int max_active_clusters(int variant, int cluster) {
       case 0: n = pf::attention_tc_max_active_clusters(cluster, 128); break;
       case 1: n = pf::attention_tc_max_active_clusters(cluster, 256); break;
       case 2: n = pf::attention_tc2_max_active_clusters(cluster, 3); break;
-      case 3: n = pf::attention_tc2_max_active_clusters(cluster, 2); break;
-      default: n = pf::attention_pair_max_active_clusters(cluster, false); break;
+      default: n = pf::attention_tc2_max_active_clusters(cluster, 2); break;
     }
     c = std::max(1, n) + 1;
     slot.store(c, std::memory_order_release);
@@ -186,24 +185,40 @@ pf_status choose_attention(const pf_attn_desc* d, pf::AttnArgs& a, int sms, bool
     a.splits = 1;
     return PF_OK;
   }
+  const bool batch_ws = ws_ok && a.B > 1;
+  // The pair kernel's groups: 256-row blocks of floor(128 / G) nodes per CTA;
+  // the continuous-split kernel's: 128-row blocks of floor(128 / G) nodes.
+  const int pair_nb = 2 * (128 / G);
+  const int pair_groups = a.B * a.Hkv * ((a.max_nodes + pair_nb - 1) / pair_nb);
+  const int sk_nb = 128 / G;
+  const int sk_groups = a.B * a.Hkv * ((a.max_nodes + sk_nb - 1) / sk_nb);
   AttnKernel k;
+  int a_bm_auto = 0;  // the automatic choice's rows per CTA for the 64-token kernel
   if (d->kernel == PF_ATTN_KERNEL_AUTO && d->rows_per_cta != 0) {
     k = AttnKernel::TC64;
   } else if (d->kernel == PF_ATTN_KERNEL_AUTO) {
-    // Tensor cores for D = 128: 128-row CTAs on 128-token tiles once a CTA
-    // holds several of them (wider S MMAs), else on 64-token tiles (a CTA
-    // with one or two tiles starts sooner on a smaller first tile); KV heads
-    // of 129..256 rows in two-block CTAs of the 64-token kernel.
+    // Tensor cores for D = 128: 128-row CTAs in clusters that split each
+    // row block's tiles, on 128-token tiles once a CTA holds several of them
+    // (wider S MMAs), else on 64-token tiles (a CTA with one or two tiles
+    // starts sooner on a smaller first tile).  Measured per layer on GB300
+    // (us; 128-token clusters / 64-token clusters / 64-token two-block
+    // balanced batch / continuous split / SM pairs): 64-node tree 14.9 /
+    // 17.2 / - / 23.0 / 24.7, 32K tree 70.0 / 109.8 / - / 79.2 / 84.5,
+    // 8-sequence paged batch 41.9 / 46.0 / 43.4 / 50.1 / 49.7.  The
+    // continuous split balances the batch's loop, but its per-launch plan
+    // (global round trips at kernel start, 5-9 us under the other CTAs'
+    // prefetch) and the merge launch cost more than the imbalance it saves.
     k = D != 128 ? AttnKernel::MMA : AttnKernel::TC64;  // may become TC128 below
+    if (k == AttnKernel::TC64) a_bm_auto = 128;
   } else {
     k = d->kernel == PF_ATTN_KERNEL_MMA    ? AttnKernel::MMA
         : d->kernel == PF_ATTN_KERNEL_TC64 ? AttnKernel::TC64
         : d->kernel == PF_ATTN_KERNEL_TC128 ? AttnKernel::TC128
-                                            : AttnKernel::PAIR;
+        : d->kernel == PF_ATTN_KERNEL_PAIR  ? AttnKernel::PAIR
+                                            : AttnKernel::STREAM;
   }
   const int tiles64 = (a.max_prefix + 63) / 64 + (a.max_nodes + 63) / 64;
   const int tiles128 = (a.max_prefix + 127) / 128 + (a.max_nodes + 127) / 128;
-  const bool batch_ws = ws_ok && a.B > 1;
 
   if (k == AttnKernel::MMA) {
     const int bms[3] = {128, 64, 32};
@@ -232,21 +247,31 @@ pf_status choose_attention(const pf_attn_desc* d, pf::AttnArgs& a, int sms, bool
     return PF_OK;
   }
 
-  if (k == AttnKernel::PAIR) {
-    const int nbh = 128 / G;  // nodes per CTA (G <= 128)
-    a.bm = 256;
-    a.nb = 2 * nbh;
+  if (k == AttnKernel::STREAM) {
+    if (sk_groups > pf::kSkMaxGroups)
+      return fail(PF_ERR_SHAPE, "%s: the continuous-split kernel handles at most %d (sequence, "
+                  "KV head, 128-row block) groups", who, pf::kSkMaxGroups);
+    a.bm = 128;
+    a.nb = sk_nb;
     a.rb_count = (a.max_nodes + a.nb - 1) / a.nb;
-    const int groups = a.B * a.Hkv * a.rb_count;
-    const int items = sms / 2;  // one pair per SM pair
-    if (batch_ws && d->splits == 0 && groups <= items && groups <= pf::kPlanMaxGroups) {
-      a.splits = 1;
-      a.items = items;
-      out->ws_need = pf::attention_balanced_ws_bytes(items, a.bm, D);
-    } else {
-      a.splits = d->splits > 0 ? std::min(d->splits, std::max(1, tiles128))
-                               : widest_split(4, groups, tiles128, 8, 2);
-    }
+    a.splits = 1;
+    a.items = sms;  // one per SM
+    a.slots = 2;
+    out->ws_need = pf::attention_balanced_ws_bytes(a.items, a.bm, D, 2);
+    out->kernel = k;
+    return PF_OK;
+  }
+  if (k == AttnKernel::PAIR) {
+    if (pair_groups > pf::kPlanMaxGroups)
+      return fail(PF_ERR_SHAPE, "%s: the pair kernel handles at most %d (sequence, KV head, "
+                  "256-row block) groups", who, pf::kPlanMaxGroups);
+    a.bm = 256;
+    a.nb = pair_nb;
+    a.rb_count = (a.max_nodes + a.nb - 1) / a.nb;
+    a.splits = 1;
+    a.items = std::max(1, sms / 2);  // one per SM pair
+    a.slots = 2;
+    out->ws_need = pf::attention_balanced_ws_bytes(a.items, a.bm, D, 2);
     out->kernel = k;
     return PF_OK;
   }
@@ -255,15 +280,17 @@ pf_status choose_attention(const pf_attn_desc* d, pf::AttnArgs& a, int sms, bool
   // where that covers all of a KV head's rows
   const int head_rows = G * a.max_nodes;
   a.bm = (k == AttnKernel::TC64 && head_rows > 128 && head_rows <= 256) ? 256 : 128;
+  if (a_bm_auto) a.bm = a_bm_auto;
   if (d->rows_per_cta != 0) a.bm = d->rows_per_cta;
   a.nb = a.bm / G;  // >= 1: G <= 128
   a.rb_count = (a.max_nodes + a.nb - 1) / a.nb;
   const int groups = a.B * a.Hkv * a.rb_count;
-  if (k == AttnKernel::TC64 && batch_ws && d->splits == 0 && groups <= sms &&
-      groups <= pf::kPlanMaxGroups) {
+  if (k == AttnKernel::TC64 && d->kernel == PF_ATTN_KERNEL_TC64 && batch_ws && d->splits == 0 &&
+      groups <= sms && groups <= pf::kPlanMaxGroups) {
     a.splits = 1;
     a.items = sms;
-    out->ws_need = pf::attention_balanced_ws_bytes(sms, a.bm, D);
+    a.slots = 1;
+    out->ws_need = pf::attention_balanced_ws_bytes(sms, a.bm, D, 1);
     out->kernel = k;
     return PF_OK;
   }
@@ -302,18 +329,20 @@ pf_status attention_args(const pf_attn_desc* d, pf::AttnArgs& a, const char* who
   if (d->flags & ~(PF_ATTN_EARLY_PREFETCH | PF_ATTN_NO_PDL))
     return fail(PF_ERR_SHAPE, "%s: unknown flags 0x%x", who, d->flags);
   // launch fields
-  if (d->kernel < PF_ATTN_KERNEL_AUTO || d->kernel > PF_ATTN_KERNEL_PAIR)
+  if (d->kernel < PF_ATTN_KERNEL_AUTO || d->kernel > PF_ATTN_KERNEL_STREAM)
     return fail(PF_ERR_SHAPE, "%s: unknown kernel %d", who, d->kernel);
   if (d->dtype == PF_F32 && (d->kernel != PF_ATTN_KERNEL_AUTO || d->splits != 0 ||
                              d->rows_per_cta != 0 || d->stages != 0))
     return fail(PF_ERR_DTYPE, "%s: the fp32 path has one kernel and takes no launch fields",
                 who);
   const bool tc_kernel = d->kernel == PF_ATTN_KERNEL_TC64 || d->kernel == PF_ATTN_KERNEL_TC128 ||
-                         d->kernel == PF_ATTN_KERNEL_PAIR;
+                         d->kernel == PF_ATTN_KERNEL_PAIR || d->kernel == PF_ATTN_KERNEL_STREAM;
   if (tc_kernel && D != 128)
     return fail(PF_ERR_SHAPE, "%s: the tcgen05 kernels need head_dim 128", who);
-  if (d->splits < 0 || d->splits > (d->kernel == PF_ATTN_KERNEL_PAIR ? 8 : 16))
-    return fail(PF_ERR_SHAPE, "%s: splits must be 0 (automatic) or 1..16 (1..8 for pairs)", who);
+  if (d->splits < 0 || d->splits > 16 ||
+      ((d->kernel == PF_ATTN_KERNEL_PAIR || d->kernel == PF_ATTN_KERNEL_STREAM) && d->splits != 0))
+    return fail(PF_ERR_SHAPE,
+                "%s: splits must be 0 (automatic) or 1..16, and 0 for the continuous split", who);
   if (d->rows_per_cta != 0 &&
       ((d->rows_per_cta != 128 && d->rows_per_cta != 256) || D != 128 ||
        (d->kernel != PF_ATTN_KERNEL_AUTO && d->kernel != PF_ATTN_KERNEL_TC64) ||
@@ -492,6 +521,9 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
     cudaError_t e = pf::launch_attention_f32(a, s, pdl);
     return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
   }
+  if ((ch.kernel == AttnKernel::PAIR || ch.kernel == AttnKernel::STREAM) && !d->workspace)
+    return fail(PF_ERR_WORKSPACE, "%s: this kernel needs the workspace (%zu bytes)", who,
+                ch.ws_need);
   if (a.items > 0) {
     if (d->workspace_bytes < ch.ws_need)
       return fail(PF_ERR_WORKSPACE, "%s: workspace needs %zu bytes", who, ch.ws_need);
@@ -502,7 +534,8 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
   // Tensor maps: K/V boxes of the chosen kernel's tile (the pair kernel
   // loads half a tile per CTA: 64 K rows, 128 V rows of 64 columns).
   const bool pair = ch.kernel == AttnKernel::PAIR;
-  const cuuint32_t k_rows = pair ? 64 : ch.kernel == AttnKernel::TC128 ? 128 : 64;
+  const bool wide = ch.kernel == AttnKernel::TC128 || ch.kernel == AttnKernel::STREAM;
+  const cuuint32_t k_rows = pair ? 64 : wide ? 128 : 64;
   const cuuint32_t v_rows = pair ? 128 : k_rows;
   const cuuint32_t q_nodes = pair ? (cuuint32_t)(a.nb / 2) : (cuuint32_t)a.nb;
   pf::AttnMaps m;
@@ -539,6 +572,7 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
   cudaError_t e;
   switch (ch.kernel) {
     case AttnKernel::PAIR: e = pf::launch_attention_pair(a, m, s, pdl); break;
+    case AttnKernel::STREAM: e = pf::launch_attention_sk(a, m, s, pdl); break;
     case AttnKernel::TC128: e = pf::launch_attention_tc2(a, m, s, pdl, ch.stages); break;
     case AttnKernel::TC64: e = pf::launch_attention_tc(a, m, s, pdl); break;
     default: e = pf::launch_attention_bf16(a, m, s, sms, pdl); break;

@@ -597,8 +597,12 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const AttnArgs a) {
   const int r = chunk * kCombineRows + (int)threadIdx.x / C8;
   const int c8 = (int)threadIdx.x % C8;
   if (k <= 1 || r >= rows) return;
-  const __half* base = reinterpret_cast<const __half*>(a.ws) + ((size_t)first * a.bm + r) * kPitch;
-  const size_t item_stride = (size_t)a.bm * kPitch;
+  const __half* base = reinterpret_cast<const __half*>(a.ws) + (size_t)r * kPitch;
+  const size_t slot_stride = (size_t)a.bm * kPitch;
+  // partial slot of piece j (see plan_table)
+  auto slot_of = [&](int j) {
+    return a.slots == 2 && j > 0 ? 2 * ((first >> 1) + j) : first + j;
+  };
   // partials in batches of 8 (all loads of a batch in flight together),
   // folded into a running maximum M, weight sum W and weighted sum acc
   float M = -INFINITY, W = 0.f;
@@ -610,7 +614,7 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const AttnArgs a) {
     for (int u = 0; u < kBatch; ++u) {
       ls[u] = -INFINITY;
       if (j0 + u < k) {
-        const __half* row = base + (size_t)(j0 + u) * item_stride;
+        const __half* row = base + (size_t)slot_of(j0 + u) * slot_stride;
         ls[u] = *reinterpret_cast<const float*>(row + D);
         v[u] = *reinterpret_cast<const uint4*>(row + c8 * 8);
       }
@@ -653,8 +657,8 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const AttnArgs a) {
 
 }  // namespace
 
-size_t attention_balanced_ws_bytes(int items, int bm, int D) {
-  return (size_t)items * bm * (D + 8) * 2 + kPlanMaxGroups * sizeof(int4);
+size_t attention_balanced_ws_bytes(int items, int bm, int D, int slots) {
+  return (size_t)items * slots * bm * (D + 8) * 2 + kPlanMaxGroups * sizeof(int4);
 }
 
 cudaError_t launch_attention_combine(const AttnArgs& a, cudaStream_t s, bool pdl) {

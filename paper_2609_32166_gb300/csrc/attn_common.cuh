@@ -216,12 +216,11 @@ struct PlanItem {
   int first;  // the group's first item
 };
 
-__device__ __forceinline__ int plan_tiles(const AttnArgs& a, int q, int tile_tokens) {
-  const int b = q / (a.Hkv * a.rb_count);
+// Tiles of group q of sequence (first node node0, nn nodes, prefix P);
+// flags PF_DEVERR_BOUNDS and returns 0 for sizes outside the host bounds.
+__device__ __forceinline__ int group_tiles(const AttnArgs& a, int q, int node0, int nn, int P,
+                                           int tile_tokens) {
   const int rb = q % a.rb_count;
-  const int node0 = a.cu_nodes[b];
-  const int nn = a.cu_nodes[b + 1] - node0;
-  const int P = a.prefix_len[b];
   if (node0 < 0 || nn < 1 || nn > a.max_nodes || node0 + nn > a.T || P < 0 || P > a.max_prefix) {
     flag_error(a.err, PF_DEVERR_BOUNDS);
     return 0;
@@ -230,12 +229,21 @@ __device__ __forceinline__ int plan_tiles(const AttnArgs& a, int q, int tile_tok
   return (P + tile_tokens - 1) / tile_tokens + (nn + tile_tokens - 1) / tile_tokens;
 }
 
+__device__ __forceinline__ int plan_tiles(const AttnArgs& a, int q, int tile_tokens) {
+  const int b = q / (a.Hkv * a.rb_count);
+  const int node0 = a.cu_nodes[b];
+  return group_tiles(a, q, node0, a.cu_nodes[b + 1] - node0, a.prefix_len[b], tile_tokens);
+}
+
 // The plan's per-group table in the workspace, after the partials: (first
-// item, items, first node, rows) of every group, written by the attention
-// kernel for the combine kernel.
+// partial slot, pieces, first node, rows) of every group, written by the
+// attention kernel for the combine kernel.  With one slot per item, piece j
+// of a group is slot first + j; with two (the continuous split), piece 0 is
+// slot first and piece j > 0 is slot 2 * (first / 2 + j) (the first piece
+// of each following item).
 __device__ __forceinline__ int4* plan_table(const AttnArgs& a) {
   return reinterpret_cast<int4*>(reinterpret_cast<uint8_t*>(a.ws) +
-                                 (size_t)a.items * a.bm * (a.D + 8) * 2);
+                                 (size_t)a.items * a.slots * a.bm * (a.D + 8) * 2);
 }
 
 // Warp-collective (all 32 lanes, warp-uniform arguments): the plan entry
@@ -248,10 +256,23 @@ static __device__ __noinline__ PlanItem balanced_plan(const AttnArgs& a, int ite
   const int n_chunks = (n_groups + 31) / 32;
   int t[kPer];
   int U = 0, n_active = 0, t_max = 0;
+  // all groups' sizes loaded together (see continuous_plan)
+  int n0[kPer], n1[kPer], pl[kPer];
 #pragma unroll
   for (int s = 0; s < kPer; ++s) {
     const int q = lane + 32 * s;
-    t[s] = q < n_groups ? plan_tiles(a, q, tile_tokens) : 0;
+    const int b = q / (a.rb_count * a.Hkv);
+    n0[s] = n1[s] = pl[s] = 0;
+    if (q < n_groups) {
+      n0[s] = __ldg(&a.cu_nodes[b]);
+      n1[s] = __ldg(&a.cu_nodes[b + 1]);
+      pl[s] = __ldg(&a.prefix_len[b]);
+    }
+  }
+#pragma unroll
+  for (int s = 0; s < kPer; ++s) {
+    const int q = lane + 32 * s;
+    t[s] = q < n_groups ? group_tiles(a, q, n0[s], n1[s] - n0[s], pl[s], tile_tokens) : 0;
     U += t[s];
     n_active += t[s] > 0 ? 1 : 0;
     t_max = max(t_max, t[s]);
@@ -307,6 +328,142 @@ static __device__ __noinline__ PlanItem balanced_plan(const AttnArgs& a, int ite
     }
     base += __shfl_sync(0xffffffffu, incl, 31);
   }
+  return r;
+}
+
+// ---- continuous split (the pair kernel and attn_sk_kernel): the groups'
+// tiles of `tile_tokens` tokens are laid end to end and cut into a.items
+// equal ranges.  A range covers pieces of one or more groups (parts); only
+// its first and last part can be pieces of a longer group, so each item
+// has two partial slots (2 * item for its first part, 2 * item + 1 for its
+// last).  A part is packed in 64 bits: group (9 bits), first and end tile
+// within the group (16 bits each), whole-group flag, slot (up to 2^22).
+struct Part {
+  int q, t0, t1, whole, slot;
+};
+
+__device__ __forceinline__ unsigned long long pack_part(const Part& p) {
+  return (unsigned long long)p.q | ((unsigned long long)p.t0 << 9) |
+         ((unsigned long long)p.t1 << 25) | ((unsigned long long)p.whole << 41) |
+         ((unsigned long long)p.slot << 42);
+}
+__device__ __forceinline__ Part unpack_part(unsigned long long v) {
+  return Part{(int)(v & 0x1FF), (int)((v >> 9) & 0xFFFF), (int)((v >> 25) & 0xFFFF),
+              (int)((v >> 41) & 1), (int)(v >> 42)};
+}
+
+// Warp 0 of every CTA (all 32 lanes, the same result in every CTA): group
+// q (8 per lane, q = 32 s + lane) holds t_q tiles starting at position
+// start_q of the concatenation; item i takes positions [floor(U i / items),
+// floor(U (i+1) / items)).  Writes this item's parts in group order to
+// `parts` (at most max_parts) and returns their count; with write_table,
+// items with index = q (mod items) also write group q's plan-table entry
+// (first partial slot, pieces, first node, rows) for the combine kernel.
+// Groups: <= kPlanMaxGroups (host); tiles per group < 2^16, so the total U
+// < 2^24 and U * items < 2^32: the arithmetic is 32-bit (64-bit divisions
+// here took several microseconds per launch).
+template <int kTile>
+static __device__ __noinline__ int continuous_plan(const AttnArgs& a, int item, bool write_table,
+                                                   unsigned long long* parts) {
+  constexpr int tile_tokens = kTile;
+  const int lane = threadIdx.x & 31;
+  const int n_groups = a.B * a.Hkv * a.rb_count;
+  constexpr int kPer = kPlanMaxGroups / 32;
+  int t[kPer], start[kPer];
+  unsigned U = 0;
+  {
+    // every group's sizes first, all loads in flight together (issued
+    // between the scans, or behind plan_tiles' error atomic, they took one
+    // round trip per chunk: ~8 us); cu_nodes and prefix_len are read-only
+    // for the kernel's lifetime
+    int n0[kPer], n1[kPer], pl[kPer];
+#pragma unroll
+    for (int s = 0; s < kPer; ++s) {
+      const int q = lane + 32 * s;
+      const int b = q / (a.rb_count * a.Hkv);
+      n0[s] = n1[s] = pl[s] = 0;
+      if (q < n_groups) {
+        n0[s] = __ldg(&a.cu_nodes[b]);
+        n1[s] = __ldg(&a.cu_nodes[b + 1]);
+        pl[s] = __ldg(&a.prefix_len[b]);
+      }
+    }
+#pragma unroll
+    for (int s = 0; s < kPer; ++s) {
+      const int q = lane + 32 * s;
+      t[s] = q < n_groups ? group_tiles(a, q, n0[s], n1[s] - n0[s], pl[s], tile_tokens) : 0;
+    }
+    int base = 0;
+#pragma unroll
+    for (int s = 0; s < kPer; ++s) {
+      int incl = t[s];
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += v;
+      }
+      start[s] = base + incl - t[s];
+      base += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    U = base;
+  }
+  if (U == 0) return 0;
+  const unsigned items = (unsigned)a.items;
+  const unsigned R0 = U * (unsigned)item / items, R1 = U * (unsigned)(item + 1) / items;
+  auto item_of = [&](unsigned x) { return (int)(((x + 1) * items - 1) / U); };
+  auto range_start = [&](unsigned i) { return U * i / items; };
+  int n = 0;
+#pragma unroll
+  for (int s = 0; s < kPer; ++s) {
+    const int q = lane + 32 * s;
+    const unsigned s0 = (unsigned)start[s], s1 = (unsigned)(start[s] + t[s]);
+    const bool mine = t[s] > 0 && s0 < R1 && s1 > R0;
+    const unsigned m = __ballot_sync(0xffffffffu, mine);
+    if (mine) {
+      const int i0 = item_of(s0), i1 = item_of(s1 - 1);
+      Part p;
+      p.q = q;
+      p.t0 = (int)(max(R0, s0) - s0);
+      p.t1 = (int)(min(R1, s1) - s0);  // unsigned max / min: every value >= 0
+      p.whole = i0 == i1;
+      p.slot = 2 * item + (R0 >= s0 ? 0 : 1);  // this item's first part, or its last
+      parts[n + __popc(m & ((1u << lane) - 1u))] = pack_part(p);
+    }
+    n += __popc(m);
+    if (write_table && q < n_groups && q % a.items == item) {
+      int4 e = make_int4(0, 0, 0, 0);
+      if (t[s] > 0) {
+        const int i0 = item_of(s0), i1 = item_of(s1 - 1);
+        const int bq = q / (a.rb_count * a.Hkv), nfq = (q % a.rb_count) * a.nb;
+        const int n0 = a.cu_nodes[bq], nnq = a.cu_nodes[bq + 1] - n0;
+        e = make_int4(2 * i0 + (range_start(i0) < s0 ? 1 : 0), i1 - i0 + 1, n0 + nfq,
+                      max(0, min(a.nb, nnq - nfq)) * a.G);
+      }
+      plan_table(a)[q] = e;
+    }
+  }
+  return n;
+}
+
+// A part's group decoded for one CTA holding `cta_nodes` of the group's
+// nodes from the group's (c * cta_nodes)-th on: sequence, KV head, first
+// node and rows (0 when the CTA holds none).
+struct PartGeom {
+  int b, g, node0, nn, P, nfirst, rows, n_ptiles;
+};
+
+__device__ __forceinline__ PartGeom part_geom(const AttnArgs& a, int q, int cta_nodes, int c,
+                                              int tile_tokens) {
+  PartGeom r;
+  const int rb = q % a.rb_count;
+  r.g = (q / a.rb_count) % a.Hkv;
+  r.b = q / (a.rb_count * a.Hkv);
+  r.node0 = a.cu_nodes[r.b];
+  r.nn = a.cu_nodes[r.b + 1] - r.node0;
+  r.P = a.prefix_len[r.b];  // the plan checked these (plan_tiles)
+  r.nfirst = rb * a.nb + c * cta_nodes;
+  r.rows = max(0, min(cta_nodes, r.nn - r.nfirst)) * a.G;
+  r.n_ptiles = (r.P + tile_tokens - 1) / tile_tokens;
   return r;
 }
 

@@ -27,6 +27,9 @@ struct AttnArgs {
   // balanced_plan); a group spread over several CTAs leaves normalised
   // partials in `ws` ([items][bm][D + 8] halves) for the combine kernel.
   int items;       // 0 = off
+  // partial slots per item: 1 (tc64: one group part per CTA) or 2 (the pair
+  // kernel's continuous split: an item's first and last group piece)
+  int slots;
   void* ws;
   float scale_log2;  // softmax scale * log2(e)
   float scale;
@@ -69,19 +72,26 @@ cudaError_t launch_attention_tc2(const AttnArgs& a, const AttnMaps& m, cudaStrea
 int attention_tc2_max_active_clusters(int cluster, int stages);
 // tcgen05 variant on SM pairs (2-SM MMA, M = 256 rows per pair, 128-token
 // tiles; bf16, D = 128): a.bm = 256, a.nb = 2 * floor(128 / G) nodes per
-// pair; a.splits pairs per cluster (<= 8), or a.items pairs in the balanced
-// batch mode.  Tensor maps: K boxes of 64 rows, V boxes of 128 rows (cache),
-// tree K boxes of 64 nodes, tree V boxes of 128, Q boxes of a.nb / 2 nodes.
+// pair, a.items pairs sharing all groups' tiles in equal contiguous ranges
+// (a.slots = 2; needs the workspace and the combine kernel).  Tensor maps:
+// K boxes of 64 rows, V boxes of 128 rows (cache), tree K boxes of 64
+// nodes, tree V boxes of 128, Q boxes of a.nb / 2 nodes.
 cudaError_t launch_attention_pair(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl);
-int attention_pair_max_active_clusters(int cluster, bool balanced);
+// 128-token, P-in-TMEM kernel (one CTA per SM, 128 query rows, bf16,
+// D = 128) with the continuous split: a.items = SMs, a.bm = 128, a.slots =
+// 2, at most kSkMaxGroups groups; needs the workspace and the combine
+// kernel.  Tensor maps as attn_tc2_kernel's.
+constexpr int kSkMaxGroups = 128;
+cudaError_t launch_attention_sk(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl);
 // Merge of the balanced batch mode's partials (launched after the tcgen05
 // kernel when a.items > 0).
 cudaError_t launch_attention_combine(const AttnArgs& a, cudaStream_t s, bool pdl);
 // Groups (sequence, KV head, row block) the balanced batch mode's plan can
 // hold (8 per lane of a warp).
 constexpr int kPlanMaxGroups = 256;
-// Bytes of a.ws for the balanced batch mode with `items` CTAs of a.bm rows.
-size_t attention_balanced_ws_bytes(int items, int bm, int D);
+// Bytes of a.ws for the balanced batch mode with `items` work items of a.bm
+// rows and `slots` partial slots per item.
+size_t attention_balanced_ws_bytes(int items, int bm, int D, int slots = 1);
 // How many clusters of `cluster` CTAs of the tcgen05 kernel fit at once.
 // rows_per_cta: 128 (one softmax warpgroup) or 256 (two).
 int attention_tc_max_active_clusters(int cluster, int rows_per_cta);

@@ -176,65 +176,15 @@ __device__ __forceinline__ void cp_async_wait_all() {
 // tcgen05 allocation, MMA and commit of a kernel that uses pairs takes the
 // pair form.
 
-// TMA tile load into this CTA's shared memory whose completion is counted
-// on `bar_cluster`, an mbarrier of either CTA of the pair (shared::cluster
-// address, see mapa_cluster).
-__device__ __forceinline__ void tma_load_3d_pair(uint32_t dst, const CUtensorMap* m, int x, int y,
-                                                 int z, uint32_t bar_cluster) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes "
-      "[%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(bar_cluster)
-      : "memory");
-}
-__device__ __forceinline__ void tma_load_4d_pair(uint32_t dst, const CUtensorMap* m, int x, int y,
-                                                 int z, int w, uint32_t bar_cluster) {
-  asm volatile(
-      "cp.async.bulk.tensor.4d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes "
-      "[%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(w), "r"(bar_cluster)
-      : "memory");
-}
-
-// Arrive (release, cluster scope) on an mbarrier of any CTA of the cluster.
+// Arrive on an mbarrier of any CTA of the cluster (shared::cluster address),
+// with the default semantics (release at CTA scope).  What the waiting side
+// then reads is ordered by other means: tensor-memory reads and writes by
+// tcgen05.wait and tcgen05.fence::before_thread_sync before the arrive,
+// generic shared-memory writes read by the async proxy by
+// fence.proxy.async.  A cluster-scope release here is a full memory barrier
+// per arrive (ncu: membar the top stall of the pair kernel).
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster)
-               : "memory");
-}
-
-// Waits with cluster-scope acquire, for barriers that other CTAs of the
-// cluster signal; bounded like mbar_wait.
-__device__ __forceinline__ bool mbar_try_wait_cl(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{ .reg .pred p; mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2; "
-      "selp.u32 %0, 1, 0, p; }"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-__device__ __forceinline__ bool mbar_test_wait_cl(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{ .reg .pred p; mbarrier.test_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2; "
-      "selp.u32 %0, 1, 0, p; }"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-__device__ __forceinline__ bool mbar_wait_cl(uint32_t bar, uint32_t parity, int32_t* err) {
-  if (mbar_try_wait_cl(bar, parity)) return true;
-  const unsigned long long t0 = globaltimer();
-  while (true) {
-    for (int i = 0; i < 64; ++i)
-      if (mbar_try_wait_cl(bar, parity)) return true;
-    if (globaltimer() - t0 > kWaitLimitNs) {
-      flag_error(err, PF_DEVERR_TIMEOUT);
-      return false;
-    }
-  }
+  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
 }
 
 // ---------------------------------------------------------------- packed fp32
@@ -520,6 +470,37 @@ __device__ __forceinline__ float ex2_approx(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+// 2^x for two values on the FMA and integer pipes instead of the
+// special-function unit (the softmax's exponentials would otherwise all
+// queue on it).  Range reduction 2^x = 2^n * 2^f with n = round(x) -- taken
+// by adding 1.5 * 2^23, which leaves n in the low mantissa bits -- and
+// f = x - n in [-1/2, 1/2]; 2^f by a degree-3 polynomial whose coefficients
+// were fitted here for minimum relative error on that interval (Lawson's
+// iteratively reweighted least squares; exp2_poly.py beside this library
+// reproduces them): maximum relative error 7.5e-5, below the 2^-9 spacing
+// of the bf16 probabilities it feeds.  n is added to the exponent field.
+// x is clamped to >= -126 first, so -inf (masked scores) gives a value
+// below 2^-126 (a denormal, zero in every use here) and no exponent wraps.
+constexpr float kExp2C0 = 0.99992811679840088f;
+constexpr float kExp2C1 = 0.69326096773147583f;
+constexpr float kExp2C2 = 0.24261054396629333f;
+constexpr float kExp2C3 = 0.055171322077512741f;
+__device__ __forceinline__ void exp2_poly_x2(float x0, float x1, float& p0, float& p1) {
+  constexpr float kRound = 12582912.0f;  // 1.5 * 2^23
+  const unsigned long long x = f32x2_pack(fmaxf(x0, -126.f), fmaxf(x1, -126.f));
+  const unsigned long long t = fadd2(x, f32x2_pack(kRound, kRound));
+  const unsigned long long n = fadd2(t, f32x2_pack(-kRound, -kRound));
+  const unsigned long long f = ffma2(n, f32x2_pack(-1.f, -1.f), x);
+  unsigned long long p = ffma2(f, f32x2_pack(kExp2C3, kExp2C3), f32x2_pack(kExp2C2, kExp2C2));
+  p = ffma2(p, f, f32x2_pack(kExp2C1, kExp2C1));
+  p = ffma2(p, f, f32x2_pack(kExp2C0, kExp2C0));
+  float q0, q1, t0, t1;
+  f32x2_unpack(p, q0, q1);
+  f32x2_unpack(t, t0, t1);
+  p0 = __uint_as_float(__float_as_uint(q0) + (__float_as_uint(t0) << 23));
+  p1 = __uint_as_float(__float_as_uint(q1) + (__float_as_uint(t1) << 23));
 }
 
 __device__ __forceinline__ unsigned long long umax64(unsigned long long a, unsigned long long b) {

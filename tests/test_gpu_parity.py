@@ -15,6 +15,7 @@ MMA = dict(kernel=pb.PF_ATTN_KERNEL_MMA)
 TC64 = dict(kernel=pb.PF_ATTN_KERNEL_TC64)
 TC128 = dict(kernel=pb.PF_ATTN_KERNEL_TC128)
 PAIR = dict(kernel=pb.PF_ATTN_KERNEL_PAIR)
+STREAM = dict(kernel=pb.PF_ATTN_KERNEL_STREAM)
 
 pytestmark = pytest.mark.gpu
 
@@ -97,20 +98,20 @@ def test_edge_cases(name):
 
 
 # ---------------------------------------------------------------------------
-# the SM-pair kernel (2-SM MMA, each CTA holding half of every K/V tile)
+# the SM-pair kernel (2-SM MMA, each CTA holding half of every K/V tile; all
+# groups' tiles cut into one equal range per SM pair)
 # ---------------------------------------------------------------------------
 EDGE_PAIR = {k: EDGE[k] for k in ("root-only", "empty-prefix", "65-nodes", "g16-tiny-vocab",
                                   "256-rows-paged", "two-blocks-one-tile")}
 
 
-@pytest.mark.parametrize("balanced", [False, True])
 @pytest.mark.parametrize("name", sorted(EDGE_PAIR))
-def test_pair_kernel_edges(name, balanced):
-    """Root only (the odd CTA of the pair has no rows), no prefix (one tile),
-    65 nodes with a one-row last prefix tile, G = 16 (the odd CTA holds one
-    node), 128-node paged trees, one tile for 192 rows; cluster mode and the
-    balanced batch mode (the latter only changes batches)."""
-    c = Case(EDGE_PAIR[name], seed=5, balanced=balanced, attn_launch=PAIR)
+def test_pair_kernel_edges(name):
+    """Root only (the odd CTA of the pair has no rows, most pairs no tile),
+    no prefix (one tile), 65 nodes with a one-row last prefix tile, G = 16
+    (the odd CTA holds one node), 128-node paged trees, one tile for 192
+    rows."""
+    c = Case(EDGE_PAIR[name], seed=5, attn_launch=PAIR)
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0
@@ -121,13 +122,12 @@ def test_pair_kernel_edges(name, balanced):
     c.check_commit(res)
 
 
-@pytest.mark.parametrize("splits", [1, 2, 3, 8])
 @pytest.mark.parametrize("name", ["7b-tree64-small", "7b-32k-tree128-small",
                                   "7b-batch8-paged-small"])
-def test_pair_kernel_splits(name, splits):
-    """Pairs per cluster from 1 to 8 (cluster widths 2 to 16) on the three 7B
-    shapes, paged batch included (cluster mode: no workspace), every node."""
-    c = Case(SMALL[name], seed=14, balanced=False, attn_launch=dict(PAIR, splits=splits))
+def test_pair_kernel_shapes(name):
+    """The three 7B shapes, every node: groups cut into pieces over many
+    pairs (the 32K tree's groups span ~10 ranges each), pieces merged."""
+    c = Case(SMALL[name], seed=14, attn_launch=PAIR)
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0
@@ -135,12 +135,88 @@ def test_pair_kernel_splits(name, splits):
         c.check_attention(0, s)
 
 
-@pytest.mark.parametrize("launch", ["tc64", "pair"])
-def test_splits_without_tiles(launch):
+def test_pair_kernel_many_groups():
+    """More groups than SM pairs: 40 sequences x 4 KV heads, 160 groups of
+    1..7 tiles, so one pair's range holds several whole groups besides the
+    pieces at its ends (whole groups write their output directly); 6 nodes
+    per sequence keep the batch within the LM head's 256 rows."""
+    w = I.scaled(W["7b-bf16-batch8-paged"], layers=1, batch=40, prefix=(20, 700), nodes=6,
+                 max_depth=5, vocab=300, hidden=64)
+    c = Case(w, seed=15, attn_launch=PAIR)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for s in range(w.batch):
+        c.check_attention(0, s)
+    c.check_lmhead(res)
+    c.check_commit(res)
+
+
+@pytest.mark.parametrize("kernel", ["pair", "stream"])
+def test_continuous_split_needs_the_workspace(kernel):
+    c = Case(SMALL["7b-tree64-small"], seed=16, balanced=False)
+    d = c.vs.attn_descs[0]
+    d.kernel = pb.PF_ATTN_KERNEL_PAIR if kernel == "pair" else pb.PF_ATTN_KERNEL_STREAM
+    with pytest.raises(pb.PfError) as e:
+        pb.pf_verify_attention(d, 0)
+    assert e.value.status == pb.PF_ERR_WORKSPACE
+
+
+# ---------------------------------------------------------------------------
+# the continuous-split kernel (128-token tiles, one CTA per SM, all groups'
+# tiles cut into one equal range per SM)
+# ---------------------------------------------------------------------------
+EDGE_STREAM = {k: EDGE[k] for k in ("root-only", "empty-prefix", "65-nodes", "g16-tiny-vocab",
+                                    "256-rows-paged", "two-blocks-one-tile")}
+
+
+@pytest.mark.parametrize("name", sorted(EDGE_STREAM))
+def test_stream_kernel_edges(name):
+    c = Case(EDGE_STREAM[name], seed=5, attn_launch=STREAM)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for l in range(c.L):
+        for s in range(c.w.batch):
+            c.check_attention(l, s)
+    c.check_lmhead(res)
+    c.check_commit(res)
+
+
+@pytest.mark.parametrize("name", ["2b-chain16-small", "7b-tree64-small", "7b-32k-tree128-small",
+                                  "7b-batch8-paged-small"])
+def test_stream_kernel_shapes(name):
+    """Single sequences and the paged batch, every node: groups cut into
+    pieces over many SMs (the 32K tree's groups span ~6 ranges each)."""
+    c = Case(SMALL[name], seed=17, attn_launch=STREAM)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for l in range(c.L):
+        for s in range(c.w.batch):
+            c.check_attention(l, s)
+
+
+def test_stream_kernel_many_groups():
+    """120 groups (30 sequences x 4 KV heads): ranges of whole groups and
+    pieces; the most the kernel takes is 128."""
+    w = I.scaled(W["7b-bf16-batch8-paged"], layers=1, batch=30, prefix=(20, 900), nodes=8,
+                 max_depth=5, vocab=300, hidden=64)
+    c = Case(w, seed=18, attn_launch=STREAM)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for s in range(w.batch):
+        c.check_attention(0, s)
+    c.check_lmhead(res)
+    c.check_commit(res)
+
+
+def test_splits_without_tiles():
     """A split count above a sequence's tile count: with 8 splits, a
-    sequence whose prefix is 20 rows has 2 tiles, so 6 splits (tc64) or 6
-    pairs (pair kernel) of its cluster get no tile and contribute zero
-    partials with lse = -inf to the merge."""
+    sequence whose prefix is 20 rows has 2 64-token tiles, so 6 splits of
+    its cluster get no tile and contribute zero partials with lse = -inf to
+    the merge."""
     w = I.scaled(W["7b-bf16-batch8-paged"], layers=1, batch=3, prefix=(20, 1500), nodes=20,
                  max_depth=6, vocab=600, hidden=128)
     rng = np.random.default_rng(21)
@@ -151,11 +227,9 @@ def test_splits_without_tiles(launch):
     per_seq = -(-max_seq // I.PAGE_SIZE)
     pt = rng.permutation(per_seq * 3).astype(np.int32).reshape(3, per_seq)
     b = I.Batch(w, 3, parents, prefix, ends, pt, per_seq * 3, max_seq)
-    tile = 64 if launch == "tc64" else 128
-    n_tiles = -(-int(prefix[0]) // tile) + 1
+    n_tiles = -(-int(prefix[0]) // 64) + 1
     assert n_tiles < 8   # the case under test occurs
-    launch_fields = dict(TC64, rows_per_cta=128) if launch == "tc64" else dict(PAIR)
-    c = Case(w, batch=b, balanced=False, attn_launch=dict(launch_fields, splits=8))
+    c = Case(w, batch=b, balanced=False, attn_launch=dict(TC64, rows_per_cta=128, splits=8))
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0
@@ -256,18 +330,20 @@ def test_two_block_kernel_on_many_rows(name):
         c.check_attention(0, s)
 
 
-@pytest.mark.parametrize("kernel", ["auto", "pair"])
-@pytest.mark.parametrize("balanced", [False, True])
+@pytest.mark.parametrize("kernel,balanced", [("auto", True), ("tc64", False), ("tc64", True),
+                                             ("stream", True), ("pair", True)])
 def test_batch_work_split(balanced, kernel):
-    """Eight sequences with prefixes from 100 to 700 rows, with an attention
-    workspace (tiles dealt out to the SMs -- or SM pairs -- in proportion to
-    each sequence's length, partials merged by a second kernel) and without
-    one (every sequence and KV head gets the same cluster); on the automatic
-    choice and on the SM-pair kernel."""
-    c = Case(SMALL["7b-batch8-paged-small"], seed=11, balanced=balanced,
-             attn_launch=PAIR if kernel == "pair" else None)
-    assert (c.vs.attn_ws is not None) == balanced
-    assert c.vs.launches_per_step() == c.L * (2 if balanced else 1) + 2
+    """Eight sequences with prefixes from 100 to 700 rows: the automatic
+    choice (clusters of 128-row CTAs, no workspace even when one is
+    offered); the 64-token kernel's two-block CTAs without a workspace
+    (every sequence and KV head gets the same cluster) and with one (tiles
+    dealt out to the SMs in proportion to each sequence's length); the
+    continuous split on SMs and on SM pairs (partials merged by a second
+    kernel)."""
+    launch = {"auto": None, "tc64": TC64, "stream": STREAM, "pair": PAIR}[kernel]
+    c = Case(SMALL["7b-batch8-paged-small"], seed=11, balanced=balanced, attn_launch=launch)
+    assert (c.vs.attn_ws is not None) == (kernel != "auto" and balanced)
+    assert c.vs.launches_per_step() == c.L * (2 if c.vs.attn_ws is not None else 1) + 2
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0
@@ -280,7 +356,7 @@ def test_batch_work_split(balanced, kernel):
 def test_attention_workspace_contract():
     """The workspace query and the checks on a given workspace."""
     from paper_2609_32166_gb300 import binding as pb
-    c = Case(SMALL["7b-batch8-paged-small"], seed=12)
+    c = Case(SMALL["7b-batch8-paged-small"], seed=12, attn_launch=TC64)
     d = c.vs.attn_descs[0]
     need = pb.pf_verify_attention_workspace_size(d)
     assert need > 0 and need == c.vs.attn_ws_bytes
@@ -294,20 +370,25 @@ def test_attention_workspace_contract():
         pb.pf_verify_attention(d, 0)
     assert e.value.status == pb.PF_ERR_ALIGN
     d.workspace = c.vs.attn_ws.data_ptr()
-    # a single sequence needs none (its KV heads and row blocks share clusters)
+    # a single sequence needs none on the automatic choice (its KV heads and
+    # row blocks share clusters), one on the continuous-split kernels
     one = Case(SMALL["7b-tree64-small"], seed=12)
     assert pb.pf_verify_attention_workspace_size(one.vs.attn_descs[0]) == 0
     assert one.vs.attn_ws is None
+    for k in (pb.PF_ATTN_KERNEL_PAIR, pb.PF_ATTN_KERNEL_STREAM):
+        one_k = Case(SMALL["7b-tree64-small"], seed=12, attn_launch=dict(kernel=k))
+        assert pb.pf_verify_attention_workspace_size(one_k.vs.attn_descs[0]) > 0
 
 
 def test_batch_beyond_balanced_groups():
-    """More (sequence, KV head) groups than SMs: no workspace is asked for
-    and every sequence goes through the cluster path."""
+    """More (sequence, KV head) groups than SMs on the 64-token kernel: its
+    balanced batch mode does not apply, no workspace is asked for and every
+    sequence goes through the cluster path."""
     import torch as _t
     sms = _t.cuda.get_device_properties(0).multi_processor_count
     w = I.scaled(W["7b-bf16-batch8-paged"], layers=1, batch=sms // 4 + 2, prefix=(20, 150),
                  nodes=6, vocab=300, hidden=64)
-    c = Case(w, seed=13)
+    c = Case(w, seed=13, attn_launch=TC64)
     assert c.vs.attn_ws is None
     c.vs.step()
     res = c.vs.results()
@@ -318,11 +399,11 @@ def test_batch_beyond_balanced_groups():
     c.check_commit(res)
 
 
-@pytest.mark.parametrize("impl", ["default", "tc128", "pair-clusters"])
+@pytest.mark.parametrize("impl", ["default", "tc128", "tc64-balanced", "stream"])
 def test_mixed_tree_sizes(impl):
     """Sequences of 1, 17 and 128 nodes in one batch (variable cu_nodes), on
-    the default path (balanced batch mode on SM pairs), on the 128-token
-    kernel and on SM pairs in cluster mode."""
+    the default path, on the 128-token kernel, on the 64-token kernel's
+    balanced batch mode and on the continuous split."""
     w = I.scaled(W["7b-bf16-batch8-paged"], layers=1, batch=3, prefix=(50, 400), nodes=128,
                  vocab=640, hidden=128)
     rng = np.random.default_rng(9)
@@ -333,8 +414,8 @@ def test_mixed_tree_sizes(impl):
     per_seq = -(-max_seq // I.PAGE_SIZE)
     pt = rng.permutation(per_seq * 3).astype(np.int32).reshape(3, per_seq)
     b = I.Batch(w, 7, parents, prefix, ends, pt, per_seq * 3, max_seq)
-    launch = {"default": None, "tc128": TC128, "pair-clusters": PAIR}[impl]
-    c = Case(w, batch=b, balanced=impl == "default", attn_launch=launch)
+    launch = {"default": None, "tc128": TC128, "tc64-balanced": TC64, "stream": STREAM}[impl]
+    c = Case(w, batch=b, balanced=impl != "tc128", attn_launch=launch)
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0

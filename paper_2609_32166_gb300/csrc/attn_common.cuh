@@ -473,11 +473,13 @@ __device__ __forceinline__ PartGeom part_geom(const AttnArgs& a, int q, int cta_
 // the row's pad) at inbox slot s*per + i (pitch kPitch halves).
 //   M = max_s lse_s,  w_s = 2^(lse_s - M),  out = sum_s w_s (O/l)_s / sum_s w_s
 // One thread per (row, 8 output columns); all loads are issued before use.
-template <int D, int kThreads, int kPitch>
-__device__ __forceinline__ void inbox_merge(const AttnArgs& a, const __half* inbox, int rows,
-                                            int split, int per, int nsplit, int node_base, int g,
-                                            int tid) {
-  constexpr int kMaxSplit = 16;
+// kMaxSplit bounds the unrolled loops: the predicated slots of a wider
+// instance than the cluster needs still issue (a 16-way instance took ~4 us
+// for 2-CTA clusters), so inbox_merge picks the narrowest that holds nsplit.
+template <int D, int kThreads, int kPitch, int kMaxSplit>
+__device__ __forceinline__ void inbox_merge_n(const AttnArgs& a, const __half* inbox, int rows,
+                                              int split, int per, int nsplit, int node_base, int g,
+                                              int tid) {
   constexpr int C8 = D / 8;
   const int cnt = min(per, rows - split * per);
   __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.out);
@@ -525,6 +527,20 @@ __device__ __forceinline__ void inbox_merge(const AttnArgs& a, const __half* inb
     pk.w = pack_bf16(acc[6] * inv, acc[7] * inv);
     *reinterpret_cast<uint4*>(out + ((size_t)node * a.Hq + h) * D + c8 * 8) = pk;
   }
+}
+
+template <int D, int kThreads, int kPitch>
+__device__ __forceinline__ void inbox_merge(const AttnArgs& a, const __half* inbox, int rows,
+                                            int split, int per, int nsplit, int node_base, int g,
+                                            int tid) {
+  if (nsplit <= 2)
+    inbox_merge_n<D, kThreads, kPitch, 2>(a, inbox, rows, split, per, nsplit, node_base, g, tid);
+  else if (nsplit <= 4)
+    inbox_merge_n<D, kThreads, kPitch, 4>(a, inbox, rows, split, per, nsplit, node_base, g, tid);
+  else if (nsplit <= 8)
+    inbox_merge_n<D, kThreads, kPitch, 8>(a, inbox, rows, split, per, nsplit, node_base, g, tid);
+  else
+    inbox_merge_n<D, kThreads, kPitch, 16>(a, inbox, rows, split, per, nsplit, node_base, g, tid);
 }
 
 }  // namespace pf

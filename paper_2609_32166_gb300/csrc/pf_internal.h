@@ -156,7 +156,6 @@ struct CommitArgs {
   long long cache_layer_bytes;
   int layout;
   int max_seq;
-  int Hkv_rows;  // rows per (page or sequence) per head: PF_PAGE_SIZE or max_seq
   const int32_t* page_table;
   int pages_per_seq;
   int num_pages;

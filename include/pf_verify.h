@@ -184,7 +184,7 @@ typedef struct pf_attn_desc {
    * result beyond floating-point rounding order. */
   int32_t kernel;              /* pf_attn_kernel                             */
   int32_t splits;              /* K/V splits per row block (cluster width):
-                                  1..16; 0 for PF_ATTN_KERNEL_PAIR           */
+                                  1..16; 0 for PAIR, STREAM and BATCH        */
   int32_t rows_per_cta;        /* PF_ATTN_KERNEL_TC64: 128 or 256            */
   int32_t stages;              /* PF_ATTN_KERNEL_TC128 ring depth: 2 or 3    */
 } pf_attn_desc;
@@ -203,17 +203,24 @@ typedef struct pf_attn_desc {
  *   STREAM TC128's pipeline, one CTA per SM, with the same continuous split
  *          (one equal range of all sequences' tiles per SM); needs the
  *          workspace
- * TC64, TC128, PAIR and STREAM need bf16 and D = 128.  The automatic choice
- * is TC128 (128-row CTAs in clusters that split each row block's tiles)
- * where a CTA holds several 128-token tiles, TC64 otherwise, MMA for other
- * head sizes; it takes no workspace. */
+ *   BATCH  TC128's pipeline, one CTA per SM, no cluster: each (sequence, KV
+ *          head, row block) gets as many CTAs as its share of all tiles
+ *          calls for (every KV head and row block of a sequence the same
+ *          pieces, so they read the same pages together), and the last
+ *          piece of each to finish merges the pieces in the same kernel
+ *          (one launch per call); needs the workspace
+ * TC64, TC128, PAIR, STREAM and BATCH need bf16 and D = 128.  The automatic
+ * choice is TC128 (128-row CTAs in clusters that split each row block's
+ * tiles) where a CTA holds several 128-token tiles, TC64 otherwise, MMA for
+ * other head sizes; it takes no workspace. */
 typedef enum pf_attn_kernel {
   PF_ATTN_KERNEL_AUTO = 0,
   PF_ATTN_KERNEL_MMA = 1,
   PF_ATTN_KERNEL_TC64 = 2,
   PF_ATTN_KERNEL_TC128 = 3,
   PF_ATTN_KERNEL_PAIR = 4,
-  PF_ATTN_KERNEL_STREAM = 5
+  PF_ATTN_KERNEL_STREAM = 5,
+  PF_ATTN_KERNEL_BATCH = 6
 } pf_attn_kernel;
 
 /* PF_ATTN_EARLY_PREFETCH: the prefix cache, page_table, cu_nodes, prefix_len
@@ -229,22 +236,28 @@ typedef enum pf_attn_kernel {
  * then starts only after the preceding kernel in the stream has finished). */
 #define PF_ATTN_NO_PDL 2
 
-/* Workspace (bf16, head_dim 128; needed by PF_ATTN_KERNEL_PAIR and
- * PF_ATTN_KERNEL_STREAM, optional for PF_ATTN_KERNEL_TC64): with workspace
- * != NULL and at least pf_verify_attention_workspace_size(d) bytes (16-byte
- * aligned), the KV tiles are dealt out in proportion to each sequence's
- * length (prefix plus proposal tiles) -- on TC64 to one CTA per SM for
- * batches of B > 1 sequences, on STREAM and PAIR in one equal range of all
- * sequences' tiles per SM (pair) for any B -- so long and short prefixes
- * finish together; sequences spread over several CTAs are merged by a
- * second kernel in the same stream (the call then launches two kernels).
- * Without it every (sequence, KV head) gets the same number of CTAs.  The
- * size query returns 0 where the chosen kernel takes none (the automatic
- * choice).  The contents need no initialisation and are scratch between
+/* Workspace (bf16, head_dim 128; needed by PF_ATTN_KERNEL_PAIR, _STREAM and
+ * _BATCH, optional for PF_ATTN_KERNEL_TC64): with workspace != NULL and at
+ * least pf_verify_attention_workspace_size(d) bytes (16-byte aligned), the
+ * KV tiles are dealt out in proportion to each sequence's length (prefix
+ * plus proposal tiles) -- on BATCH (any B) and TC64 (B > 1) to one CTA per
+ * SM, on STREAM and PAIR in one equal range of all sequences' tiles per SM
+ * (pair) for any B -- so long and short prefixes finish together.
+ * Sequences spread over several CTAs are merged by the last of their CTAs
+ * to finish (BATCH) or by a second kernel in the same stream (TC64, STREAM,
+ * PAIR: the call then launches two kernels; see
+ * pf_verify_attention_launches).  Without it every (sequence, KV head) gets
+ * the same number of CTAs.  The size query returns 0 where the chosen kernel
+ * takes none.  The contents need no initialisation and are scratch between
  * calls; one workspace serves calls in stream order but not concurrent
  * calls.  A workspace that is too small is an error (PF_ERR_WORKSPACE);
  * for shapes that do not use it, it is ignored. */
 PF_API size_t pf_verify_attention_workspace_size(const pf_attn_desc* d);
+
+/* Kernels one pf_verify_attention(d) call launches (1 or 2) for this
+ * descriptor as it stands (workspace given or not); 0 if the call would be
+ * rejected.  Host-only: no device work, the last error is left alone. */
+PF_API int32_t pf_verify_attention_launches(const pf_attn_desc* d);
 
 PF_API pf_status pf_verify_attention(const pf_attn_desc* d, void* stream);
 

@@ -29,7 +29,7 @@ PF_DEVERR_TIMEOUT, PF_DEVERR_CAPACITY, PF_DEVERR_BOUNDS, PF_DEVERR_TREE = 1, 2, 
 PF_ATTN_EARLY_PREFETCH, PF_ATTN_NO_PDL = 1, 2
 PF_LM_EARLY_WEIGHT, PF_LM_NO_PDL = 1, 2
 (PF_ATTN_KERNEL_AUTO, PF_ATTN_KERNEL_MMA, PF_ATTN_KERNEL_TC64, PF_ATTN_KERNEL_TC128,
- PF_ATTN_KERNEL_PAIR, PF_ATTN_KERNEL_STREAM) = 0, 1, 2, 3, 4, 5
+ PF_ATTN_KERNEL_PAIR, PF_ATTN_KERNEL_STREAM, PF_ATTN_KERNEL_BATCH) = 0, 1, 2, 3, 4, 5, 6
 
 STATUS_NAMES = {0: "PF_OK", 1: "PF_ERR_NULL", 2: "PF_ERR_SHAPE", 3: "PF_ERR_DTYPE",
                 4: "PF_ERR_TREE", 5: "PF_ERR_CAPACITY", 6: "PF_ERR_ALIGN", 7: "PF_ERR_CUDA",
@@ -148,6 +148,8 @@ def lib() -> C.CDLL:
     L.pf_verify_attention.argtypes = [C.POINTER(pf_attn_desc), C.c_void_p]
     L.pf_verify_attention_workspace_size.restype = C.c_size_t
     L.pf_verify_attention_workspace_size.argtypes = [C.POINTER(pf_attn_desc)]
+    L.pf_verify_attention_launches.restype = C.c_int32
+    L.pf_verify_attention_launches.argtypes = [C.POINTER(pf_attn_desc)]
     L.pf_lmhead_accept_workspace_size.restype = C.c_size_t
     L.pf_lmhead_accept_workspace_size.argtypes = [C.POINTER(pf_lm_desc)]
     L.pf_lmhead_accept.restype = C.c_int
@@ -228,6 +230,10 @@ def pf_tree_prepare_device(parent: int, cu_nodes: int, batch: int, total_nodes: 
 
 def pf_verify_attention_workspace_size(desc: pf_attn_desc) -> int:
     return int(lib().pf_verify_attention_workspace_size(C.byref(desc)))
+
+
+def pf_verify_attention_launches(desc: pf_attn_desc) -> int:
+    return int(lib().pf_verify_attention_launches(C.byref(desc)))
 
 
 def pf_verify_attention(desc: pf_attn_desc, stream: int = 0) -> None:

@@ -108,7 +108,18 @@ pf_status check_cache_view(const pf_kv_view& c, int need_rows, const char* who) 
 // follows from the shape, unless the descriptor's launch fields ask for
 // something specific; nothing is read from the environment.
 // ---------------------------------------------------------------------------
-enum class AttnKernel { F32, MMA, TC64, TC128, PAIR, STREAM };
+enum class AttnKernel { F32, MMA, TC64, TC128, PAIR, STREAM, BATCH };
+
+// A distinct epoch for every call of a kernel that merges its own pieces
+// (the group tickets in the workspace compare it): 1 .. 2^40 - 1, wrapping.
+unsigned long long next_epoch() {
+  static std::atomic<unsigned long long> counter{0};
+  unsigned long long e;
+  do {
+    e = (counter.fetch_add(1, std::memory_order_relaxed) + 1) & ((1ull << 40) - 1);
+  } while (e == 0);
+  return e;
+}
 
 // kernel index 0..2: mma.sync BM 32/64/128
 int max_cluster_for(int kernel, int D, int want) {
@@ -192,6 +203,10 @@ pf_status choose_attention(const pf_attn_desc* d, pf::AttnArgs& a, int sms, bool
   const int pair_groups = a.B * a.Hkv * ((a.max_nodes + pair_nb - 1) / pair_nb);
   const int sk_nb = 128 / G;
   const int sk_groups = a.B * a.Hkv * ((a.max_nodes + sk_nb - 1) / sk_nb);
+  // The per-sequence balanced split: (sequence, KV head, 128-row block)
+  // groups, at most one CTA each per SM and within the plan's capacity.
+  const int batch_groups = a.B * a.Hkv * ((a.max_nodes + 128 / G - 1) / (128 / G));
+  const bool batch_fits = batch_groups <= std::min(sms, pf::kPlanMaxGroups);
   AttnKernel k;
   int a_bm_auto = 0;  // the automatic choice's rows per CTA for the 64-token kernel
   if (d->kernel == PF_ATTN_KERNEL_AUTO && d->rows_per_cta != 0) {
@@ -208,6 +223,13 @@ pf_status choose_attention(const pf_attn_desc* d, pf::AttnArgs& a, int sms, bool
     // continuous split balances the batch's loop, but its per-launch plan
     // (global round trips at kernel start, 5-9 us under the other CTAs'
     // prefetch) and the merge launch cost more than the imbalance it saves.
+    // The batch kernel (pieces in proportion to each sequence's tiles,
+    // merged by the last piece in the same launch) balances the 8-sequence
+    // batch's loop (at most 19 instead of 24 tiles per CTA) but measured
+    // 46.4 us (paged) and 34.5 us (contiguous cache) against 37.7 and 32.3
+    // for the clusters: its tile loads take longer under 152 one-CTA
+    // launches (2.1 against 1.6 us per paged 64 KB tile, the same DRAM
+    // bytes), and its last-piece merge adds ~5 us to the layer's tail.
     k = D != 128 ? AttnKernel::MMA : AttnKernel::TC64;  // may become TC128 below
     if (k == AttnKernel::TC64) a_bm_auto = 128;
   } else {
@@ -215,6 +237,7 @@ pf_status choose_attention(const pf_attn_desc* d, pf::AttnArgs& a, int sms, bool
         : d->kernel == PF_ATTN_KERNEL_TC64 ? AttnKernel::TC64
         : d->kernel == PF_ATTN_KERNEL_TC128 ? AttnKernel::TC128
         : d->kernel == PF_ATTN_KERNEL_PAIR  ? AttnKernel::PAIR
+        : d->kernel == PF_ATTN_KERNEL_BATCH ? AttnKernel::BATCH
                                             : AttnKernel::STREAM;
   }
   const int tiles64 = (a.max_prefix + 63) / 64 + (a.max_nodes + 63) / 64;
@@ -247,6 +270,20 @@ pf_status choose_attention(const pf_attn_desc* d, pf::AttnArgs& a, int sms, bool
     return PF_OK;
   }
 
+  if (k == AttnKernel::BATCH) {
+    if (!batch_fits)
+      return fail(PF_ERR_SHAPE, "%s: the batch kernel handles at most %d (sequence, KV head, "
+                  "128-row block) groups on this device", who, std::min(sms, pf::kPlanMaxGroups));
+    a.bm = 128;
+    a.nb = 128 / G;
+    a.rb_count = (a.max_nodes + a.nb - 1) / a.nb;
+    a.splits = 1;
+    a.items = sms;  // one CTA per SM
+    a.slots = 1;
+    out->ws_need = pf::attention_balanced_ws_bytes(a.items, a.bm, D, 1);
+    out->kernel = k;
+    return PF_OK;
+  }
   if (k == AttnKernel::STREAM) {
     if (sk_groups > pf::kSkMaxGroups)
       return fail(PF_ERR_SHAPE, "%s: the continuous-split kernel handles at most %d (sequence, "
@@ -329,20 +366,25 @@ pf_status attention_args(const pf_attn_desc* d, pf::AttnArgs& a, const char* who
   if (d->flags & ~(PF_ATTN_EARLY_PREFETCH | PF_ATTN_NO_PDL))
     return fail(PF_ERR_SHAPE, "%s: unknown flags 0x%x", who, d->flags);
   // launch fields
-  if (d->kernel < PF_ATTN_KERNEL_AUTO || d->kernel > PF_ATTN_KERNEL_STREAM)
+  if (d->kernel < PF_ATTN_KERNEL_AUTO || d->kernel > PF_ATTN_KERNEL_BATCH)
     return fail(PF_ERR_SHAPE, "%s: unknown kernel %d", who, d->kernel);
   if (d->dtype == PF_F32 && (d->kernel != PF_ATTN_KERNEL_AUTO || d->splits != 0 ||
                              d->rows_per_cta != 0 || d->stages != 0))
     return fail(PF_ERR_DTYPE, "%s: the fp32 path has one kernel and takes no launch fields",
                 who);
   const bool tc_kernel = d->kernel == PF_ATTN_KERNEL_TC64 || d->kernel == PF_ATTN_KERNEL_TC128 ||
-                         d->kernel == PF_ATTN_KERNEL_PAIR || d->kernel == PF_ATTN_KERNEL_STREAM;
+                         d->kernel == PF_ATTN_KERNEL_PAIR || d->kernel == PF_ATTN_KERNEL_STREAM ||
+                         d->kernel == PF_ATTN_KERNEL_BATCH;
   if (tc_kernel && D != 128)
     return fail(PF_ERR_SHAPE, "%s: the tcgen05 kernels need head_dim 128", who);
   if (d->splits < 0 || d->splits > 16 ||
-      ((d->kernel == PF_ATTN_KERNEL_PAIR || d->kernel == PF_ATTN_KERNEL_STREAM) && d->splits != 0))
+      ((d->kernel == PF_ATTN_KERNEL_PAIR || d->kernel == PF_ATTN_KERNEL_STREAM ||
+        d->kernel == PF_ATTN_KERNEL_BATCH) &&
+       d->splits != 0))
     return fail(PF_ERR_SHAPE,
-                "%s: splits must be 0 (automatic) or 1..16, and 0 for the continuous split", who);
+                "%s: splits must be 0 (automatic) or 1..16, and 0 for the kernels that split "
+                "by the plan",
+                who);
   if (d->rows_per_cta != 0 &&
       ((d->rows_per_cta != 128 && d->rows_per_cta != 256) || D != 128 ||
        (d->kernel != PF_ATTN_KERNEL_AUTO && d->kernel != PF_ATTN_KERNEL_TC64) ||
@@ -411,7 +453,7 @@ extern "C" {
 
 const char* pf_last_error(void) { return g_last_error.c_str(); }
 
-int32_t pf_version(void) { return 200; }
+int32_t pf_version(void) { return 201; }
 
 pf_status pf_tree_prepare(const int32_t* parent, int32_t n_nodes, int32_t* depth_out,
                           uint64_t* mask_out) {
@@ -478,6 +520,23 @@ size_t pf_verify_attention_workspace_size(const pf_attn_desc* d) {
   return ok ? ch.ws_need : 0;
 }
 
+int32_t pf_verify_attention_launches(const pf_attn_desc* d) {
+  if (!d) return 0;
+  const std::string saved = g_last_error;  // a query leaves the last error alone
+  pf::AttnArgs a = {};
+  AttnChoice ch;
+  const int sms = num_sms();
+  const bool ok = sms > 0 && attention_args(d, a, "") == PF_OK &&
+                  choose_attention(d, a, sms, d->workspace != nullptr, &ch, "") == PF_OK;
+  g_last_error = saved;
+  if (!ok) return 0;
+  if ((ch.kernel == AttnKernel::PAIR || ch.kernel == AttnKernel::STREAM ||
+       ch.kernel == AttnKernel::BATCH) &&
+      !d->workspace)
+    return 0;
+  return a.items > 0 && ch.kernel != AttnKernel::BATCH ? 2 : 1;
+}
+
 pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
   static const char* who = "pf_verify_attention";
   if (!d) return fail(PF_ERR_NULL, "%s: desc is NULL", who);
@@ -521,7 +580,9 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
     cudaError_t e = pf::launch_attention_f32(a, s, pdl);
     return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
   }
-  if ((ch.kernel == AttnKernel::PAIR || ch.kernel == AttnKernel::STREAM) && !d->workspace)
+  if ((ch.kernel == AttnKernel::PAIR || ch.kernel == AttnKernel::STREAM ||
+       ch.kernel == AttnKernel::BATCH) &&
+      !d->workspace)
     return fail(PF_ERR_WORKSPACE, "%s: this kernel needs the workspace (%zu bytes)", who,
                 ch.ws_need);
   if (a.items > 0) {
@@ -534,7 +595,8 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
   // Tensor maps: K/V boxes of the chosen kernel's tile (the pair kernel
   // loads half a tile per CTA: 64 K rows, 128 V rows of 64 columns).
   const bool pair = ch.kernel == AttnKernel::PAIR;
-  const bool wide = ch.kernel == AttnKernel::TC128 || ch.kernel == AttnKernel::STREAM;
+  const bool wide = ch.kernel == AttnKernel::TC128 || ch.kernel == AttnKernel::STREAM ||
+                    ch.kernel == AttnKernel::BATCH;
   const cuuint32_t k_rows = pair ? 64 : wide ? 128 : 64;
   const cuuint32_t v_rows = pair ? 128 : k_rows;
   const cuuint32_t q_nodes = pair ? (cuuint32_t)(a.nb / 2) : (cuuint32_t)a.nb;
@@ -573,11 +635,16 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
   switch (ch.kernel) {
     case AttnKernel::PAIR: e = pf::launch_attention_pair(a, m, s, pdl); break;
     case AttnKernel::STREAM: e = pf::launch_attention_sk(a, m, s, pdl); break;
-    case AttnKernel::TC128: e = pf::launch_attention_tc2(a, m, s, pdl, ch.stages); break;
+    case AttnKernel::TC128: e = pf::launch_attention_tc2(a, m, s, pdl, ch.stages, false); break;
+    case AttnKernel::BATCH:
+      a.epoch = next_epoch();
+      e = pf::launch_attention_tc2(a, m, s, pdl, 3, true);
+      break;
     case AttnKernel::TC64: e = pf::launch_attention_tc(a, m, s, pdl); break;
     default: e = pf::launch_attention_bf16(a, m, s, sms, pdl); break;
   }
-  if (e == cudaSuccess && a.items > 0) e = pf::launch_attention_combine(a, s, pdl);
+  if (e == cudaSuccess && a.items > 0 && ch.kernel != AttnKernel::BATCH)
+    e = pf::launch_attention_combine(a, s, pdl);
   return e == cudaSuccess ? PF_OK : cuda_fail(e, who);
 }
 

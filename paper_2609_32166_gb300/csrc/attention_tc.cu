@@ -658,7 +658,8 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const AttnArgs a) {
 }  // namespace
 
 size_t attention_balanced_ws_bytes(int items, int bm, int D, int slots) {
-  return (size_t)items * slots * bm * (D + 8) * 2 + kPlanMaxGroups * sizeof(int4);
+  return (size_t)items * slots * bm * (D + 8) * 2 + kPlanMaxGroups * sizeof(int4) +
+         kPlanMaxGroups * sizeof(unsigned long long);
 }
 
 cudaError_t launch_attention_combine(const AttnArgs& a, cudaStream_t s, bool pdl) {

@@ -19,6 +19,15 @@
 //              more than 2^8; at the end O / l and the log2-sum-exp go to the
 //              merge, as in attn_tc_kernel.
 //
+// Work split: a cluster of a.splits CTAs per (sequence, KV head, row block)
+// group, each taking a contiguous slice of the group's tiles, merged through
+// distributed shared memory; or (BAL, a batch with the workspace) one CTA per
+// SM and no cluster, each group spread over as many CTAs as its share of all
+// tiles calls for (balanced_plan: the groups of one sequence get equal
+// pieces, so the CTAs of its KV heads and row blocks read the same pages at
+// the same time), each piece leaving a normalised partial in the workspace
+// and the last piece of a group to finish merging them (group tickets).
+//
 // TMEM columns: S[0] 0..127, S[1] 128..255, O 256..383, P[0] 384..447,
 // P[1] 448..511.
 #include <cuda_fp16.h>
@@ -58,7 +67,10 @@ struct W2Smem {
   static constexpr int kBarOff = kLateInbox ? kQEnd : kInboxOff + kInboxSlots * kRowBytes;
   // kv_full[S] kv_empty[S] q_full s_full[2] s_empty[2] p_full[2] pv_done[2] inbox
   static constexpr int kNumBars = 2 * STAGES + 1 + 8 + 1;
-  static constexpr int kTotal = kBarOff + kNumBars * 8 + 16;
+  // then the TMEM address (16 bytes), the balanced mode's plan entry (an
+  // int4) and its last-piece flag
+  static constexpr int kPlanOff = kBarOff + kNumBars * 8 + 16;
+  static constexpr int kTotal = kPlanOff + 32;
   static_assert(128 * kRowBytes <= kStageBytes, "staged rows fit in the ring's first stage");
   static_assert(!kLateInbox || kInboxOff + kInboxSlots * kRowBytes <= kQOff, "inbox fits in the ring");
   static_assert(kTotal + 1024 <= 232448, "shared memory budget");
@@ -123,7 +135,7 @@ __device__ __forceinline__ void umma_bf16_tmem_a(uint32_t d_tmem, uint32_t a_tme
       : "memory");
 }
 
-template <int STAGES>
+template <int STAGES, bool BAL>
 __global__ void __launch_bounds__(kW2Threads, 1)
     attn_tc2_kernel(const __grid_constant__ CUtensorMap tm_q,
                     const __grid_constant__ CUtensorMap tm_tk,
@@ -158,7 +170,26 @@ __global__ void __launch_bounds__(kW2Threads, 1)
   const bool early = (a.flags & PF_ATTN_EARLY_PREFETCH) != 0;
   if (!early) pdl_wait();
 
-  const int group = blockIdx.x / nsplit;
+  // This CTA's group and its piece of the group's tiles: split `split` of
+  // the cluster, or (BAL) the item the plan gives it.
+  int group = blockIdx.x / nsplit, part = split, nparts = nsplit, first_item = 0;
+  int4* plan_slot = reinterpret_cast<int4*>(smem + S::kPlanOff);
+  if constexpr (BAL) {
+    if (warp == 0) {
+      const PlanItem it = balanced_plan(a, (int)blockIdx.x, -1, nullptr, kW);
+      if (lane == 0) *plan_slot = make_int4(it.group, it.j, it.k, it.first);
+    }
+    __syncthreads();
+    const int4 pi = *plan_slot;
+    if (pi.x < 0) {
+      if (early) pdl_wait();  // the grid completes only after the preceding kernel
+      return;                 // uniform over the CTA: no work for this item
+    }
+    group = pi.x;
+    part = pi.y;
+    nparts = pi.z;
+    first_item = pi.w;
+  }
   const int rb = group % a.rb_count;
   const int g = (group / a.rb_count) % a.Hkv;
   const int b = group / (a.rb_count * a.Hkv);
@@ -178,8 +209,9 @@ __global__ void __launch_bounds__(kW2Threads, 1)
   const int ntiles = n_ptiles + n_qtiles;
   // Split s takes tiles [t_begin, t_end) of the order (proposal tiles,
   // prefix tiles), and processes its prefix tiles first (as in attn_tc_kernel).
-  const int t_begin = (int)((long long)ntiles * split / nsplit);
-  const int t_end = (int)((long long)ntiles * (split + 1) / nsplit);
+  // (BAL: piece `part` of the group's `nparts`)
+  const int t_begin = (int)((long long)ntiles * part / nparts);
+  const int t_end = (int)((long long)ntiles * (part + 1) / nparts);
   const int my_tiles = t_end - t_begin;
   const int pre_lo = max(t_begin, n_qtiles);
   const int my_ptiles = max(0, t_end - pre_lo);
@@ -454,14 +486,34 @@ __global__ void __launch_bounds__(kW2Threads, 1)
   const float inv_l = (my_tiles > 0 && l > 0.f) ? 1.f / l : 0.f;
 
   if (nsplit == 1) {
-    // ---- single split: O / l is the output
+    // ---- single split: O / l is the output -- or (BAL, a group spread over
+    // several CTAs) this piece's normalised partial and log2-sum-exp
+    const bool piece = BAL && nparts > 1;
     if (has_row) {
       uint32_t ov[D];
 #pragma unroll
       for (int c0 = 0; c0 < D; c0 += 32)
         tmem_ld_32(o_addr + c0, *reinterpret_cast<uint32_t(*)[32]>(&ov[c0]));
       tmem_ld_wait();
-      if (r < rows) {
+      if (piece && r < rows) {
+        if (!(inv_l > 0.f)) {
+          // no column reached this row in this piece: 0 with lse = -inf
+#pragma unroll
+          for (int c = 0; c < D; ++c) ov[c] = 0u;
+        }
+        __half* dst = reinterpret_cast<__half*>(a.ws) + ((size_t)blockIdx.x * a.bm + r) * S::kPitch;
+#pragma unroll
+        for (int c = 0; c < D; c += 8) {
+          uint4 pk;
+          pk.x = pack_half(__uint_as_float(ov[c]) * inv_l, __uint_as_float(ov[c + 1]) * inv_l);
+          pk.y = pack_half(__uint_as_float(ov[c + 2]) * inv_l, __uint_as_float(ov[c + 3]) * inv_l);
+          pk.z = pack_half(__uint_as_float(ov[c + 4]) * inv_l, __uint_as_float(ov[c + 5]) * inv_l);
+          pk.w = pack_half(__uint_as_float(ov[c + 6]) * inv_l, __uint_as_float(ov[c + 7]) * inv_l);
+          *reinterpret_cast<uint4*>(dst + c) = pk;
+        }
+        *reinterpret_cast<float*>(dst + D) = inv_l > 0.f ? m_ref + __log2f(l) : -INFINITY;
+        __threadfence();  // before this piece's ticket (after the barrier below)
+      } else if (r < rows) {
         const int node = node0 + nfirst + r / a.G;
         const int h = g * a.G + r % a.G;
         __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(a.out) + ((size_t)node * a.Hq + h) * D;
@@ -481,6 +533,41 @@ __global__ void __launch_bounds__(kW2Threads, 1)
     if (warp == 1) {
       tc_fence_after();
       tmem_dealloc(tmem, kW2TmemCols);
+    }
+    if (piece) {
+      // the group's last piece to arrive merges every piece's partial
+      int* last_slot = reinterpret_cast<int*>(plan_slot + 1);
+      if (tid == 0)
+        *last_slot = ticket_arrive_last(&group_tickets(a)[group], a.epoch, nparts, a.err) ? 1 : 0;
+      __syncthreads();
+      if (*last_slot) {
+        __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.out);
+        // The pieces' partials sit in consecutive slots: as many as the idle
+        // ring holds come in with one bulk copy (one L2 round trip instead of
+        // one per merged row); more are merged straight from L2.
+        constexpr int kSlotBytes = 128 * S::kRowBytes;  // a.bm = 128 rows
+        constexpr int kStaged = STAGES * S::kStageBytes / kSlotBytes;
+        if (nparts <= kStaged) {
+          if (tid == 0) {
+            fence_proxy_async_global();  // the pieces' stores, acquired above, before the copy
+            const uint32_t bytes = (uint32_t)(nparts * kSlotBytes);
+            mbar_arrive_expect_tx(smem_u32(inbox_full), bytes);
+            bulk_load_g2s(smem_u32(smem),
+                          static_cast<const uint8_t*>(a.ws) + (size_t)first_item * kSlotBytes,
+                          bytes, smem_u32(inbox_full));
+          }
+          if (mbar_wait(smem_u32(inbox_full), 0, a.err))
+            merge_rows_smem<D, kStaged>(a, smem, S::kRowBytes, kSlotBytes, nparts, rows, 0,
+                                        node0 + nfirst, g, tid, kW2Threads);
+        } else {
+          for (int it = tid; it < rows * (D / 8); it += kW2Threads) {
+            const int rr = it / (D / 8), c8 = it % (D / 8);
+            const int node = node0 + nfirst + rr / a.G;
+            const int h = g * a.G + rr % a.G;
+            merge_pieces_row<D>(a, first_item, nparts, rr, c8, out + ((size_t)node * a.Hq + h) * D);
+          }
+        }
+      }
     }
     return;
   }
@@ -563,8 +650,9 @@ template <int STAGES>
 static int tc2_max_active_clusters_impl(int cluster) {
   const int smem = tc2_smem_bytes<STAGES>();
   static DeviceMemo limit;
-  if (ensure_smem_limit((const void*)attn_tc2_kernel<STAGES>, smem, limit) != cudaSuccess) return 0;
-  if (cluster > 8 && cudaFuncSetAttribute(attn_tc2_kernel<STAGES>,
+  if (ensure_smem_limit((const void*)attn_tc2_kernel<STAGES, false>, smem, limit) != cudaSuccess)
+    return 0;
+  if (cluster > 8 && cudaFuncSetAttribute(attn_tc2_kernel<STAGES, false>,
                                           cudaFuncAttributeNonPortableClusterSizeAllowed,
                                           1) != cudaSuccess)
     return 0;
@@ -580,27 +668,32 @@ static int tc2_max_active_clusters_impl(int cluster) {
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, attn_tc2_kernel<STAGES>, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, attn_tc2_kernel<STAGES, false>, &cfg) != cudaSuccess) {
     cudaGetLastError();
     return 0;
   }
   return n;
 }
 
-template <int STAGES>
+template <int STAGES, bool BAL>
 static cudaError_t launch_tc2(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl) {
   const int smem = tc2_smem_bytes<STAGES>();
   static DeviceMemo limit;
   static DeviceMemo nonportable;
-  cudaError_t e = ensure_smem_limit((const void*)attn_tc2_kernel<STAGES>, smem, limit);
+  cudaError_t e = ensure_smem_limit((const void*)attn_tc2_kernel<STAGES, BAL>, smem, limit);
   if (e != cudaSuccess) return e;
+  if (BAL) {
+    // one CTA per item, no cluster
+    return launch_ex(attn_tc2_kernel<STAGES, BAL>, dim3(a.items), dim3(kW2Threads), smem, s, 1,
+                     pdl, m.q, m.tk, m.tv, m.ck, m.cv, a);
+  }
   if (a.splits > 8) {
-    e = ensure_nonportable_cluster((const void*)attn_tc2_kernel<STAGES>, nonportable);
+    e = ensure_nonportable_cluster((const void*)attn_tc2_kernel<STAGES, BAL>, nonportable);
     if (e != cudaSuccess) return e;
   }
   const dim3 grid(a.B * a.Hkv * a.rb_count * a.splits);
-  return launch_ex(attn_tc2_kernel<STAGES>, grid, dim3(kW2Threads), smem, s, a.splits, pdl, m.q,
-                   m.tk, m.tv, m.ck, m.cv, a);
+  return launch_ex(attn_tc2_kernel<STAGES, BAL>, grid, dim3(kW2Threads), smem, s, a.splits, pdl,
+                   m.q, m.tk, m.tv, m.ck, m.cv, a);
 }
 
 // Ring depth: 3 stages (inbox in the ring, peers send after every CTA of
@@ -611,8 +704,9 @@ int attention_tc2_max_active_clusters(int cluster, int stages) {
 }
 
 cudaError_t launch_attention_tc2(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl,
-                                 int stages) {
-  return stages == 2 ? launch_tc2<2>(a, m, s, pdl) : launch_tc2<3>(a, m, s, pdl);
+                                 int stages, bool balanced) {
+  if (balanced) return launch_tc2<3, true>(a, m, s, pdl);
+  return stages == 2 ? launch_tc2<2, false>(a, m, s, pdl) : launch_tc2<3, false>(a, m, s, pdl);
 }
 
 }  // namespace pf

@@ -246,6 +246,99 @@ __device__ __forceinline__ int4* plan_table(const AttnArgs& a) {
                                  (size_t)a.items * a.slots * a.bm * (a.D + 8) * 2);
 }
 
+// One 64-bit arrival ticket per group after the plan table, for the kernels
+// that merge a spread group's pieces themselves (the last piece to finish
+// merges).  A ticket holds (call epoch << 24 | pieces arrived); a ticket
+// whose epoch is not this call's counts as 0, so the workspace needs no
+// initialisation, and the last piece resets the count to 0, so a captured
+// launch replayed with the same epoch starts from 0 again.
+__device__ __forceinline__ unsigned long long* group_tickets(const AttnArgs& a) {
+  return reinterpret_cast<unsigned long long*>(plan_table(a) + kPlanMaxGroups);
+}
+
+// One thread per piece, after every write of the piece's partial is ordered
+// before it (writers' __threadfence + a CTA barrier): true for the piece
+// that completes the group.  Each failed compare-and-swap means another
+// piece's arrival succeeded, so the loop ends after at most k rounds; it is
+// bounded all the same.
+__device__ __forceinline__ bool ticket_arrive_last(unsigned long long* ticket,
+                                                   unsigned long long epoch, int k, int32_t* err) {
+  constexpr unsigned long long kCount = (1ull << 24) - 1;
+  unsigned long long old = atomicAdd(ticket, 0ull);
+  for (int round = 0; round < 4096; ++round) {
+    const unsigned long long cnt = (old >> 24) == epoch ? (old & kCount) : 0ull;
+    const bool last = (int)cnt + 1 == k;
+    const unsigned long long want = (epoch << 24) | (last ? 0ull : cnt + 1);
+    const unsigned long long seen = atomicCAS(ticket, old, want);
+    if (seen == old) {
+      __threadfence();  // the other pieces' partials are visible to this CTA
+      return last;
+    }
+    old = seen;
+  }
+  flag_error(err, PF_DEVERR_TIMEOUT);
+  return false;
+}
+
+// Merge of group pieces' partials from global memory (the format of
+// attn_tc_kernel's staged rows: fp16 O / l, then the log2-sum-exp as a float
+// in the row's pad, pitch D + 8 halves): row r, output columns c8*8 ..
+// c8*8+7, pieces in slots first .. first + k - 1 of bm rows each, read past
+// L1 (other CTAs wrote them during this launch).  Batches of 8 pieces, all
+// loads of a batch in flight together, folded into a running maximum.
+//   out = sum_j 2^(lse_j - M) (O/l)_j / sum_j 2^(lse_j - M),  M = max_j lse_j
+template <int D>
+__device__ __forceinline__ void merge_pieces_row(const AttnArgs& a, int first, int k, int r,
+                                                 int c8, __nv_bfloat16* dst) {
+  constexpr int kPitch = D + 8, kBatch = 8;
+  const __half* base = reinterpret_cast<const __half*>(a.ws) + (size_t)r * kPitch;
+  const size_t slot_stride = (size_t)a.bm * kPitch;
+  float M = -INFINITY, W = 0.f;
+  float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  for (int j0 = 0; j0 < k; j0 += kBatch) {
+    float ls[kBatch];
+    uint4 v[kBatch];
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      ls[u] = -INFINITY;
+      if (j0 + u < k) {
+        const __half* row = base + (size_t)(first + j0 + u) * slot_stride;
+        ls[u] = __ldcg(reinterpret_cast<const float*>(row + D));
+        v[u] = __ldcg(reinterpret_cast<const uint4*>(row + c8 * 8));
+      }
+    }
+    float Mb = M;
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) Mb = fmaxf(Mb, ls[u]);
+    if (Mb == -INFINITY) continue;  // nothing reached this row yet
+    const float sc = M == -INFINITY ? 0.f : ex2_approx(M - Mb);
+    W *= sc;
+#pragma unroll
+    for (int c = 0; c < 8; ++c) acc[c] *= sc;
+    M = Mb;
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      if (ls[u] == -INFINITY) continue;  // absent or empty partial
+      const float w = ex2_approx(ls[u] - M);
+      W += w;
+      const __half2* h2 = reinterpret_cast<const __half2*>(&v[u]);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const float2 f = __half22float2(h2[c]);
+        acc[2 * c] = fmaf(w, f.x, acc[2 * c]);
+        acc[2 * c + 1] = fmaf(w, f.y, acc[2 * c + 1]);
+      }
+    }
+  }
+  const float inv = W > 0.f ? __fdividef(1.f, W) : 0.f;
+  uint4 pk;
+  pk.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+  pk.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+  pk.z = pack_bf16(acc[4] * inv, acc[5] * inv);
+  pk.w = pack_bf16(acc[6] * inv, acc[7] * inv);
+  *reinterpret_cast<uint4*>(dst + c8 * 8) = pk;
+}
+
 // Warp-collective (all 32 lanes, warp-uniform arguments): the plan entry
 // of item `item`, and in *grp that of group `group` (j = 0) if group >= 0.
 static __device__ __noinline__ PlanItem balanced_plan(const AttnArgs& a, int item, int group,
@@ -529,14 +622,88 @@ __device__ __forceinline__ void inbox_merge_n(const AttnArgs& a, const __half* i
   }
 }
 
+// The same merge for k <= kMaxK pieces held in shared memory, latency-lean:
+// a unit is (row, a quarter of its 8-column chunks); the unit's k
+// log-sum-exps are read once and turned into normalised weights, then its
+// four chunks' loads of every piece are all issued before any is used (the
+// one-CTA-per-SM kernels run 6 warps, too few to hide one load-use chain
+// per output chunk).  Piece j of local row i is at base + j * slot_stride +
+// i * row_pitch (bytes): fp16 O / l, then the float log2-sum-exp at byte
+// 2 * D.  Local row i is output row row0 + i of the group.
+template <int D, int kMaxK>
+__device__ __forceinline__ void merge_rows_smem(const AttnArgs& a, const uint8_t* base,
+                                                int row_pitch, int slot_stride, int k, int nrows,
+                                                int row0, int node_base, int g, int tid,
+                                                int nthreads) {
+  constexpr int C8 = D / 8, kQ = 4, kPer = C8 / kQ;  // 4 chunks per unit
+  __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.out);
+  for (int u = tid; u < nrows * kQ; u += nthreads) {
+    const int i = u / kQ, q = u % kQ;
+    const uint8_t* row = base + i * row_pitch;
+    float w[kMaxK];
+    float M = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < kMaxK; ++j) {
+      w[j] = j < k ? *reinterpret_cast<const float*>(row + j * slot_stride + 2 * D) : -INFINITY;
+      M = fmaxf(M, w[j]);
+    }
+    const float Mu = M == -INFINITY ? 0.f : M;
+    float W = 0.f;
+#pragma unroll
+    for (int j = 0; j < kMaxK; ++j) {
+      w[j] = w[j] == -INFINITY ? 0.f : ex2_approx(w[j] - Mu);  // absent or empty: 0
+      W += w[j];
+    }
+    const float inv = W > 0.f ? __fdividef(1.f, W) : 0.f;
+    uint4 v[kPer][kMaxK];
+#pragma unroll
+    for (int c = 0; c < kPer; ++c)
+#pragma unroll
+      for (int j = 0; j < kMaxK; ++j)
+        if (w[j] != 0.f)
+          v[c][j] = *reinterpret_cast<const uint4*>(row + j * slot_stride + (q * kPer + c) * 16);
+    const int r = row0 + i;
+    const int node = node_base + r / a.G;
+    const int h = g * a.G + r % a.G;
+    uint4* dst = reinterpret_cast<uint4*>(out + ((size_t)node * a.Hq + h) * D) + q * kPer;
+#pragma unroll
+    for (int c = 0; c < kPer; ++c) {
+      float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int j = 0; j < kMaxK; ++j) {
+        if (w[j] == 0.f) continue;  // its O may hold anything (0 * NaN)
+        const __half2* h2 = reinterpret_cast<const __half2*>(&v[c][j]);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 f = __half22float2(h2[e]);
+          acc[2 * e] = fmaf(w[j], f.x, acc[2 * e]);
+          acc[2 * e + 1] = fmaf(w[j], f.y, acc[2 * e + 1]);
+        }
+      }
+      uint4 pk;
+      pk.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+      pk.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+      pk.z = pack_bf16(acc[4] * inv, acc[5] * inv);
+      pk.w = pack_bf16(acc[6] * inv, acc[7] * inv);
+      dst[c] = pk;
+    }
+  }
+}
+
 template <int D, int kThreads, int kPitch>
 __device__ __forceinline__ void inbox_merge(const AttnArgs& a, const __half* inbox, int rows,
                                             int split, int per, int nsplit, int node_base, int g,
                                             int tid) {
+  // up to 4 peers: the latency-lean unit merge; wider clusters have few rows
+  // per CTA and keep one thread per (row, chunk)
+  const int cnt = max(0, min(per, rows - split * per));
+  const uint8_t* base = reinterpret_cast<const uint8_t*>(inbox);
   if (nsplit <= 2)
-    inbox_merge_n<D, kThreads, kPitch, 2>(a, inbox, rows, split, per, nsplit, node_base, g, tid);
+    merge_rows_smem<D, 2>(a, base, kPitch * 2, per * kPitch * 2, nsplit, cnt, split * per,
+                          node_base, g, tid, kThreads);
   else if (nsplit <= 4)
-    inbox_merge_n<D, kThreads, kPitch, 4>(a, inbox, rows, split, per, nsplit, node_base, g, tid);
+    merge_rows_smem<D, 4>(a, base, kPitch * 2, per * kPitch * 2, nsplit, cnt, split * per,
+                          node_base, g, tid, kThreads);
   else if (nsplit <= 8)
     inbox_merge_n<D, kThreads, kPitch, 8>(a, inbox, rows, split, per, nsplit, node_base, g, tid);
   else

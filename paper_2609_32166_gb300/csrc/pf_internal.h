@@ -31,6 +31,9 @@ struct AttnArgs {
   // kernel's continuous split: an item's first and last group piece)
   int slots;
   void* ws;
+  // this call's epoch for the group tickets of the kernels that merge their
+  // own pieces (see group_tickets): distinct for every call, < 2^40
+  unsigned long long epoch;
   float scale_log2;  // softmax scale * log2(e)
   float scale;
   const int32_t* cu_nodes;
@@ -65,10 +68,14 @@ bool attention_cluster_fits(int D, int bm, int cluster);
 // tcgen05 variant (bf16, D = 128, a.bm = 128 or 256 query rows per CTA).
 cudaError_t launch_attention_tc(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl);
 // tcgen05 variant with 128-token K/V tiles and P in tensor memory (bf16,
-// D = 128, a.bm = 128, cluster split-KV only); its tensor maps hold
-// 128-row cache boxes and 128-node proposal boxes.
+// D = 128, a.bm = 128); its tensor maps hold 128-row cache boxes and
+// 128-node proposal boxes.  Cluster split-KV (a.items = 0), or with
+// `balanced` one CTA per item (a.items = SMs, a.slots = 1, no cluster):
+// groups spread over CTAs in proportion to their tiles (balanced_plan), the
+// last piece of a group to finish merging the pieces' partials from the
+// workspace (group tickets, a.epoch); no combine kernel.
 cudaError_t launch_attention_tc2(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl,
-                                 int stages);
+                                 int stages, bool balanced);
 int attention_tc2_max_active_clusters(int cluster, int stages);
 // tcgen05 variant on SM pairs (2-SM MMA, M = 256 rows per pair, 128-token
 // tiles; bf16, D = 128): a.bm = 256, a.nb = 2 * floor(128 / G) nodes per
@@ -90,7 +97,8 @@ cudaError_t launch_attention_combine(const AttnArgs& a, cudaStream_t s, bool pdl
 // hold (8 per lane of a warp).
 constexpr int kPlanMaxGroups = 256;
 // Bytes of a.ws for the balanced batch mode with `items` work items of a.bm
-// rows and `slots` partial slots per item.
+// rows and `slots` partial slots per item: the partials, the plan table
+// (kPlanMaxGroups int4) and the group tickets (kPlanMaxGroups u64).
 size_t attention_balanced_ws_bytes(int items, int bm, int D, int slots = 1);
 // How many clusters of `cluster` CTAs of the tcgen05 kernel fit at once.
 // rows_per_cta: 128 (one softmax warpgroup) or 256 (two).

@@ -277,8 +277,9 @@ class VerifyStep:
         pb.pf_kv_commit(self.commit_desc, s)
 
     def launches_per_step(self) -> int:
-        # the attention call launches a second (merge) kernel when it has a workspace
-        return self.L * (2 if self.attn_ws is not None else 1) + 2
+        # what each attention call launches (one kernel, or two with a separate
+        # merge), the LM head, the commit
+        return sum(pb.pf_verify_attention_launches(d) for d in self.attn_descs) + 2
 
     # ------------------------------------------------------------------ results
     def results(self) -> dict:

@@ -131,8 +131,12 @@ def _attn_desc(**kw):
           max_prefix_len=17), pb.PF_ERR_CAPACITY),
     (dict(q=0x10008), pb.PF_ERR_ALIGN),
     # launch fields
-    (dict(kernel=6), pb.PF_ERR_SHAPE),
+    (dict(kernel=7), pb.PF_ERR_SHAPE),
     (dict(kernel=pb.PF_ATTN_KERNEL_STREAM, splits=2), pb.PF_ERR_SHAPE),
+    (dict(kernel=pb.PF_ATTN_KERNEL_BATCH, splits=2), pb.PF_ERR_SHAPE),
+    (dict(kernel=pb.PF_ATTN_KERNEL_BATCH, head_dim=64), pb.PF_ERR_SHAPE),
+    (dict(kernel=pb.PF_ATTN_KERNEL_BATCH, stages=2), pb.PF_ERR_SHAPE),
+    (dict(kernel=pb.PF_ATTN_KERNEL_BATCH, rows_per_cta=128), pb.PF_ERR_SHAPE),
     (dict(kernel=-1), pb.PF_ERR_SHAPE),
     (dict(kernel=pb.PF_ATTN_KERNEL_PAIR, splits=9), pb.PF_ERR_SHAPE),
     (dict(kernel=pb.PF_ATTN_KERNEL_TC64, splits=17), pb.PF_ERR_SHAPE),

@@ -16,6 +16,7 @@ TC64 = dict(kernel=pb.PF_ATTN_KERNEL_TC64)
 TC128 = dict(kernel=pb.PF_ATTN_KERNEL_TC128)
 PAIR = dict(kernel=pb.PF_ATTN_KERNEL_PAIR)
 STREAM = dict(kernel=pb.PF_ATTN_KERNEL_STREAM)
+BATCH = dict(kernel=pb.PF_ATTN_KERNEL_BATCH)
 
 pytestmark = pytest.mark.gpu
 
@@ -152,11 +153,13 @@ def test_pair_kernel_many_groups():
     c.check_commit(res)
 
 
-@pytest.mark.parametrize("kernel", ["pair", "stream"])
+@pytest.mark.parametrize("kernel", ["pair", "stream", "batch"])
 def test_continuous_split_needs_the_workspace(kernel):
     c = Case(SMALL["7b-tree64-small"], seed=16, balanced=False)
     d = c.vs.attn_descs[0]
-    d.kernel = pb.PF_ATTN_KERNEL_PAIR if kernel == "pair" else pb.PF_ATTN_KERNEL_STREAM
+    d.kernel = {"pair": pb.PF_ATTN_KERNEL_PAIR, "stream": pb.PF_ATTN_KERNEL_STREAM,
+                "batch": pb.PF_ATTN_KERNEL_BATCH}[kernel]
+    assert pb.pf_verify_attention_launches(d) == 0
     with pytest.raises(pb.PfError) as e:
         pb.pf_verify_attention(d, 0)
     assert e.value.status == pb.PF_ERR_WORKSPACE
@@ -210,6 +213,78 @@ def test_stream_kernel_many_groups():
         c.check_attention(0, s)
     c.check_lmhead(res)
     c.check_commit(res)
+
+
+# ---------------------------------------------------------------------------
+# the batch kernel (128-token tiles, one CTA per SM, each group spread over
+# CTAs in proportion to its tiles, the last piece merging in the kernel)
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("name", sorted(EDGE_STREAM))
+def test_batch_kernel_edges(name):
+    c = Case(EDGE_STREAM[name], seed=6, attn_launch=BATCH)
+    assert c.vs.launches_per_step() == c.L + 2  # no merge kernel
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for l in range(c.L):
+        for s in range(c.w.batch):
+            c.check_attention(l, s)
+    c.check_lmhead(res)
+    c.check_commit(res)
+
+
+@pytest.mark.parametrize("name", ["2b-chain16-small", "7b-tree64-small", "7b-32k-tree128-small",
+                                  "7b-batch8-paged-small"])
+def test_batch_kernel_shapes(name):
+    """Every node: single sequences (a group's tiles spread over up to all
+    SMs, many pieces per merge) and the paged batch."""
+    c = Case(SMALL[name], seed=19, attn_launch=BATCH)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for l in range(c.L):
+        for s in range(c.w.batch):
+            c.check_attention(l, s)
+
+
+def test_batch_kernel_many_groups():
+    """144 groups (36 sequences x 4 KV heads, 252 proposal rows) of 1..9
+    tiles on the SMs: most groups whole on one CTA, the longest in pieces."""
+    w = I.scaled(W["7b-bf16-batch8-paged"], layers=1, batch=36, prefix=(20, 900), nodes=7,
+                 max_depth=5, vocab=300, hidden=64)
+    c = Case(w, seed=20, attn_launch=BATCH)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for s in range(w.batch):
+        c.check_attention(0, s)
+    c.check_lmhead(res)
+    c.check_commit(res)
+
+
+def test_batch_kernel_tickets_need_no_initialisation():
+    """A workspace full of 0xff bytes (and one left by other calls), then a
+    CUDA graph of the layer replayed three times with the same epoch: every
+    result equals the eager call's (the last piece resets its ticket)."""
+    c = Case(SMALL["7b-batch8-paged-small"], seed=21, attn_launch=BATCH)
+    c.vs.attn_ws.fill_(0xff)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for s in range(c.w.batch):
+        c.check_attention(0, s)
+    ref = c.vs.attn_out.clone()
+    stream = torch.cuda.Stream()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        c.vs.attention(0, torch.cuda.current_stream().cuda_stream)
+    for _ in range(3):
+        c.vs.attn_out.zero_()
+        with torch.cuda.stream(stream):
+            g.replay()
+        stream.synchronize()
+        assert torch.equal(c.vs.attn_out[0], ref[0])
+    assert c.vs.results()["err"] == 0
 
 
 def test_splits_without_tiles():
@@ -330,8 +405,9 @@ def test_two_block_kernel_on_many_rows(name):
         c.check_attention(0, s)
 
 
-@pytest.mark.parametrize("kernel,balanced", [("auto", True), ("tc64", False), ("tc64", True),
-                                             ("stream", True), ("pair", True)])
+@pytest.mark.parametrize("kernel,balanced", [("auto", True), ("auto", False), ("tc64", False),
+                                             ("tc64", True), ("stream", True), ("pair", True),
+                                             ("batch", True)])
 def test_batch_work_split(balanced, kernel):
     """Eight sequences with prefixes from 100 to 700 rows: the automatic
     choice (clusters of 128-row CTAs, no workspace even when one is
@@ -339,11 +415,13 @@ def test_batch_work_split(balanced, kernel):
     (every sequence and KV head gets the same cluster) and with one (tiles
     dealt out to the SMs in proportion to each sequence's length); the
     continuous split on SMs and on SM pairs (partials merged by a second
-    kernel)."""
-    launch = {"auto": None, "tc64": TC64, "stream": STREAM, "pair": PAIR}[kernel]
+    kernel); the batch kernel (pieces in proportion to each sequence's
+    tiles, merged by the last piece in the same launch)."""
+    launch = {"auto": None, "tc64": TC64, "stream": STREAM, "pair": PAIR, "batch": BATCH}[kernel]
     c = Case(SMALL["7b-batch8-paged-small"], seed=11, balanced=balanced, attn_launch=launch)
-    assert (c.vs.attn_ws is not None) == (kernel != "auto" and balanced)
-    assert c.vs.launches_per_step() == c.L * (2 if c.vs.attn_ws is not None else 1) + 2
+    assert (c.vs.attn_ws is not None) == (balanced and kernel != "auto")
+    merge_kernel = balanced and kernel in ("tc64", "stream", "pair")
+    assert c.vs.launches_per_step() == c.L * (2 if merge_kernel else 1) + 2
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0
@@ -370,12 +448,14 @@ def test_attention_workspace_contract():
         pb.pf_verify_attention(d, 0)
     assert e.value.status == pb.PF_ERR_ALIGN
     d.workspace = c.vs.attn_ws.data_ptr()
-    # a single sequence needs none on the automatic choice (its KV heads and
-    # row blocks share clusters), one on the continuous-split kernels
+    # the automatic choice needs none (its KV heads and row blocks share
+    # clusters), the continuous-split and batch kernels one for any batch
     one = Case(SMALL["7b-tree64-small"], seed=12)
     assert pb.pf_verify_attention_workspace_size(one.vs.attn_descs[0]) == 0
     assert one.vs.attn_ws is None
-    for k in (pb.PF_ATTN_KERNEL_PAIR, pb.PF_ATTN_KERNEL_STREAM):
+    auto = Case(SMALL["7b-batch8-paged-small"], seed=12)
+    assert pb.pf_verify_attention_workspace_size(auto.vs.attn_descs[0]) == 0
+    for k in (pb.PF_ATTN_KERNEL_PAIR, pb.PF_ATTN_KERNEL_STREAM, pb.PF_ATTN_KERNEL_BATCH):
         one_k = Case(SMALL["7b-tree64-small"], seed=12, attn_launch=dict(kernel=k))
         assert pb.pf_verify_attention_workspace_size(one_k.vs.attn_descs[0]) > 0
 
@@ -399,11 +479,11 @@ def test_batch_beyond_balanced_groups():
     c.check_commit(res)
 
 
-@pytest.mark.parametrize("impl", ["default", "tc128", "tc64-balanced", "stream"])
+@pytest.mark.parametrize("impl", ["default", "batch", "tc64-balanced", "stream"])
 def test_mixed_tree_sizes(impl):
     """Sequences of 1, 17 and 128 nodes in one batch (variable cu_nodes), on
-    the default path, on the 128-token kernel, on the 64-token kernel's
-    balanced batch mode and on the continuous split."""
+    the default path (clusters), on the batch kernel, on the 64-token
+    kernel's balanced batch mode and on the continuous split."""
     w = I.scaled(W["7b-bf16-batch8-paged"], layers=1, batch=3, prefix=(50, 400), nodes=128,
                  vocab=640, hidden=128)
     rng = np.random.default_rng(9)
@@ -414,8 +494,8 @@ def test_mixed_tree_sizes(impl):
     per_seq = -(-max_seq // I.PAGE_SIZE)
     pt = rng.permutation(per_seq * 3).astype(np.int32).reshape(3, per_seq)
     b = I.Batch(w, 7, parents, prefix, ends, pt, per_seq * 3, max_seq)
-    launch = {"default": None, "tc128": TC128, "tc64-balanced": TC64, "stream": STREAM}[impl]
-    c = Case(w, batch=b, balanced=impl != "tc128", attn_launch=launch)
+    launch = {"default": None, "batch": BATCH, "tc64-balanced": TC64, "stream": STREAM}[impl]
+    c = Case(w, batch=b, attn_launch=launch)
     c.vs.step()
     res = c.vs.results()
     assert res["err"] == 0

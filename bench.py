@@ -640,16 +640,29 @@ def measure_workload(w, args, K, stream, flush, peaks, weight_dev=None, world=1,
 # ---------------------------------------------------------------------------
 # end to end through the library's calls
 # ---------------------------------------------------------------------------
+def e2e_cuts(L: int) -> list:
+    """Layer boundaries of the end-to-end leg's host copies: a first copy of
+    the per-step arrays and layer 0, then growing groups of layers (for 28
+    layers: 1-3, 4-9, 10-17, 18-27 with the hidden states), so each copy
+    lands before the layers that read it while the earlier layers run."""
+    return sorted({max(1, min(L - 1, int(round(L * f)))) for f in (1 / 28, 4 / 28, 10 / 28, 18 / 28)}
+                  ) if L > 1 else []
+
+
 def run_e2e(vs, w, K, stream, flush, world, tok_table, planned):
     """The same metric end to end, as a caller of the library sees it, timed
     on the host wall clock: every step copies its inputs (queries, proposal
-    K/V of every layer, hidden states, tokens, tree and lengths: one packed
-    arena) from pinned host memory, issues the C-ABI calls eagerly -- the
-    device tree bitmaps (pf_tree_prepare_device), L attention calls, the LM
-    head, the commit -- reads its outputs (accepted lengths, tokens, new
-    lengths: one arena) back and synchronises.  The L2 flush between steps
-    is outside the timed region.  A second figure replays the same step as
-    one CUDA graph between the copies (device events)."""
+    K/V of every layer, hidden states, tokens, tree and lengths) from pinned
+    host memory, issues the C-ABI calls eagerly -- the device tree bitmaps
+    (pf_tree_prepare_device), L attention calls, the LM head, the commit --
+    reads its outputs (accepted lengths, tokens, new lengths: one arena)
+    back and synchronises.  The input copy goes in a few pieces on a copy
+    stream (the per-step arrays and layer 0 first, then groups of layers,
+    the hidden states last), each layer's attention waiting only for the
+    piece that holds its inputs, so the copy overlaps the earlier layers.
+    The L2 flush between steps is outside the timed region.  A second
+    figure replays the same step -- copies, calls and the read-back -- as
+    one CUDA graph (device events around it)."""
     import torch
     host_in = vs.in_arena.detach().cpu().pin_memory()
     host_out = torch.empty(vs.out_arena.numel(), dtype=torch.uint8).pin_memory()
@@ -659,7 +672,32 @@ def run_e2e(vs, w, K, stream, flush, world, tok_table, planned):
     acc_off = vs.accept_len.data_ptr() - vs.out_arena.data_ptr()
     h2d, d2h = host_in.numel(), host_out.numel()
     n = min(K, 200)
-    sp = stream.cuda_stream
+    segs = vs.input_segments(e2e_cuts(vs.L))
+    copy_stream = torch.cuda.Stream()
+    landed = [torch.cuda.Event() for _ in segs]
+
+    def issue():
+        """One step's copies and calls on `stream` (and the copy stream)."""
+        sp = torch.cuda.current_stream().cuda_stream
+        cur = torch.cuda.current_stream()
+        copy_stream.wait_stream(cur)  # the arena is free: the previous step is done
+        with torch.cuda.stream(copy_stream):
+            for (o, nb, _, _), ev in zip(segs, landed):
+                vs.in_arena[o:o + nb].copy_(host_in[o:o + nb], non_blocking=True)
+                ev.record(copy_stream)
+        cur.wait_event(landed[0])
+        vs.tree_prepare(sp)
+        si = 0
+        for l in range(vs.L):
+            while segs[si][3] <= l:
+                si += 1
+                cur.wait_event(landed[si])
+            vs.attention(l, sp)
+        for ev in landed[si + 1:]:
+            cur.wait_event(ev)  # the hidden states' piece
+        vs.lmhead(sp)
+        vs.commit(sp)
+        host_out.copy_(vs.out_arena, non_blocking=True)
 
     def one(k, graph=None, events=None):
         host_in[tok_off:tok_off + tok_bytes].copy_(host_tokens[k % len(host_tokens)])
@@ -670,12 +708,10 @@ def run_e2e(vs, w, K, stream, flush, world, tok_table, planned):
         with torch.cuda.stream(stream):
             if events:
                 events[0].record(stream)
-            vs.in_arena.copy_(host_in, non_blocking=True)
             if graph is None:
-                vs.step(sp, tree_prepare=True)
+                issue()
             else:
                 graph.replay()
-            host_out.copy_(vs.out_arena, non_blocking=True)
             if events:
                 events[1].record(stream)
         stream.synchronize()
@@ -692,10 +728,10 @@ def run_e2e(vs, w, K, stream, flush, world, tok_table, planned):
         wall.append(t)
         tok += got
     t_wall = max_over_ranks(float(np.sum(wall)), world, "cuda")
-    # graph variant
+    # graph variant: the copies, the calls and the read-back in one graph
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g, stream=stream):
-        vs.step(torch.cuda.current_stream().cuda_stream, tree_prepare=True)
+        issue()
     with torch.cuda.stream(stream):
         g.replay()
     stream.synchronize()
@@ -711,14 +747,16 @@ def run_e2e(vs, w, K, stream, flush, world, tok_table, planned):
     return {"value": whole_job_rate(tok, t_wall, world), "unit": "tokens/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n,
             "ms_per_step": t_wall * 1e3 / n,
-            "timing": "host wall clock (time.perf_counter) around H2D, eager C-ABI calls "
-                      "(pf_tree_prepare_device, %d x pf_verify_attention, pf_lmhead_accept, "
-                      "pf_kv_commit), D2H and a stream synchronise, per step" % vs.L,
-            "copies_per_step": {"h2d": 1, "d2h": 1},
+            "timing": "host wall clock (time.perf_counter) around the H2D copies, eager C-ABI "
+                      "calls (pf_tree_prepare_device, %d x pf_verify_attention, "
+                      "pf_lmhead_accept, pf_kv_commit), D2H and a stream synchronise, per step"
+                      % vs.L,
+            "copies_per_step": {"h2d": len(segs), "d2h": 1},
+            "h2d_pieces_first_layers": [s[2] for s in segs],
             "graph": {"value": whole_job_rate(gtok, t_graph * 1e-3, world),
                       "ms_per_step": t_graph / n,
-                      "timing": "the same step as one CUDA-graph replay between the copies, "
-                                "device events around copies and replay"}}
+                      "timing": "the same step (copies, calls, read-back) as one CUDA-graph "
+                                "replay, device events around it"}}
 
 
 # ---------------------------------------------------------------------------

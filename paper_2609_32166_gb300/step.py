@@ -148,10 +148,72 @@ class VerifyStep:
         # one copy each way.
         # (the ancestor bitmaps are derived on the device from the parent
         # array by pf_tree_prepare_device, so they are not among the inputs)
-        self.in_arena = self._arena(("q", "tree_k", "tree_v", "hidden", "tokens", "parent",
-                                     "cu_nodes", "prefix_len"), device)
+        self.in_arena = self._input_arena(device)
         self.out_arena = self._arena(("accept_len", "out_tokens", "new_len"), device)
         self._build_descs()
+
+    def _input_arena(self, device) -> torch.Tensor:
+        """The step's inputs in one 256-byte-aligned byte arena, in the order
+        the step consumes them: the per-step arrays (tokens, parent array,
+        cu_nodes, prefix lengths), then one block per layer holding that
+        layer's q, proposal K and proposal V, then the hidden states.  q,
+        tree_k and tree_v become [L, ...] views with the block as their layer
+        stride, so a host copy can be issued layer by layer
+        (input_segments) and the commit still sees one layer stride."""
+        al = lambda x: (x + 255) // 256 * 256
+        es = self.q.element_size()
+        qb = self.q[0].numel() * es
+        kb = self.tree_k[0].numel() * es
+        q_o, k_o = 0, al(qb)
+        v_o = al(k_o + kb)
+        blk = al(v_o + kb)
+        off, heads = 0, {}
+        for n in ("tokens", "parent", "cu_nodes", "prefix_len"):
+            t = getattr(self, n)
+            off = al(off)
+            heads[n] = off
+            off += t.numel() * t.element_size()
+        layers0 = al(off)
+        hid_o = al(layers0 + self.L * blk)
+        total = hid_o + self.hidden.numel() * self.hidden.element_size()
+        arena = torch.empty(total, dtype=torch.uint8, device=device)
+        for n, o in heads.items():
+            t = getattr(self, n)
+            v = arena[o:o + t.numel() * t.element_size()].view(t.dtype).view(t.shape)
+            v.copy_(t)
+            setattr(self, n, v)
+        h = self.hidden
+        hv = arena[hid_o:hid_o + h.numel() * h.element_size()].view(h.dtype).view(h.shape)
+        hv.copy_(h)
+        self.hidden = hv
+        elems = arena[layers0:layers0 + self.L * blk].view(self.q.dtype)
+        base = elems.storage_offset()
+        for n, o in (("q", q_o), ("tree_k", k_o), ("tree_v", v_o)):
+            t = getattr(self, n)
+            stride = (blk // es,) + tuple(t[0].stride())
+            v = torch.as_strided(elems, tuple(t.shape), stride, base + o // es)
+            v.copy_(t)
+            setattr(self, n, v)
+        self._layers0, self._layer_block, self._hidden_off = layers0, blk, hid_o
+        return arena
+
+    def input_segments(self, boundaries) -> list:
+        """Byte ranges (offset, nbytes, first layer, end layer) of the input
+        arena for a layer-by-layer host copy: the first range holds the
+        per-step arrays and layers [0, boundaries[0]), each next one the
+        layers up to the next boundary, the last one also the hidden states
+        (end layer = L + 1 marks it)."""
+        cuts = [0] + [b for b in boundaries if 0 < b < self.L] + [self.L]
+        segs = []
+        for i in range(len(cuts) - 1):
+            l0, l1 = cuts[i], cuts[i + 1]
+            start = 0 if i == 0 else self._layers0 + l0 * self._layer_block
+            end = self._layers0 + l1 * self._layer_block
+            last = i == len(cuts) - 2
+            if last:
+                end = self.in_arena.numel()
+            segs.append((start, end - start, l0, self.L + 1 if last else l1))
+        return segs
 
     def _arena(self, names, device) -> torch.Tensor:
         """Move the named tensors into one 256-byte-aligned byte arena and
@@ -236,7 +298,7 @@ class VerifyStep:
         c.cu_nodes, c.prefix_len = self.cu_nodes.data_ptr(), self.prefix_len.data_ptr()
         c.accept_len, c.path = self.accept_len.data_ptr(), self.path.data_ptr()
         c.tree_k, c.tree_v = self.tree_k.data_ptr(), self.tree_v.data_ptr()
-        c.tree_layer_stride = self.tree_k[0].numel()
+        c.tree_layer_stride = self.tree_k.stride(0)  # elements between layers' proposal K/V
         c.cache = self._view(0)
         c.cache_layer_stride = self.cache_k[0].numel()
         c.new_len = self.new_len.data_ptr()

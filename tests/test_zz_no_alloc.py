@@ -51,3 +51,19 @@ def test_noalloc_rejects_more_rows_than_its_scratch_holds():
         pb.pf_lmhead_accept_noalloc(d, 0)
     assert e.value.status == pb.PF_ERR_SHAPE
     assert "scratch" in pb.pf_last_error()
+
+
+def test_noalloc_checks_the_descriptor_before_clearing_its_scratch():
+    """A descriptor the workspace entry point rejects is rejected with the
+    same status, before the scratch is cleared (nothing is queued)."""
+    d = pb.pf_lm_desc()
+    d.dtype, d.batch, d.hidden, d.vocab = pb.PF_BF16, 1, 64, 1000
+    d.total_nodes, d.max_nodes = 4, 4
+    fake = 0x10000
+    for f in ("cu_nodes", "hidden_states", "tokens", "parent", "argmax", "accept_len", "path",
+              "out_tokens"):
+        setattr(d, f, fake)
+    d.weight = None
+    with pytest.raises(pb.PfError) as e:
+        pb.pf_lmhead_accept_noalloc(d, 0)
+    assert e.value.status == pb.PF_ERR_NULL

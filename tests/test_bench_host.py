@@ -118,3 +118,49 @@ def test_cpu_baseline_mode_is_whole_steps_only_where_they_are_cheap():
     assert b.cpu_mode(W["2b-bf16-chain16"]) == "whole"
     for name in ("7b-bf16-tree64", "7b-bf16-batch8-paged", "7b-bf16-32k-tree128"):
         assert b.cpu_mode(W[name]) == "layer"
+
+
+def test_e2e_copy_pieces_follow_the_layers():
+    b = _bench()
+    assert b.e2e_cuts(28) == [1, 4, 10, 18]
+    assert b.e2e_cuts(1) == []
+    assert b.e2e_cuts(2) == [1]
+    for L in range(2, 40):
+        cuts = b.e2e_cuts(L)
+        assert cuts == sorted(set(cuts)) and all(0 < c < L for c in cuts)
+
+
+def test_input_arena_is_blocked_by_layer():
+    """The step's input arena on the host side (torch on the CPU): q and the
+    proposal K/V of layer l are one block, the views carry the original
+    values, the commit's layer stride is the block, and the copy pieces
+    tile the arena in order with the hidden states in the last one."""
+    import numpy as np
+    import torch
+    from paper_2609_32166_gb300.step import VerifyStep
+    w = inputs.scaled(inputs.WORKLOADS["7b-bf16-batch8-paged"], layers=3, prefix=(40, 100),
+                      vocab=300, hidden=64, batch=2)
+    batch = inputs.make_batch(w, 0)
+    vs = VerifyStep(w, batch, np.zeros(batch.total_nodes, np.int32), device="cpu")
+    bits = lambda t: t.contiguous().view(torch.int16).numpy().view(np.uint16)
+    for l in range(w.layers):
+        assert np.array_equal(bits(vs.q[l]), inputs.layer_q(w, batch, l))
+        tk, tv = inputs.layer_tree_kv(w, batch, l)
+        assert np.array_equal(bits(vs.tree_k[l]), tk) and np.array_equal(bits(vs.tree_v[l]), tv)
+        assert vs.q[l].is_contiguous() and vs.tree_k[l].is_contiguous()
+    blk = vs.tree_k.stride(0) * vs.tree_k.element_size()
+    assert vs.q.stride(0) == vs.tree_k.stride(0) == vs.tree_v.stride(0)
+    assert vs.tree_k[1].data_ptr() - vs.tree_k[0].data_ptr() == blk
+    assert vs.commit_desc.tree_layer_stride == vs.tree_k.stride(0)
+    assert np.array_equal(bits(vs.hidden), inputs.hidden_states(w, batch))
+    segs = vs.input_segments([1, 2])
+    assert [s[2:] for s in segs] == [(0, 1), (1, 2), (2, w.layers + 1)]
+    off = 0
+    for o, nb, _, _ in segs:
+        assert o == off and nb > 0
+        off += nb
+    assert off == vs.in_arena.numel()
+    base = vs.in_arena.data_ptr()
+    assert vs.q[1].data_ptr() - base == segs[1][0]  # a piece starts at its first layer's block
+    assert vs.hidden.data_ptr() - base >= segs[-1][0]
+    assert vs.tokens.data_ptr() - base < segs[0][1]

@@ -1031,7 +1031,13 @@ def main():
         dist.init_process_group("nccl")
 
     import __graft_entry__
+    # one process per GPU: local rank 0 builds (or finds the library up to
+    # date) before the others look, so no two ranks write it at once
+    if world > 1 and local != 0:
+        dist.barrier()
     __graft_entry__.build()
+    if world > 1 and local == 0:
+        dist.barrier()
 
     peaks = load_peaks()
     hbm_peak = peak_values(peaks)[0]

@@ -630,6 +630,15 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
     cuuint32_t box[4] = {64, PF_PAGE_SIZE, 1, 1};
     if ((st = make_map(&m.ck, 4, d->cache.k, dims, str, box, "cache.k")) != PF_OK) return st;
     if ((st = make_map(&m.cv, 4, d->cache.v, dims, str, box, "cache.v")) != PF_OK) return st;
+    if (wide) {
+      // the 128-token kernels' V: both 64-column halves of a page in one box
+      cuuint64_t dims5[5] = {64, PF_PAGE_SIZE, 2, (cuuint64_t)a.Hkv, (cuuint64_t)a.num_pages};
+      cuuint64_t str5[4] = {D * es, 64 * es, PF_PAGE_SIZE * D * es,
+                            (cuuint64_t)a.Hkv * PF_PAGE_SIZE * D * es};
+      cuuint32_t box5[5] = {64, PF_PAGE_SIZE, 2, 1, 1};
+      if ((st = make_map(&m.cv_page, 5, d->cache.v, dims5, str5, box5, "cache.v pages")) != PF_OK)
+        return st;
+    }
   }
   cudaError_t e;
   switch (ch.kernel) {

@@ -78,13 +78,17 @@ struct W2Smem {
 
 // TMA loads of one 128-token K/V tile into a ring stage: K then V, each two
 // 64-column halves of 128 rows.  Prefix cache: one 3-D box of 128 rows per
-// half (contiguous) or one 4-D box per 16-token page holding prefix rows
-// (paged); past the prefix, the proposal's own rows (one box of 128 nodes).
+// half (contiguous) or, paged, one 4-D box of K per 16-token page and half
+// and one 5-D box of V per page holding both halves; past the prefix, the
+// proposal's own rows (one box of 128 nodes).  A paged prefix tile's V
+// lands page by page, [page][half][16 rows][64 columns] (w2_v_desc); every
+// other tile's K and V, and a paged tile's K, half by half, [half][128
+// rows][64 columns].
 __device__ __forceinline__ void w2_issue_tile(const AttnArgs& a, const CUtensorMap* tm_ck,
-                                              const CUtensorMap* tm_cv, const CUtensorMap* tm_tk,
-                                              const CUtensorMap* tm_tv, uint8_t* stage,
-                                              uint32_t bar, int t, int n_ptiles, int b, int g,
-                                              int node0, int P, Pages8 pg) {
+                                              const CUtensorMap* tm_cv, const CUtensorMap* tm_cvp,
+                                              const CUtensorMap* tm_tk, const CUtensorMap* tm_tv,
+                                              uint8_t* stage, uint32_t bar, int t, int n_ptiles,
+                                              int b, int g, int node0, int P, Pages8 pg) {
   using S = W2Smem<2>;  // the tile layout does not depend on the ring depth
   uint8_t* sk = stage;
   uint8_t* sv = stage + S::kTileBytes;
@@ -105,11 +109,10 @@ __device__ __forceinline__ void w2_issue_tile(const AttnArgs& a, const CUtensorM
       for (int p = 0; p < 8; ++p) {
         if (p >= npages) break;
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int off = h * S::kHalfBytes + p * PF_PAGE_SIZE * 128;
-          tma_load_4d(smem_u32(sk + off), tm_ck, h * 64, 0, g, pages[p], bar);
-          tma_load_4d(smem_u32(sv + off), tm_cv, h * 64, 0, g, pages[p], bar);
-        }
+        for (int h = 0; h < 2; ++h)
+          tma_load_4d(smem_u32(sk + h * S::kHalfBytes + p * PF_PAGE_SIZE * 128), tm_ck, h * 64, 0,
+                      g, pages[p], bar);
+        tma_load_5d(smem_u32(sv + p * 2 * PF_PAGE_SIZE * 128), tm_cvp, 0, 0, 0, g, pages[p], bar);
       }
     }
   } else {
@@ -121,6 +124,16 @@ __device__ __forceinline__ void w2_issue_tile(const AttnArgs& a, const CUtensorM
       tma_load_3d(smem_u32(sv + h * S::kHalfBytes), tm_tv, h * 64, g, node0 + j * kW, bar);
     }
   }
+}
+
+// PV's B operand for keys 16 kt .. 16 kt + 15 of the tile's V at v0: in
+// the page layout the 16 keys are one page (its halves 2 KB apart), else
+// 16 rows of both 16 KB halves.
+__device__ __forceinline__ uint64_t w2_v_desc(uint32_t v0, int kt, bool page_layout) {
+  using S = W2Smem<2>;
+  return page_layout
+             ? umma_desc_sw128_lbo(v0 + kt * 2 * PF_PAGE_SIZE * 128, PF_PAGE_SIZE * 128, 1024)
+             : umma_desc_sw128_lbo(v0 + kt * 16 * 128, S::kHalfBytes, 1024);
 }
 
 // D[tmem] (+)= A[tmem] * B[smem]^T, kind::f16: A is M rows (TMEM lanes) x 16
@@ -141,7 +154,8 @@ __global__ void __launch_bounds__(kW2Threads, 1)
                     const __grid_constant__ CUtensorMap tm_tk,
                     const __grid_constant__ CUtensorMap tm_tv,
                     const __grid_constant__ CUtensorMap tm_ck,
-                    const __grid_constant__ CUtensorMap tm_cv, const AttnArgs a) {
+                    const __grid_constant__ CUtensorMap tm_cv,
+                    const __grid_constant__ CUtensorMap tm_cvp, const AttnArgs a) {
   using S = W2Smem<STAGES>;
   constexpr int kW2Stages = STAGES;
   constexpr int D = 128;
@@ -242,7 +256,7 @@ __global__ void __launch_bounds__(kW2Threads, 1)
 #pragma unroll
     for (int i = 0; i < kW2Stages; ++i)
       if (i < first && i < my_ptiles)
-        w2_issue_tile(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
+        w2_issue_tile(a, &tm_ck, &tm_cv, &tm_cvp, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
                       smem_u32(&kv_full[i]), tile_at(i), n_ptiles, b, g, node0, P, pg[i]);
   }
   if (early) pdl_wait();
@@ -254,7 +268,7 @@ __global__ void __launch_bounds__(kW2Threads, 1)
                   smem_u32(q_full));
     for (int i = 0; i < first; ++i)
       if (i >= my_ptiles)  // proposal tiles: no page entries
-        w2_issue_tile(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
+        w2_issue_tile(a, &tm_ck, &tm_cv, &tm_cvp, &tm_tk, &tm_tv, sKV + i * S::kStageBytes,
                       smem_u32(&kv_full[i]), tile_at(i), n_ptiles, b, g, node0, P,
                       no_pages8());
   }
@@ -280,7 +294,7 @@ __global__ void __launch_bounds__(kW2Threads, 1)
         const int t = tile_at(i);
         const Pages8 pg = kv_tile_pages8(a, t, n_ptiles, b, P);  // in flight during the wait
         if (!mbar_wait(smem_u32(&kv_empty[st]), ((i / kW2Stages) & 1) ^ 1, a.err)) break;
-        w2_issue_tile(a, &tm_ck, &tm_cv, &tm_tk, &tm_tv, sKV + st * S::kStageBytes,
+        w2_issue_tile(a, &tm_ck, &tm_cv, &tm_cvp, &tm_tk, &tm_tv, sKV + st * S::kStageBytes,
                       smem_u32(&kv_full[st]), t, n_ptiles, b, g, node0, P, pg);
       }
     }
@@ -320,11 +334,11 @@ __global__ void __launch_bounds__(kW2Threads, 1)
           if (mbar_test_wait(smem_u32(&p_full[pb]), (j >> 1) & 1)) {
             tc_fence_after();
             const uint32_t v0 = smem_u32(sKV + stj * S::kStageBytes + S::kTileBytes);
+            const bool vpage = a.layout != PF_KV_CONTIGUOUS && tile_at(j) < n_ptiles;
 #pragma unroll
             for (int kt = 0; kt < kW / 16; ++kt)
-              umma_bf16_tmem_a(tmem + kColO, tmem + kColP + pb * 64 + kt * 8,
-                               umma_desc_sw128_lbo(v0 + kt * 16 * 128, S::kHalfBytes, 1024), id_o,
-                               (j > 0 || kt > 0) ? 1u : 0u);
+              umma_bf16_tmem_a(tmem + kColO, tmem + kColP + pb * 64 + kt * 8, w2_v_desc(v0, kt, vpage),
+                               id_o, (j > 0 || kt > 0) ? 1u : 0u);
             umma_commit(smem_u32(&pv_done[pb]));
             umma_commit(smem_u32(&kv_empty[stj]));
             ++np;
@@ -464,10 +478,20 @@ __global__ void __launch_bounds__(kW2Threads, 1)
         // The rows from `valid` on are one contiguous run per 64-column half.
         uint4* vt = reinterpret_cast<uint4*>(sKV + st * S::kStageBytes + S::kTileBytes);
         const int per_half = (kW - valid) * 8;   // 16-byte chunks past the end
+        if (a.layout == PF_KV_CONTIGUOUS) {
 #pragma unroll
-        for (int h = 0; h < 2; ++h)
-          for (int c = rl; c < per_half; c += 128)
-            vt[h * kW * 8 + valid * 8 + c] = make_uint4(0, 0, 0, 0);
+          for (int h = 0; h < 2; ++h)
+            for (int c = rl; c < per_half; c += 128)
+              vt[h * kW * 8 + valid * 8 + c] = make_uint4(0, 0, 0, 0);
+        } else {
+          // page layout: row r of half h at chunk (r / 16) * 256 + h * 128 + (r % 16) * 8
+#pragma unroll
+          for (int h = 0; h < 2; ++h)
+            for (int c = rl; c < per_half; c += 128) {
+              const int r = valid + (c >> 3);
+              vt[(r >> 4) * 256 + h * 128 + (r & 15) * 8 + (c & 7)] = make_uint4(0, 0, 0, 0);
+            }
+        }
         fence_proxy_async_smem();
       }
       tc_fence_before();
@@ -685,7 +709,7 @@ static cudaError_t launch_tc2(const AttnArgs& a, const AttnMaps& m, cudaStream_t
   if (BAL) {
     // one CTA per item, no cluster
     return launch_ex(attn_tc2_kernel<STAGES, BAL>, dim3(a.items), dim3(kW2Threads), smem, s, 1,
-                     pdl, m.q, m.tk, m.tv, m.ck, m.cv, a);
+                     pdl, m.q, m.tk, m.tv, m.ck, m.cv, m.cv_page, a);
   }
   if (a.splits > 8) {
     e = ensure_nonportable_cluster((const void*)attn_tc2_kernel<STAGES, BAL>, nonportable);
@@ -693,7 +717,7 @@ static cudaError_t launch_tc2(const AttnArgs& a, const AttnMaps& m, cudaStream_t
   }
   const dim3 grid(a.B * a.Hkv * a.rb_count * a.splits);
   return launch_ex(attn_tc2_kernel<STAGES, BAL>, grid, dim3(kW2Threads), smem, s, a.splits, pdl,
-                   m.q, m.tk, m.tv, m.ck, m.cv, a);
+                   m.q, m.tk, m.tv, m.ck, m.cv, m.cv_page, a);
 }
 
 // Ring depth: 3 stages (inbox in the ring, peers send after every CTA of

@@ -56,6 +56,10 @@ struct AttnArgs {
 
 struct AttnMaps {
   CUtensorMap q, tk, tv, ck, cv;
+  // paged cache only: V of one (page, KV head) as a 5-D map (64 columns, 16
+  // rows, the two 64-column halves, head, page), so that one box brings both
+  // halves of a page in [half][row][column] order
+  CUtensorMap cv_page;
 };
 
 cudaError_t launch_attention_bf16(const AttnArgs& a, const AttnMaps& m, cudaStream_t s,

@@ -53,7 +53,8 @@ LMHEAD_TRAFFIC = (os.path.join(ROOT, "profiles", "lmhead_traffic.txt"),
                   ("lmhead.cu", "pf_ptx.cuh"))
 ATTENTION_TRAFFIC = (os.path.join(ROOT, "profiles", "attention_traffic.txt"),
                      ("api.cu", "attention.cu", "attention_tc.cu", "attention_tc2.cu",
-                      "attention_pair.cu", "attn_common.cuh", "pf_internal.h", "pf_ptx.cuh"))
+                      "attention_2blk.cu", "attention_pair.cu", "attn_common.cuh",
+                      "pf_internal.h", "pf_ptx.cuh"))
 
 
 def parse(argv=None):

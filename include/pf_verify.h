@@ -187,6 +187,15 @@ typedef struct pf_attn_desc {
                                   1..16; 0 for PAIR, STREAM and BATCH        */
   int32_t rows_per_cta;        /* PF_ATTN_KERNEL_TC64: 128 or 256            */
   int32_t stages;              /* PF_ATTN_KERNEL_TC128 ring depth: 2 or 3    */
+  /* Optional host copies of cu_nodes[B+1] and prefix_len[B] (NULL: not
+   * given).  With both given and splits = 0, PF_ATTN_KERNEL_TWO_BLOCK deals
+   * the CTAs of its clusters out to the (sequence, KV head) groups in
+   * proportion to their tiles (a team of CTAs per group inside one cluster)
+   * where that shortens the longest piece.  The kernels read only the
+   * device arrays: host copies that differ from them cost balance, never
+   * correctness.  Read during the call only. */
+  const int32_t* host_cu_nodes;
+  const int32_t* host_prefix_len;
 } pf_attn_desc;
 
 /* Attention kernels (bf16; the fp32 path has one kernel and takes 0).
@@ -209,7 +218,11 @@ typedef struct pf_attn_desc {
  *          pieces, so they read the same pages together), and the last
  *          piece of each to finish merges the pieces in the same kernel
  *          (one launch per call); needs the workspace
- * TC64, TC128, PAIR, STREAM and BATCH need bf16 and D = 128.  The automatic
+ *   TWO_BLOCK  TC128's tiles with two 128-row blocks of one (sequence, KV
+ *          head) per CTA, so that each K/V tile enters the SM once for up
+ *          to 256 query rows (KV heads with more than 128 rows: G x nodes);
+ *          clusters split the tiles as for TC128
+ * TC64, TC128, PAIR, STREAM, BATCH and TWO_BLOCK need bf16 and D = 128.  The automatic
  * choice is TC128 (128-row CTAs in clusters that split each row block's
  * tiles) where a CTA holds several 128-token tiles, TC64 otherwise, MMA for
  * other head sizes; it takes no workspace. */
@@ -220,7 +233,8 @@ typedef enum pf_attn_kernel {
   PF_ATTN_KERNEL_TC128 = 3,
   PF_ATTN_KERNEL_PAIR = 4,
   PF_ATTN_KERNEL_STREAM = 5,
-  PF_ATTN_KERNEL_BATCH = 6
+  PF_ATTN_KERNEL_BATCH = 6,
+  PF_ATTN_KERNEL_TWO_BLOCK = 7
 } pf_attn_kernel;
 
 /* PF_ATTN_EARLY_PREFETCH: the prefix cache, page_table, cu_nodes, prefix_len

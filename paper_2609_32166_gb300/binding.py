@@ -29,7 +29,8 @@ PF_DEVERR_TIMEOUT, PF_DEVERR_CAPACITY, PF_DEVERR_BOUNDS, PF_DEVERR_TREE = 1, 2, 
 PF_ATTN_EARLY_PREFETCH, PF_ATTN_NO_PDL = 1, 2
 PF_LM_EARLY_WEIGHT, PF_LM_NO_PDL = 1, 2
 (PF_ATTN_KERNEL_AUTO, PF_ATTN_KERNEL_MMA, PF_ATTN_KERNEL_TC64, PF_ATTN_KERNEL_TC128,
- PF_ATTN_KERNEL_PAIR, PF_ATTN_KERNEL_STREAM, PF_ATTN_KERNEL_BATCH) = 0, 1, 2, 3, 4, 5, 6
+ PF_ATTN_KERNEL_PAIR, PF_ATTN_KERNEL_STREAM, PF_ATTN_KERNEL_BATCH,
+ PF_ATTN_KERNEL_TWO_BLOCK) = 0, 1, 2, 3, 4, 5, 6, 7
 
 STATUS_NAMES = {0: "PF_OK", 1: "PF_ERR_NULL", 2: "PF_ERR_SHAPE", 3: "PF_ERR_DTYPE",
                 4: "PF_ERR_TREE", 5: "PF_ERR_CAPACITY", 6: "PF_ERR_ALIGN", 7: "PF_ERR_CUDA",
@@ -62,7 +63,8 @@ class pf_attn_desc(C.Structure):
                 ("out", C.c_void_p), ("error_flag", C.c_void_p), ("flags", C.c_int32),
                 ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t),
                 ("kernel", C.c_int32), ("splits", C.c_int32), ("rows_per_cta", C.c_int32),
-                ("stages", C.c_int32)]
+                ("stages", C.c_int32), ("host_cu_nodes", C.c_void_p),
+                ("host_prefix_len", C.c_void_p)]
 
 
 class pf_lm_desc(C.Structure):

@@ -14,6 +14,7 @@
 #include <mutex>
 #include <algorithm>
 #include <string>
+#include <vector>
 
 #include "pf_internal.h"
 
@@ -108,7 +109,7 @@ pf_status check_cache_view(const pf_kv_view& c, int need_rows, const char* who) 
 // follows from the shape, unless the descriptor's launch fields ask for
 // something specific; nothing is read from the environment.
 // ---------------------------------------------------------------------------
-enum class AttnKernel { F32, MMA, TC64, TC128, PAIR, STREAM, BATCH };
+enum class AttnKernel { F32, MMA, TC64, TC128, PAIR, STREAM, BATCH, TWOBLK };
 
 // A distinct epoch for every call of a kernel that merges its own pieces
 // (the group tickets in the workspace compare it): 1 .. 2^40 - 1, wrapping.
@@ -146,7 +147,7 @@ int max_cluster_for(int kernel, int D, int want) {
 // variant (memoised per device): 0 tc64 128 rows, 1 tc64 256 rows, 2 tc128
 // 3 stages, 3 tc128 2 stages.
 int max_active_clusters(int variant, int cluster) {
-  static std::atomic<int> cache[64][4][17];
+  static std::atomic<int> cache[64][5][17];
   int dev = 0;
   cudaGetDevice(&dev);
   std::atomic<int>& slot = cache[dev & 63][variant][cluster];
@@ -157,7 +158,8 @@ int max_active_clusters(int variant, int cluster) {
       case 0: n = pf::attention_tc_max_active_clusters(cluster, 128); break;
       case 1: n = pf::attention_tc_max_active_clusters(cluster, 256); break;
       case 2: n = pf::attention_tc2_max_active_clusters(cluster, 3); break;
-      default: n = pf::attention_tc2_max_active_clusters(cluster, 2); break;
+      case 3: n = pf::attention_tc2_max_active_clusters(cluster, 2); break;
+      default: n = pf::attention_2blk_max_active_clusters(cluster); break;
     }
     c = std::max(1, n) + 1;
     slot.store(c, std::memory_order_release);
@@ -180,7 +182,106 @@ struct AttnChoice {
   AttnKernel kernel;
   int stages;       // TC128 ring depth
   size_t ws_need;   // workspace bytes the balanced batch mode needs (0: not used)
+  pf::TeamPlan tp;  // TWOBLK with a.team = 1
 };
+
+// Team plan of the two-block kernel from host copies of cu_nodes and
+// prefix_len: clusters of s CTAs, each (sequence, KV head, pair of row
+// blocks) group a team of k CTAs inside one cluster.  For a target of at
+// most X tiles per CTA every group needs k = ceil(tiles / X) CTAs; the teams
+// are packed largest first into the first cluster with room (first-fit
+// decreasing), and the smallest X whose teams fit wins, over every even
+// cluster size whose clusters all fit on the GPU at once (ties: the smaller
+// cluster).  A cluster's spare CTAs then join its team with the most tiles
+// per CTA.  Used only where X is below the one-group clusters' tiles per CTA
+// (`uniform_splits` CTAs per group).
+bool make_team_plan(pf::AttnArgs& a, const int32_t* hcu, const int32_t* hP, int sms,
+                    int uniform_splits, pf::TeamPlan* tp, int* tiles_per_cta = nullptr) {
+  struct Grp {
+    int id, t;
+  };
+  if ((long long)a.B * a.Hkv * a.rb_count > 4096) return false;  // 12-bit group ids
+  std::vector<Grp> gs;
+  for (int b = 0; b < a.B; ++b) {
+    const int nn = hcu[b + 1] - hcu[b], P = hP[b];
+    if (nn < 1 || nn > a.max_nodes || P < 0 || P > a.max_prefix) return false;
+    const int t = (P + 127) / 128 + (nn + 127) / 128;
+    const int pairs = (nn + a.nb - 1) / a.nb;
+    for (int g = 0; g < a.Hkv; ++g)
+      for (int rb = 0; rb < pairs; ++rb) gs.push_back({(b * a.Hkv + g) * a.rb_count + rb, t});
+  }
+  const int G = (int)gs.size();
+  if (G < 2) return false;
+  std::stable_sort(gs.begin(), gs.end(), [](const Grp& x, const Grp& y) { return x.t > y.t; });
+  long long total = 0;
+  for (const Grp& x : gs) total += x.t;
+  int best_x = (gs[0].t + uniform_splits - 1) / uniform_splits;  // to beat
+  int best_s = 0;
+  std::vector<int> best_k, best_c;
+  std::vector<int> k(G), cl(G);
+  for (int s = 2; s <= 16; s += 2) {
+    const int C = std::min(std::min(max_active_clusters(4, s), sms / s), pf::kTeamMaxCtas / s);
+    if (C < 1) continue;
+    const long long lo_total = (total + (long long)C * s - 1) / ((long long)C * s);
+    const int lo = std::max((int)lo_total, (gs[0].t + s - 1) / s);
+    for (int X = std::max(lo, 1); X < best_x; ++X) {
+      long long need = 0;
+      for (int j = 0; j < G; ++j) need += (k[j] = (gs[j].t + X - 1) / X);
+      if (need > (long long)C * s) continue;
+      // first-fit decreasing (gs is sorted by tiles, so k is non-increasing)
+      std::vector<int> room(C, s);
+      bool ok = true;
+      for (int j = 0; j < G && ok; ++j) {
+        int c = 0;
+        while (c < C && room[c] < k[j]) ++c;
+        if (c == C) {
+          ok = false;
+        } else {
+          cl[j] = c;
+          room[c] -= k[j];
+        }
+      }
+      if (!ok) continue;
+      for (int c = 0; c < C; ++c)
+        while (room[c] > 0) {
+          int jb = -1;
+          for (int j = 0; j < G; ++j)
+            if (cl[j] == c && (jb < 0 || (long long)gs[j].t * k[jb] > (long long)gs[jb].t * k[j]))
+              jb = j;
+          if (jb < 0) break;  // a cluster without teams stays empty
+          ++k[jb];
+          --room[c];
+        }
+      best_x = X;
+      best_s = s;
+      best_k = k;
+      best_c = cl;
+      break;
+    }
+  }
+  if (best_s == 0) return false;
+  // number the used clusters, lay each one's teams out from rank 0
+  const int s = best_s;
+  std::vector<int> cidx(pf::kTeamMaxCtas, -1), next_rank;
+  int used = 0;
+  for (int j = 0; j < G; ++j)
+    if (cidx[best_c[j]] < 0) {
+      cidx[best_c[j]] = used++;
+      next_rank.push_back(0);
+    }
+  for (int i = 0; i < pf::kTeamMaxCtas; ++i) tp->e[i] = pf::team_entry(0, 0, 0, 0);
+  for (int j = 0; j < G; ++j) {
+    const int c = cidx[best_c[j]], base = next_rank[c];
+    for (int part = 0; part < best_k[j]; ++part)
+      tp->e[c * s + base + part] = pf::team_entry(gs[j].id, part, best_k[j], base);
+    next_rank[c] += best_k[j];
+  }
+  a.team = 1;
+  a.splits = s;
+  a.team_ctas = used * s;
+  if (tiles_per_cta) *tiles_per_cta = best_x;
+  return true;
+}
 
 // Validates the launch fields and fills a.bm, a.nb, a.rb_count, a.splits
 // and, when `ws_ok` and the shape allows, the balanced batch mode (a.items).
@@ -200,6 +301,8 @@ pf_status choose_attention(const pf_attn_desc* d, pf::AttnArgs& a, int sms, bool
   // The pair kernel's groups: 256-row blocks of floor(128 / G) nodes per CTA;
   // the continuous-split kernel's: 128-row blocks of floor(128 / G) nodes.
   const int pair_nb = 2 * (128 / G);
+  const int tiles64 = (a.max_prefix + 63) / 64 + (a.max_nodes + 63) / 64;
+  const int tiles128 = (a.max_prefix + 127) / 128 + (a.max_nodes + 127) / 128;
   const int pair_groups = a.B * a.Hkv * ((a.max_nodes + pair_nb - 1) / pair_nb);
   const int sk_nb = 128 / G;
   const int sk_groups = a.B * a.Hkv * ((a.max_nodes + sk_nb - 1) / sk_nb);
@@ -232,16 +335,39 @@ pf_status choose_attention(const pf_attn_desc* d, pf::AttnArgs& a, int sms, bool
     // bytes), and its last-piece merge adds ~5 us to the layer's tail.
     k = D != 128 ? AttnKernel::MMA : AttnKernel::TC64;  // may become TC128 below
     if (k == AttnKernel::TC64) a_bm_auto = 128;
+    // A batch whose KV heads have more than 128 rows, with the host's copies
+    // of the lengths: two 128-row blocks per CTA and teams of a cluster's
+    // CTAs per group, sized by the groups' tiles, where the plan leaves each
+    // CTA at least 4 tiles (its fixed per-launch cost is higher than the
+    // one-block kernel's).  8-sequence batch (prefixes 2048..6144, 32-node
+    // trees), us per layer: 33.7 against 35.7 (paged), 32.5 against 32.6
+    // (contiguous cache).  Single sequences keep the one-block clusters
+    // (64-node tree 16.4 against 13.6, 32K tree 87.9 against 68.1).
+    if (D == 128 && a.B > 1 && G * a.max_nodes > 128 && d->host_cu_nodes &&
+        d->host_prefix_len) {
+      pf::AttnArgs t = a;
+      t.bm = 256;
+      t.nb = pair_nb;
+      t.rb_count = (t.max_nodes + t.nb - 1) / t.nb;
+      const int uniform = widest_split(4, t.B * t.Hkv * t.rb_count, tiles128, 16, 1);
+      int per_cta = 0;
+      if (make_team_plan(t, d->host_cu_nodes, d->host_prefix_len, sms, uniform, &out->tp,
+                         &per_cta) &&
+          per_cta >= 4) {
+        a = t;
+        out->kernel = AttnKernel::TWOBLK;
+        return PF_OK;
+      }
+    }
   } else {
     k = d->kernel == PF_ATTN_KERNEL_MMA    ? AttnKernel::MMA
         : d->kernel == PF_ATTN_KERNEL_TC64 ? AttnKernel::TC64
         : d->kernel == PF_ATTN_KERNEL_TC128 ? AttnKernel::TC128
         : d->kernel == PF_ATTN_KERNEL_PAIR  ? AttnKernel::PAIR
         : d->kernel == PF_ATTN_KERNEL_BATCH ? AttnKernel::BATCH
+        : d->kernel == PF_ATTN_KERNEL_TWO_BLOCK ? AttnKernel::TWOBLK
                                             : AttnKernel::STREAM;
   }
-  const int tiles64 = (a.max_prefix + 63) / 64 + (a.max_nodes + 63) / 64;
-  const int tiles128 = (a.max_prefix + 127) / 128 + (a.max_nodes + 127) / 128;
 
   if (k == AttnKernel::MMA) {
     const int bms[3] = {128, 64, 32};
@@ -281,6 +407,20 @@ pf_status choose_attention(const pf_attn_desc* d, pf::AttnArgs& a, int sms, bool
     a.items = sms;  // one CTA per SM
     a.slots = 1;
     out->ws_need = pf::attention_balanced_ws_bytes(a.items, a.bm, D, 1);
+    out->kernel = k;
+    return PF_OK;
+  }
+  if (k == AttnKernel::TWOBLK) {
+    // two 128-row blocks of floor(128 / G) nodes per CTA, clusters over the
+    // 128-token tiles: one group per cluster, or (host lengths given) teams
+    a.bm = 256;
+    a.nb = pair_nb;
+    a.rb_count = (a.max_nodes + a.nb - 1) / a.nb;
+    const int groups = a.B * a.Hkv * a.rb_count;
+    a.splits = d->splits > 0 ? std::min(d->splits, tiles128)
+                             : widest_split(4, groups, tiles128, 16, 1);
+    if (d->splits == 0 && d->host_cu_nodes && d->host_prefix_len)
+      make_team_plan(a, d->host_cu_nodes, d->host_prefix_len, sms, a.splits, &out->tp);
     out->kernel = k;
     return PF_OK;
   }
@@ -366,7 +506,7 @@ pf_status attention_args(const pf_attn_desc* d, pf::AttnArgs& a, const char* who
   if (d->flags & ~(PF_ATTN_EARLY_PREFETCH | PF_ATTN_NO_PDL))
     return fail(PF_ERR_SHAPE, "%s: unknown flags 0x%x", who, d->flags);
   // launch fields
-  if (d->kernel < PF_ATTN_KERNEL_AUTO || d->kernel > PF_ATTN_KERNEL_BATCH)
+  if (d->kernel < PF_ATTN_KERNEL_AUTO || d->kernel > PF_ATTN_KERNEL_TWO_BLOCK)
     return fail(PF_ERR_SHAPE, "%s: unknown kernel %d", who, d->kernel);
   if (d->dtype == PF_F32 && (d->kernel != PF_ATTN_KERNEL_AUTO || d->splits != 0 ||
                              d->rows_per_cta != 0 || d->stages != 0))
@@ -374,7 +514,7 @@ pf_status attention_args(const pf_attn_desc* d, pf::AttnArgs& a, const char* who
                 who);
   const bool tc_kernel = d->kernel == PF_ATTN_KERNEL_TC64 || d->kernel == PF_ATTN_KERNEL_TC128 ||
                          d->kernel == PF_ATTN_KERNEL_PAIR || d->kernel == PF_ATTN_KERNEL_STREAM ||
-                         d->kernel == PF_ATTN_KERNEL_BATCH;
+                         d->kernel == PF_ATTN_KERNEL_BATCH || d->kernel == PF_ATTN_KERNEL_TWO_BLOCK;
   if (tc_kernel && D != 128)
     return fail(PF_ERR_SHAPE, "%s: the tcgen05 kernels need head_dim 128", who);
   if (d->splits < 0 || d->splits > 16 ||
@@ -596,10 +736,11 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
   // loads half a tile per CTA: 64 K rows, 128 V rows of 64 columns).
   const bool pair = ch.kernel == AttnKernel::PAIR;
   const bool wide = ch.kernel == AttnKernel::TC128 || ch.kernel == AttnKernel::STREAM ||
-                    ch.kernel == AttnKernel::BATCH;
+                    ch.kernel == AttnKernel::BATCH || ch.kernel == AttnKernel::TWOBLK;
   const cuuint32_t k_rows = pair ? 64 : wide ? 128 : 64;
   const cuuint32_t v_rows = pair ? 128 : k_rows;
-  const cuuint32_t q_nodes = pair ? (cuuint32_t)(a.nb / 2) : (cuuint32_t)a.nb;
+  const cuuint32_t q_nodes =
+      pair || ch.kernel == AttnKernel::TWOBLK ? (cuuint32_t)(a.nb / 2) : (cuuint32_t)a.nb;
   pf::AttnMaps m;
   const cuuint64_t es = 2;
   {
@@ -649,6 +790,7 @@ pf_status pf_verify_attention(const pf_attn_desc* d, void* stream) {
       a.epoch = next_epoch();
       e = pf::launch_attention_tc2(a, m, s, pdl, 3, true);
       break;
+    case AttnKernel::TWOBLK: e = pf::launch_attention_2blk(a, m, ch.tp, s, pdl); break;
     case AttnKernel::TC64: e = pf::launch_attention_tc(a, m, s, pdl); break;
     default: e = pf::launch_attention_bf16(a, m, s, sms, pdl); break;
   }

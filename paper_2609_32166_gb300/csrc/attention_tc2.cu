@@ -136,18 +136,6 @@ __device__ __forceinline__ uint64_t w2_v_desc(uint32_t v0, int kt, bool page_lay
              : umma_desc_sw128_lbo(v0 + kt * 16 * 128, S::kHalfBytes, 1024);
 }
 
-// D[tmem] (+)= A[tmem] * B[smem]^T, kind::f16: A is M rows (TMEM lanes) x 16
-// bf16 (8 columns of packed pairs) starting at column a_tmem.
-__device__ __forceinline__ void umma_bf16_tmem_a(uint32_t d_tmem, uint32_t a_tmem,
-                                                 uint64_t b_desc, uint32_t idesc,
-                                                 uint32_t accumulate) {
-  asm volatile(
-      "{ .reg .pred p; setp.ne.b32 p, %4, 0; "
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p; }" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-
 template <int STAGES, bool BAL>
 __global__ void __launch_bounds__(kW2Threads, 1)
     attn_tc2_kernel(const __grid_constant__ CUtensorMap tm_q,

@@ -30,6 +30,11 @@ struct AttnArgs {
   // partial slots per item: 1 (tc64: one group part per CTA) or 2 (the pair
   // kernel's continuous split: an item's first and last group piece)
   int slots;
+  // two-block kernel: 1 = the CTAs follow a TeamPlan (teams of a cluster's
+  // CTAs per group) instead of one group per cluster; team_ctas = its CTAs
+  // (a multiple of the cluster size a.splits)
+  int team;
+  int team_ctas;
   void* ws;
   // this call's epoch for the group tickets of the kernels that merge their
   // own pieces (see group_tickets): distinct for every call, < 2^40
@@ -81,6 +86,24 @@ cudaError_t launch_attention_tc(const AttnArgs& a, const AttnMaps& m, cudaStream
 cudaError_t launch_attention_tc2(const AttnArgs& a, const AttnMaps& m, cudaStream_t s, bool pdl,
                                  int stages, bool balanced);
 int attention_tc2_max_active_clusters(int cluster, int stages);
+// tcgen05 variant with 128-token K/V tiles and two 128-row blocks per CTA
+// (bf16, D = 128, a.bm = 256, a.nb = 2 * floor(128 / G) nodes per CTA),
+// cluster split-KV over a.splits CTAs; needs the 128-token tensor maps and,
+// for a paged cache, m.cv_page.
+// The two-block kernel's team plan: CTA x works on piece part of the
+// nparts pieces of group `group`, whose pieces are the CTAs base ..
+// base + nparts - 1 of x's cluster (cluster ranks); nparts = 0: no work.
+// Packed as group | part << 12 | nparts << 17 | base << 22.
+constexpr int kTeamMaxCtas = 160;
+struct TeamPlan {
+  uint32_t e[kTeamMaxCtas];
+};
+__host__ __device__ constexpr uint32_t team_entry(int group, int part, int nparts, int base) {
+  return (uint32_t)group | (uint32_t)part << 12 | (uint32_t)nparts << 17 | (uint32_t)base << 22;
+}
+cudaError_t launch_attention_2blk(const AttnArgs& a, const AttnMaps& m, const TeamPlan& tp,
+                                  cudaStream_t s, bool pdl);
+int attention_2blk_max_active_clusters(int cluster);
 // tcgen05 variant on SM pairs (2-SM MMA, M = 256 rows per pair, 128-token
 // tiles; bf16, D = 128): a.bm = 256, a.nb = 2 * floor(128 / G) nodes per
 // pair, a.items pairs sharing all groups' tiles in equal contiguous ranges

@@ -83,6 +83,9 @@ class VerifyStep:
         self.mask = torch.from_numpy(mask.view(np.int64)).to(device)
         self.cu_nodes = torch.from_numpy(batch.cu_nodes).to(device)
         self.prefix_len = torch.from_numpy(batch.prefix_lens.astype(np.int32)).to(device)
+        # host copies for the launch plan (read by the attention call only)
+        self.h_cu_nodes = np.array(batch.cu_nodes, dtype=np.int32)
+        self.h_prefix_len = np.array(batch.prefix_lens, dtype=np.int32)
         self.parent = torch.from_numpy(batch.parent_flat).to(device)
         self.tokens = torch.from_numpy(np.asarray(tokens, dtype=np.int32)).to(device)
         self.page_table = (torch.from_numpy(batch.page_table).to(device)
@@ -268,6 +271,8 @@ class VerifyStep:
             # after the last layer: every layer but the first may request its
             # cache tiles while the previous layer is still finishing.
             d.flags = pb.PF_ATTN_EARLY_PREFETCH if l > 0 else 0
+            d.host_cu_nodes = self.h_cu_nodes.ctypes.data
+            d.host_prefix_len = self.h_prefix_len.ctypes.data
             for k, v in self.attn_launch.items():
                 setattr(d, k, int(v))
             self.attn_descs.append(d)

@@ -131,7 +131,11 @@ def _attn_desc(**kw):
           max_prefix_len=17), pb.PF_ERR_CAPACITY),
     (dict(q=0x10008), pb.PF_ERR_ALIGN),
     # launch fields
-    (dict(kernel=7), pb.PF_ERR_SHAPE),
+    (dict(kernel=8), pb.PF_ERR_SHAPE),
+    (dict(kernel=pb.PF_ATTN_KERNEL_TWO_BLOCK, head_dim=64), pb.PF_ERR_SHAPE),
+    (dict(kernel=pb.PF_ATTN_KERNEL_TWO_BLOCK, stages=3), pb.PF_ERR_SHAPE),
+    (dict(kernel=pb.PF_ATTN_KERNEL_TWO_BLOCK, rows_per_cta=256), pb.PF_ERR_SHAPE),
+    (dict(kernel=pb.PF_ATTN_KERNEL_TWO_BLOCK, splits=17), pb.PF_ERR_SHAPE),
     (dict(kernel=pb.PF_ATTN_KERNEL_STREAM, splits=2), pb.PF_ERR_SHAPE),
     (dict(kernel=pb.PF_ATTN_KERNEL_BATCH, splits=2), pb.PF_ERR_SHAPE),
     (dict(kernel=pb.PF_ATTN_KERNEL_BATCH, head_dim=64), pb.PF_ERR_SHAPE),
@@ -345,8 +349,10 @@ def test_tree_prepare_device_rejects_bad_arguments(kw, status):
 
 
 def test_launch_fields_reach_the_library():
-    """The launch fields sit after the workspace in pf_attn_desc and the
-    stage request at the end of pf_lm_desc, as the header declares them."""
+    """The launch fields sit after the workspace in pf_attn_desc, followed by
+    the optional host copies of the lengths, and the stage request at the end
+    of pf_lm_desc, as the header declares them."""
     names = [f[0] for f in pb.pf_attn_desc._fields_]
-    assert names[-4:] == ["kernel", "splits", "rows_per_cta", "stages"]
+    assert names[-6:] == ["kernel", "splits", "rows_per_cta", "stages", "host_cu_nodes",
+                          "host_prefix_len"]
     assert [f[0] for f in pb.pf_lm_desc._fields_][-1] == "stages"

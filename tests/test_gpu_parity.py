@@ -9,7 +9,8 @@ import torch
 
 from paper_2609_32166_gb300 import binding as pb
 from paper_2609_32166_gb300 import inputs as I
-from tests.parity import Case
+from oracle import attention as OA
+from tests.parity import Case, values
 
 MMA = dict(kernel=pb.PF_ATTN_KERNEL_MMA)
 TC64 = dict(kernel=pb.PF_ATTN_KERNEL_TC64)
@@ -391,6 +392,111 @@ def test_128_token_tile_kernel_paged(stages):
         c.check_attention(0, s)
     c.check_lmhead(res)
     c.check_commit(res)
+
+
+# ---------------------------------------------------------------------------
+# two 128-row blocks per CTA on 128-token tiles (PF_ATTN_KERNEL_TWO_BLOCK):
+# K and V in separate ring units, each block's P written over its S columns
+# ---------------------------------------------------------------------------
+TWO_BLOCK = dict(kernel=pb.PF_ATTN_KERNEL_TWO_BLOCK)
+EDGE_2BLK = {k: EDGE[k] for k in ("root-only", "empty-prefix", "65-nodes", "g16-tiny-vocab",
+                                  "256-rows-paged", "two-blocks-one-tile")}
+
+
+@pytest.mark.parametrize("name", sorted(EDGE_2BLK))
+def test_two_block_128_kernel_edges(name):
+    """Root only (one row, block B empty), no prefix, two proposal tiles with
+    a prefix one row past a tile boundary, G = 16, 256 rows on a paged cache,
+    and 192 rows in one tile (the direct epilogue)."""
+    c = Case(EDGE_2BLK[name], seed=5, balanced=False, attn_launch=TWO_BLOCK)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for l in range(c.L):
+        for s in range(c.w.batch):
+            c.check_attention(l, s)
+    c.check_lmhead(res)
+    c.check_commit(res)
+
+
+@pytest.mark.parametrize("name", ["7b-tree64-small", "7b-32k-tree128-small",
+                                  "7b-batch8-paged-small"])
+def test_two_block_128_kernel(name):
+    """448 and 896 rows per KV head (two and four two-block CTAs per head),
+    and eight sequences of 224 rows on a paged cache whose shortest prefixes
+    leave some splits of a cluster without tiles."""
+    c = Case(SMALL[name], seed=12, balanced=False, attn_launch=TWO_BLOCK)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for l in range(c.L):
+        for s in range(c.w.batch):
+            c.check_attention(l, s)
+
+
+@pytest.mark.parametrize("host_lengths", ["given", "absent", "stale"])
+def test_two_block_128_kernel_teams(host_lengths):
+    """Eight sequences with prefixes from 100 to 1500 rows: with the host's
+    copies of the lengths (teams of a cluster's CTAs per group, sized by the
+    groups' tiles), without them (one group per cluster), and with copies
+    that disagree with the device arrays (a plan made for other lengths
+    still covers every tile once)."""
+    w = I.scaled(SMALL["7b-batch8-paged-small"], prefix=(100, 1500))
+    c = Case(w, seed=15, balanced=False, attn_launch=TWO_BLOCK)
+    if host_lengths == "absent":
+        for d in c.vs.attn_descs:
+            d.host_cu_nodes = d.host_prefix_len = None
+    elif host_lengths == "stale":
+        c.vs.h_prefix_len[:] = c.vs.h_prefix_len[::-1].copy()
+    c.vs.attention(0)
+    res = c.vs.results()
+    assert res["err"] == 0
+    for s in range(w.batch):
+        c.check_attention(0, s)
+
+
+@pytest.mark.parametrize("splits", [1, 2, 3, 4, 5, 6, 7, 8, 9, 16])
+def test_two_block_128_kernel_splits(splits):
+    """Every cluster width from one CTA (no merge) to 16 (wider than the
+    nine tiles: splits without tiles merge a zero partial)."""
+    c = Case(SMALL["7b-tree64-small"], seed=13, balanced=False,
+             attn_launch=dict(TWO_BLOCK, splits=splits))
+    c.vs.attention(0)
+    res = c.vs.results()
+    assert res["err"] == 0
+    c.check_attention(0, 0)
+
+
+@pytest.mark.parametrize("kernel", ["tc128", "two_block"])
+@pytest.mark.parametrize("layout", ["contiguous", "paged"])
+def test_growing_scores_rescale_the_accumulator(kernel, layout):
+    """Prefix keys scaled up along the sequence (x1 to x12), so that within a
+    split's six tiles the row maximum outgrows the running one by more than
+    the kernels' lazy rescale threshold (2^8) and the accumulated O and row
+    sum are rescaled; checked against the oracle on the same scaled keys."""
+    w = I.scaled(SMALL["7b-tree64-small"], layout=layout, prefix=(1500, 1500))
+    launch = dict({"tc128": TC128, "two_block": TWO_BLOCK}[kernel], splits=2)
+    c = Case(w, seed=14, balanced=False, attn_launch=launch)
+    b = c.batch
+    pk, pv = I.layer_prefix_kv(w, b, 0, 0)
+    P = pk.shape[1]
+    ramp = np.linspace(1.0, 12.0, P, dtype=np.float32)[None, :, None]
+    pk2 = I.round_to_bf16_bits(values(pk, "bf16") * ramp)
+    ck = np.zeros(I.cache_shape(w, b), dtype=np.uint16)
+    I.place_prefix(w, b, ck, 0, pk2)
+    c.vs.cache_k[0] = torch.from_numpy(ck.view(np.int16)).view(torch.bfloat16).to(
+        c.vs.cache_k.device)
+    c.vs.attention(0)
+    res = c.vs.results()
+    assert res["err"] == 0
+    c0, c1 = int(b.cu_nodes[0]), int(b.cu_nodes[1])
+    q = values(I.layer_q(w, b, 0), "bf16")[c0:c1]
+    tk, tv = (values(x, "bf16")[c0:c1] for x in I.layer_tree_kv(w, b, 0))
+    ref = OA.tree_attention(q, values(pk2, "bf16"), values(pv, "bf16"), tk, tv, b.parents[0])
+    got = c.vs.attn_out[0, c0:c1].float().cpu().numpy().astype(np.float64)
+    assert np.isfinite(got).all()
+    err = float(np.abs(got - ref).max())
+    assert err <= 2e-2, err
 
 
 @pytest.mark.parametrize("name", ["7b-tree64-small", "7b-32k-tree128-small"])

@@ -222,10 +222,13 @@ typedef struct pf_attn_desc {
  *          head) per CTA, so that each K/V tile enters the SM once for up
  *          to 256 query rows (KV heads with more than 128 rows: G x nodes);
  *          clusters split the tiles as for TC128
- * TC64, TC128, PAIR, STREAM, BATCH and TWO_BLOCK need bf16 and D = 128.  The automatic
- * choice is TC128 (128-row CTAs in clusters that split each row block's
- * tiles) where a CTA holds several 128-token tiles, TC64 otherwise, MMA for
- * other head sizes; it takes no workspace. */
+ * TC64, TC128, PAIR, STREAM, BATCH and TWO_BLOCK need bf16 and D = 128.
+ * The automatic choice takes no workspace: TWO_BLOCK with teams for a batch
+ * (B > 1) whose KV heads have more than 128 query rows, when host_cu_nodes
+ * and host_prefix_len are given and the team plan leaves each CTA at least
+ * four tiles; otherwise TC128 (128-row CTAs in clusters that split each row
+ * block's tiles) where a CTA holds several 128-token tiles, TC64 otherwise,
+ * MMA for other head sizes. */
 typedef enum pf_attn_kernel {
   PF_ATTN_KERNEL_AUTO = 0,
   PF_ATTN_KERNEL_MMA = 1,

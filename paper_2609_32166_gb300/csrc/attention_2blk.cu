@@ -365,45 +365,59 @@ __global__ void __launch_bounds__(kBThreads, 1)
         ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&s_full[x]), i & 1, a.err));
         if (!ok) break;  // warp-uniform
         tc_fence_after();
-        uint32_t sraw[kW];
-#pragma unroll
-        for (int c0 = 0; c0 < kW; c0 += 32)
-          tmem_ld_32(tmem + lane_base + col_s + c0, *reinterpret_cast<uint32_t(*)[32]>(&sraw[c0]));
-        tmem_ld_wait();
-        float sv[kW];
-#pragma unroll
-        for (int c = 0; c < kW; ++c) sv[c] = __uint_as_float(sraw[c]);
-
         const int t = tile_at(i);
         const bool is_prefix = t < n_ptiles;
         const int valid = is_prefix ? min(kW, P - t * kW) : kW;
-        if (!is_prefix || valid < kW) {
-          // masked tile: prefix columns past the end, or proposal columns
-          // that are not ancestors of this row's node (columns 0..63 are
-          // nodes 0..63, columns 64..127 nodes 64..127)
-          uint64_t v0, v1;
-          if (is_prefix) {
-            v0 = valid >= 64 ? ~0ull : ((1ull << valid) - 1ull);
-            v1 = valid >= 128 ? ~0ull : (valid <= 64 ? 0ull : ((1ull << (valid - 64)) - 1ull));
-          } else {
-            v0 = mk0;
-            v1 = mk1;
-          }
-#pragma unroll
-          for (int c = 0; c < 64; ++c) {
-            if (!((v0 >> c) & 1ull)) sv[c] = -INFINITY;
-            if (!((v1 >> c) & 1ull)) sv[64 + c] = -INFINITY;
-          }
+        // masked tile: prefix columns past the end, or proposal columns that
+        // are not ancestors of this row's node (columns 0..63 are nodes
+        // 0..63, columns 64..127 nodes 64..127)
+        const bool masked = !is_prefix || valid < kW;
+        uint64_t vm[2] = {mk0, mk1};
+        if (is_prefix) {
+          vm[0] = valid >= 64 ? ~0ull : ((1ull << valid) - 1ull);
+          vm[1] = valid >= 128 ? ~0ull : (valid <= 64 ? 0ull : ((1ull << (valid - 64)) - 1ull));
         }
+        // The scores are read from TMEM twice, 64 columns at a time (the row
+        // maximum, then P), so that no more than 64 of them are in registers:
+        // a thread of this 10-warp CTA has 168.  A masked tile's first pass
+        // writes the masked scores back, so the second needs no mask.
+        auto load_half = [&](int h, float (&sv)[64]) {
+          uint32_t sr[64];
+          tmem_ld_32(tmem + lane_base + col_s + 64 * h, *reinterpret_cast<uint32_t(*)[32]>(&sr[0]));
+          tmem_ld_32(tmem + lane_base + col_s + 64 * h + 32,
+                     *reinterpret_cast<uint32_t(*)[32]>(&sr[32]));
+          tmem_ld_wait();
+#pragma unroll
+          for (int c = 0; c < 64; ++c) sv[c] = __uint_as_float(sr[c]);
+        };
         // row maximum of the raw scores (scale > 0 commutes with max): eight
-        // running three-input maxima, few registers beside the 128 scores
+        // running three-input maxima
         float m8[8];
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          m8[k] = fmax3(sv[k], sv[8 + k], sv[16 + k]);
+        for (int h = 0; h < 2; ++h) {
+          float sv[64];
+          load_half(h, sv);
+          if (masked) {
+            uint64_t v = vm[h];
+            uint32_t sm[64];
 #pragma unroll
-          for (int j = 3; j < 15; j += 2) m8[k] = fmax3(m8[k], sv[8 * j + k], sv[8 * j + 8 + k]);
-          m8[k] = fmaxf(m8[k], sv[120 + k]);
+            for (int c = 0; c < 64; ++c) {
+              if (!(v & 1ull)) sv[c] = -INFINITY;
+              v >>= 1;
+              sm[c] = __float_as_uint(sv[c]);
+            }
+            tmem_st_32(tmem + lane_base + col_s + 64 * h, *reinterpret_cast<uint32_t(*)[32]>(&sm[0]));
+            tmem_st_32(tmem + lane_base + col_s + 64 * h + 32,
+                       *reinterpret_cast<uint32_t(*)[32]>(&sm[32]));
+            tmem_st_wait();
+          }
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            float m = h ? fmax3(m8[k], sv[k], sv[8 + k]) : fmaxf(sv[k], sv[8 + k]);
+#pragma unroll
+            for (int j = 2; j < 8; j += 2) m = fmax3(m, sv[8 * j + k], sv[8 * j + 8 + k]);
+            m8[k] = m;
+          }
         }
         const float mx =
             fmax3(fmax3(m8[0], m8[1], m8[2]), fmax3(m8[3], m8[4], m8[5]), fmaxf(m8[6], m8[7])) *
@@ -419,26 +433,31 @@ __global__ void __launch_bounds__(kBThreads, 1)
           m_ref = m_new;
         }
         // p = 2^(s * scale_log2 - m): one paired FMA per two scores, one MUFU
-        // per score; the row sum in four paired accumulators
+        // per score; the row sum in four paired accumulators.  P_X goes over
+        // the S_X columns this thread has read: half h into columns
+        // 32 h .. 32 h + 31, once that half's scores are in registers.
         const float neg_mu = m_ref == -INFINITY ? 0.f : -m_ref;
         const unsigned long long sc2 = f32x2_pack(a.scale_log2, a.scale_log2);
         const unsigned long long mu2 = f32x2_pack(neg_mu, neg_mu);
         unsigned long long rs2[4] = {0ull, 0ull, 0ull, 0ull};
-        uint32_t pk[kW / 2];
 #pragma unroll
-        for (int c = 0; c < kW / 2; ++c) {
-          float x0, x1;
-          f32x2_unpack(ffma2(f32x2_pack(sv[2 * c], sv[2 * c + 1]), sc2, mu2), x0, x1);
-          const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
-          rs2[c & 3] = fadd2(rs2[c & 3], f32x2_pack(p0, p1));
-          pk[c] = pack_bf16(p0, p1);
+        for (int h = 0; h < 2; ++h) {
+          float sv[64];
+          load_half(h, sv);
+          uint32_t pk[32];
+#pragma unroll
+          for (int c = 0; c < 32; ++c) {
+            float x0, x1;
+            f32x2_unpack(ffma2(f32x2_pack(sv[2 * c], sv[2 * c + 1]), sc2, mu2), x0, x1);
+            const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+            rs2[c & 3] = fadd2(rs2[c & 3], f32x2_pack(p0, p1));
+            pk[c] = pack_bf16(p0, p1);
+          }
+          tmem_st_32(tmem + lane_base + col_s + 32 * h, pk);
         }
         float r0, r1;
         f32x2_unpack(fadd2(fadd2(rs2[0], rs2[1]), fadd2(rs2[2], rs2[3])), r0, r1);
         l += r0 + r1;
-        // P_X over the S_X columns this thread has read
-        tmem_st_32(tmem + lane_base + col_s, *reinterpret_cast<uint32_t(*)[32]>(&pk[0]));
-        tmem_st_32(tmem + lane_base + col_s + 32, *reinterpret_cast<uint32_t(*)[32]>(&pk[32]));
         tmem_st_wait();
         if (any_resc) {
           // O_X *= alpha before PV_X(i) adds this tile (after the scores and

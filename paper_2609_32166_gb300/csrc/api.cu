@@ -195,8 +195,8 @@ struct AttnChoice {
 // cluster).  A cluster's spare CTAs then join its team with the most tiles
 // per CTA.  Used only where X is below the one-group clusters' tiles per CTA
 // (`uniform_splits` CTAs per group).
-bool make_team_plan(pf::AttnArgs& a, const int32_t* hcu, const int32_t* hP, int sms,
-                    int uniform_splits, pf::TeamPlan* tp, int* tiles_per_cta = nullptr) {
+bool plan_teams(pf::AttnArgs& a, const int32_t* hcu, const int32_t* hP, int sms,
+                int uniform_splits, pf::TeamPlan* tp, int* tiles_per_cta) {
   struct Grp {
     int id, t;
   };
@@ -280,6 +280,56 @@ bool make_team_plan(pf::AttnArgs& a, const int32_t* hcu, const int32_t* hP, int 
   a.splits = s;
   a.team_ctas = used * s;
   if (tiles_per_cta) *tiles_per_cta = best_x;
+  return true;
+}
+
+// plan_teams behind a one-entry cache: the calls of one verify step (every
+// layer) and the size queries share the same lengths and shape, so the plan
+// is made once per step.
+bool make_team_plan(pf::AttnArgs& a, const int32_t* hcu, const int32_t* hP, int sms,
+                    int uniform_splits, pf::TeamPlan* tp, int* tiles_per_cta = nullptr) {
+  struct Entry {
+    bool valid = false, ok = false;
+    int dev = -1, B = 0, Hkv = 0, rb_count = 0, nb = 0, max_nodes = 0, max_prefix = 0, sms = 0,
+        uniform = 0;
+    std::vector<int32_t> cu, P;
+    pf::TeamPlan tp;
+    int splits = 0, team_ctas = 0, per_cta = 0;
+  };
+  static std::mutex mu;
+  static Entry e;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  std::lock_guard<std::mutex> lock(mu);
+  const bool hit = e.valid && e.dev == dev && e.B == a.B && e.Hkv == a.Hkv &&
+                   e.rb_count == a.rb_count && e.nb == a.nb && e.max_nodes == a.max_nodes &&
+                   e.max_prefix == a.max_prefix && e.sms == sms && e.uniform == uniform_splits &&
+                   std::memcmp(e.cu.data(), hcu, sizeof(int32_t) * (a.B + 1)) == 0 &&
+                   std::memcmp(e.P.data(), hP, sizeof(int32_t) * a.B) == 0;
+  if (!hit) {
+    pf::AttnArgs t = a;
+    e.ok = plan_teams(t, hcu, hP, sms, uniform_splits, &e.tp, &e.per_cta);
+    e.splits = t.splits;
+    e.team_ctas = t.team_ctas;
+    e.valid = true;
+    e.dev = dev;
+    e.B = a.B;
+    e.Hkv = a.Hkv;
+    e.rb_count = a.rb_count;
+    e.nb = a.nb;
+    e.max_nodes = a.max_nodes;
+    e.max_prefix = a.max_prefix;
+    e.sms = sms;
+    e.uniform = uniform_splits;
+    e.cu.assign(hcu, hcu + a.B + 1);
+    e.P.assign(hP, hP + a.B);
+  }
+  if (!e.ok) return false;
+  *tp = e.tp;
+  a.team = 1;
+  a.splits = e.splits;
+  a.team_ctas = e.team_ctas;
+  if (tiles_per_cta) *tiles_per_cta = e.per_cta;
   return true;
 }
 

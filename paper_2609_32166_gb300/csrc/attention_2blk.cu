@@ -556,7 +556,8 @@ __global__ void __launch_bounds__(kBThreads, 1)
   // ---- split-KV merge: each row's normalised partial and its
   // log2-sum-exp are staged in the idle ring, one bulk copy per peer moves
   // the rows it merges into its inbox (behind the staged rows), and every
-  // CTA merges its own rows from its inbox.
+  // CTA merges its own rows from its inbox.  A CTA's partials of the rows it
+  // merges itself are staged straight into its own inbox slots.
   // (the group's pieces: CTAs base .. base + nparts - 1 of the cluster)
   const int per = (rows + nparts - 1) / nparts;
   const int cnt_mine = max(0, min(per, rows - part * per));
@@ -566,10 +567,13 @@ __global__ void __launch_bounds__(kBThreads, 1)
   __syncthreads();
   cluster_arrive_release();
   if (tid == 0)
-    mbar_arrive_expect_tx(smem_u32(inbox_full), (uint32_t)(nparts * cnt_mine * S::kRowBytes));
+    mbar_arrive_expect_tx(smem_u32(inbox_full),
+                          (uint32_t)((nparts - 1) * cnt_mine * S::kRowBytes));
   if (has_row) {
     // O in two 64-column halves (a whole row beside the rest would spill)
-    __half* dst = stage_rows + min(r, 255) * S::kPitch;
+    // (own rows: inbox slot part * per + i is CTA row r itself)
+    const bool own = r >= part * per && r < part * per + cnt_mine;
+    __half* dst = (own ? sInbox : stage_rows) + min(r, 255) * S::kPitch;
     // no column reached this row in this split (a split without tiles never
     // writes O): its partial is 0 with lse = -inf, whatever the unwritten
     // accumulator holds (0 * NaN would poison the merge)
@@ -603,7 +607,7 @@ __global__ void __launch_bounds__(kBThreads, 1)
   if (tid < nparts) {
     const int q = tid;
     const int cnt = min(per, rows - q * per);
-    if (cnt > 0) {
+    if (cnt > 0 && q != part) {
       const uint32_t src = smem_u32(stage_rows + q * per * S::kPitch);
       const uint32_t dst = mapa_cluster(smem_u32(sInbox + part * per * S::kPitch), base + q);
       bulk_copy_s2cluster(dst, src, (uint32_t)(cnt * S::kRowBytes),

@@ -276,6 +276,39 @@ PF_API size_t pf_verify_attention_workspace_size(const pf_attn_desc* d);
  * rejected.  Host-only: no device work, the last error is left alone. */
 PF_API int32_t pf_verify_attention_launches(const pf_attn_desc* d);
 
+/* pf_verify_attention_team_plan -- the team plan that PF_ATTN_KERNEL_TWO_BLOCK
+ * makes from host copies of the lengths (see host_cu_nodes above), for
+ * inspection and host-side tests.  Host-only: no device work, the last error
+ * is left alone.
+ *   cu_nodes[batch + 1], prefix_len[batch]   host arrays, read only
+ *   n_kv_heads, group (query heads per KV head, 1..128), max_nodes,
+ *   max_prefix_len     as in pf_attn_desc (bf16, head_dim 128)
+ *   num_sms            SMs the launch may use (>= 1)
+ *   max_clusters       [17] or NULL: max_clusters[s] = how many clusters of s
+ *                      CTAs of the kernel fit on the GPU at once (NULL: the
+ *                      current device's figures, which needs a GPU)
+ *   uniform_splits     CTAs per group of the one-group clusters to beat
+ *   entries            [PF_TEAM_MAX_CTAS] out, one word per CTA: group |
+ *                      piece << 12 | pieces << 17 | rank of the team's first
+ *                      CTA in its cluster << 22 (pieces = 0: no work), group =
+ *                      (sequence * n_kv_heads + KV head) * pairs + pair of
+ *                      row blocks, pairs = ceil(max_nodes / (2 * floor(128 /
+ *                      group)))
+ *   cluster_size, ctas, tiles_per_cta   out: CTAs per cluster, CTAs of the
+ *                      launch (a multiple of it), the longest piece in tiles
+ * Returns 1 with the plan written, 0 where no team plan beats the one-group
+ * clusters or the lengths contradict the bounds, -1 for a NULL pointer or a
+ * size out of range. */
+#define PF_TEAM_MAX_CTAS 160
+PF_API int32_t pf_verify_attention_team_plan(const int32_t* cu_nodes,
+                                             const int32_t* prefix_len, int32_t batch,
+                                             int32_t n_kv_heads, int32_t group,
+                                             int32_t max_nodes, int32_t max_prefix_len,
+                                             int32_t num_sms, const int32_t* max_clusters,
+                                             int32_t uniform_splits, uint32_t* entries,
+                                             int32_t* cluster_size, int32_t* ctas,
+                                             int32_t* tiles_per_cta);
+
 PF_API pf_status pf_verify_attention(const pf_attn_desc* d, void* stream);
 
 /*

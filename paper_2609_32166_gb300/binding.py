@@ -152,6 +152,9 @@ def lib() -> C.CDLL:
     L.pf_verify_attention_workspace_size.argtypes = [C.POINTER(pf_attn_desc)]
     L.pf_verify_attention_launches.restype = C.c_int32
     L.pf_verify_attention_launches.argtypes = [C.POINTER(pf_attn_desc)]
+    L.pf_verify_attention_team_plan.restype = C.c_int32
+    L.pf_verify_attention_team_plan.argtypes = [C.c_void_p, C.c_void_p] + [C.c_int32] * 6 + [
+        C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]
     L.pf_lmhead_accept_workspace_size.restype = C.c_size_t
     L.pf_lmhead_accept_workspace_size.argtypes = [C.POINTER(pf_lm_desc)]
     L.pf_lmhead_accept.restype = C.c_int
@@ -236,6 +239,27 @@ def pf_verify_attention_workspace_size(desc: pf_attn_desc) -> int:
 
 def pf_verify_attention_launches(desc: pf_attn_desc) -> int:
     return int(lib().pf_verify_attention_launches(C.byref(desc)))
+
+
+PF_TEAM_MAX_CTAS = 160
+
+
+def pf_verify_attention_team_plan(cu_nodes, prefix_len, n_kv_heads: int, group: int,
+                                  max_nodes: int, max_prefix_len: int, num_sms: int,
+                                  max_clusters, uniform_splits: int):
+    """The two-block kernel's team plan for host lengths: (status, entries
+    [PF_TEAM_MAX_CTAS] uint32, cluster size, CTAs, longest piece in tiles)."""
+    import numpy as np
+    cu = np.ascontiguousarray(cu_nodes, dtype=np.int32)
+    pl = np.ascontiguousarray(prefix_len, dtype=np.int32)
+    mc = None if max_clusters is None else np.ascontiguousarray(max_clusters, dtype=np.int32)
+    entries = np.zeros(PF_TEAM_MAX_CTAS, dtype=np.uint32)
+    out = np.zeros(3, dtype=np.int32)
+    st = lib().pf_verify_attention_team_plan(
+        cu.ctypes.data, pl.ctypes.data, len(pl), n_kv_heads, group, max_nodes, max_prefix_len,
+        num_sms, None if mc is None else mc.ctypes.data, uniform_splits, entries.ctypes.data,
+        out[0:].ctypes.data, out[1:].ctypes.data, out[2:].ctypes.data)
+    return int(st), entries, int(out[0]), int(out[1]), int(out[2])
 
 
 def pf_verify_attention(desc: pf_attn_desc, stream: int = 0) -> None:

@@ -196,7 +196,8 @@ struct AttnChoice {
 // per CTA.  Used only where X is below the one-group clusters' tiles per CTA
 // (`uniform_splits` CTAs per group).
 bool plan_teams(pf::AttnArgs& a, const int32_t* hcu, const int32_t* hP, int sms,
-                int uniform_splits, pf::TeamPlan* tp, int* tiles_per_cta) {
+                int uniform_splits, pf::TeamPlan* tp, int* tiles_per_cta,
+                const int32_t* fits = nullptr) {
   struct Grp {
     int id, t;
   };
@@ -220,7 +221,8 @@ bool plan_teams(pf::AttnArgs& a, const int32_t* hcu, const int32_t* hP, int sms,
   std::vector<int> best_k, best_c;
   std::vector<int> k(G), cl(G);
   for (int s = 2; s <= 16; s += 2) {
-    const int C = std::min(std::min(max_active_clusters(4, s), sms / s), pf::kTeamMaxCtas / s);
+    const int C = std::min(std::min(fits ? (int)fits[s] : max_active_clusters(4, s), sms / s),
+                           pf::kTeamMaxCtas / s);
     if (C < 1) continue;
     const long long lo_total = (total + (long long)C * s - 1) / ((long long)C * s);
     const int lo = std::max((int)lo_total, (gs[0].t + s - 1) / s);
@@ -708,6 +710,40 @@ size_t pf_verify_attention_workspace_size(const pf_attn_desc* d) {
                   choose_attention(d, a, sms, true, &ch, "") == PF_OK;
   g_last_error = saved;
   return ok ? ch.ws_need : 0;
+}
+
+int32_t pf_verify_attention_team_plan(const int32_t* cu_nodes, const int32_t* prefix_len,
+                                      int32_t batch, int32_t n_kv_heads, int32_t group,
+                                      int32_t max_nodes, int32_t max_prefix_len, int32_t sms_count,
+                                      const int32_t* max_clusters, int32_t uniform_splits,
+                                      uint32_t* entries, int32_t* cluster_size, int32_t* ctas,
+                                      int32_t* tiles_per_cta) {
+  static_assert(PF_TEAM_MAX_CTAS == pf::kTeamMaxCtas, "team plan size");
+  if (!cu_nodes || !prefix_len || !entries || !cluster_size || !ctas || !tiles_per_cta) return -1;
+  if (batch < 1 || n_kv_heads < 1 || group < 1 || group > 128 || max_nodes < 1 ||
+      max_nodes > PF_MAX_NODES || max_prefix_len < 0 || sms_count < 1 || uniform_splits < 1)
+    return -1;
+  if (!max_clusters && num_sms() <= 0) return -1;  // the device's figures need a GPU
+  pf::AttnArgs a = {};
+  a.B = batch;
+  a.Hkv = n_kv_heads;
+  a.G = group;
+  a.max_nodes = max_nodes;
+  a.max_prefix = max_prefix_len;
+  a.nb = 2 * (128 / group);
+  a.rb_count = (max_nodes + a.nb - 1) / a.nb;
+  pf::TeamPlan tp;
+  int per_cta = 0;
+  const std::string saved = g_last_error;
+  const bool ok = plan_teams(a, cu_nodes, prefix_len, sms_count, uniform_splits, &tp, &per_cta,
+                             max_clusters);
+  g_last_error = saved;
+  if (!ok) return 0;
+  std::memcpy(entries, tp.e, sizeof(tp.e));
+  *cluster_size = a.splits;
+  *ctas = a.team_ctas;
+  *tiles_per_cta = per_cta;
+  return 1;
 }
 
 int32_t pf_verify_attention_launches(const pf_attn_desc* d) {

@@ -262,15 +262,22 @@ bool plan_teams(pf::AttnArgs& a, const int32_t* hcu, const int32_t* hP, int sms,
     }
   }
   if (best_s == 0) return false;
-  // number the used clusters, lay each one's teams out from rank 0
+  // Number the used clusters by their longest piece, longest first: CTAs
+  // start as the preceding kernel's CTAs leave, the lowest-numbered first,
+  // so the last to start get the shortest pieces.  Each cluster's teams are
+  // laid out from rank 0.
   const int s = best_s;
-  std::vector<int> cidx(pf::kTeamMaxCtas, -1), next_rank;
-  int used = 0;
-  for (int j = 0; j < G; ++j)
-    if (cidx[best_c[j]] < 0) {
-      cidx[best_c[j]] = used++;
-      next_rank.push_back(0);
-    }
+  std::vector<int> longest(pf::kTeamMaxCtas, 0), order;
+  for (int j = 0; j < G; ++j) {
+    const int c = best_c[j];
+    if (longest[c] == 0) order.push_back(c);
+    longest[c] = std::max(longest[c], (gs[j].t + best_k[j] - 1) / best_k[j]);
+  }
+  std::stable_sort(order.begin(), order.end(),
+                   [&](int x, int y) { return longest[x] > longest[y]; });
+  std::vector<int> cidx(pf::kTeamMaxCtas, -1), next_rank(order.size(), 0);
+  const int used = (int)order.size();
+  for (int i = 0; i < used; ++i) cidx[order[i]] = i;
   for (int i = 0; i < pf::kTeamMaxCtas; ++i) tp->e[i] = pf::team_entry(0, 0, 0, 0);
   for (int j = 0; j < G; ++j) {
     const int c = cidx[best_c[j]], base = next_rank[c];

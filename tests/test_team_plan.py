@@ -5,8 +5,9 @@ Checked on random batches: every (sequence, KV head, pair of row blocks)
 group that holds nodes is one team of consecutive CTAs inside one cluster,
 its pieces 0..k-1 each exactly once at cluster ranks base..base+k-1; no
 other group appears; the launch is whole clusters, no more than fit and no
-more CTAs than SMs; the reported longest piece is the plan's and beats the
-one-group clusters it was asked to beat."""
+more CTAs than SMs, numbered longest piece first; the reported longest
+piece is the plan's and beats the one-group clusters it was asked to
+beat."""
 import math
 
 import numpy as np
@@ -63,11 +64,16 @@ def check_plan(cu, P, hkv, G, max_nodes, max_prefix, sms, table, uniform):
         longest = max(longest, math.ceil(want[g] / t["k"]))
     assert span == longest
     assert span < math.ceil(max(want.values()) / uniform)
-    # no cluster holds more CTAs than it has
-    used = {}
-    for t in teams.values():
-        used[t["cluster"]] = used.get(t["cluster"], 0) + t["k"]
+    # no cluster holds more CTAs than it has; every cluster of the launch
+    # holds a team; clusters come longest piece first (they start in order)
+    used, piece = {}, {}
+    for g, t in teams.items():
+        c = t["cluster"]
+        used[c] = used.get(c, 0) + t["k"]
+        piece[c] = max(piece.get(c, 0), math.ceil(want[g] / t["k"]))
     assert all(v <= s for v in used.values())
+    assert sorted(used) == list(range(ctas // s))
+    assert all(piece[c] >= piece[c + 1] for c in range(ctas // s - 1))
     return s, ctas, span
 
 

@@ -164,3 +164,25 @@ def test_input_arena_is_blocked_by_layer():
     assert vs.q[1].data_ptr() - base == segs[1][0]  # a piece starts at its first layer's block
     assert vs.hidden.data_ptr() - base >= segs[-1][0]
     assert vs.tokens.data_ptr() - base < segs[0][1]
+
+
+def test_attention_descriptors_carry_host_copies_of_the_lengths():
+    """Every layer's attention descriptor points at the step's own host
+    copies of cu_nodes and prefix_len (the two-block kernel's team plan is
+    made from them): equal to the batch's lengths, and copies, so that
+    changing them leaves the batch -- and the oracle that reads it -- alone."""
+    import ctypes as C
+    import numpy as np
+    from paper_2609_32166_gb300.step import VerifyStep
+    w = inputs.scaled(inputs.WORKLOADS["7b-bf16-batch8-paged"], layers=2, prefix=(40, 100),
+                      vocab=300, hidden=64, batch=3)
+    batch = inputs.make_batch(w, 0)
+    vs = VerifyStep(w, batch, np.zeros(batch.total_nodes, np.int32), device="cpu")
+    B = w.batch
+    for d in vs.attn_descs:
+        cu = np.ctypeslib.as_array(C.cast(d.host_cu_nodes, C.POINTER(C.c_int32)), (B + 1,))
+        pl = np.ctypeslib.as_array(C.cast(d.host_prefix_len, C.POINTER(C.c_int32)), (B,))
+        assert np.array_equal(cu, batch.cu_nodes) and np.array_equal(pl, batch.prefix_lens)
+    before = batch.prefix_lens.copy()
+    vs.h_prefix_len[:] = vs.h_prefix_len[::-1].copy()
+    assert np.array_equal(batch.prefix_lens, before)

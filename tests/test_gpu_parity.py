@@ -499,6 +499,26 @@ def test_growing_scores_rescale_the_accumulator(kernel, layout):
     assert err <= 2e-2, err
 
 
+@pytest.mark.parametrize("kernel", ["auto", "two_block"])
+@pytest.mark.parametrize("nodes", [2, 17, 63, 64, 127])
+def test_node_count_sweep(nodes, kernel):
+    """Proposal sizes around the 64- and 128-token tile edges (1, 9, 65 and
+    128 nodes are among the edge cases), two sequences with prefixes of 448
+    and 515 rows (a multiple of 64 but not of 128; a multiple of neither),
+    every node and head, then the LM head, acceptance and commit."""
+    w = I.scaled(W["7b-bf16-tree64"], layers=1, batch=2, prefix=(333, 517), nodes=nodes,
+                 max_depth=min(nodes - 1, 12), vocab=700, hidden=128)
+    launch = None if kernel == "auto" else TWO_BLOCK
+    c = Case(w, seed=16, balanced=False, attn_launch=launch)
+    c.vs.step()
+    res = c.vs.results()
+    assert res["err"] == 0
+    for s in range(w.batch):
+        c.check_attention(0, s)
+    c.check_lmhead(res)
+    c.check_commit(res)
+
+
 @pytest.mark.parametrize("name", ["7b-tree64-small", "7b-32k-tree128-small"])
 def test_two_block_kernel_on_many_rows(name):
     """Two 128-row blocks per CTA (64-token kernel, rows_per_cta = 256) where

@@ -125,3 +125,25 @@ def test_rejects_inconsistent_lengths_and_bad_arguments():
                                             GB300_LIKE, 2)[0] == -1
     assert pb.pf_verify_attention_team_plan(cu, [100, 100], 2, 7, 10, 100, 0,
                                             GB300_LIKE, 2)[0] == -1
+
+
+def test_null_pointers_and_the_device_figures():
+    """NULL arrays are rejected; without a cluster-fit table the figures come
+    from the current device, so without a GPU the call is refused."""
+    import torch
+    L = pb.lib()
+    entries = np.zeros(pb.PF_TEAM_MAX_CTAS, np.uint32)
+    out = np.zeros(3, np.int32)
+    cu = np.array([0, 10, 20], np.int32)
+    P = np.array([300, 900], np.int32)
+    args = [cu.ctypes.data, P.ctypes.data, 2, 4, 7, 10, 900, 152, None, 2, entries.ctypes.data,
+            out[0:].ctypes.data, out[1:].ctypes.data, out[2:].ctypes.data]
+    for i in (0, 1, 10, 11, 12, 13):
+        bad = list(args)
+        bad[i] = None
+        assert L.pf_verify_attention_team_plan(*bad) == -1
+    st = L.pf_verify_attention_team_plan(*args)
+    if torch.cuda.is_available():
+        assert st in (0, 1)
+    else:
+        assert st == -1
